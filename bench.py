@@ -1,0 +1,470 @@
+"""Benchmark of the depth-attention mix hot path (Low-Rank Attention Residuals).
+
+Workload (one step): every residual read site t = 1..49 of a 24-layer PreNorm
+decoder with S-LR-AttnRes keys (last r = 16 of d = 1024 coordinates), T = 16384
+tokens (batch 8 x sequence 2048), bf16 storage, fp32 accumulation.  A step is
+the forward sweep (site t mixes the first t sources of the stacked buffer) and
+the backward sweep t = 49..1, which writes (site 49) and then accumulates
+(sites 48..1) the source gradients, as a training step does.  Inputs are
+synthetic (normal values with a per-source scale, N(0, 0.02^2) queries, normal
+upstream gradients), drawn on the device with a seeded generator.
+
+Metric: algorithmic HBM bytes of the step / step time (GB/s), the fraction of
+the measured HBM copy peak, and tokens/s per site.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 (launched by torch.distributed.run) every rank runs its own replica
+of the workload on its own GPU (independent token batches, no exchange: weak
+scaling); the reported value is all ranks' bytes over the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "depth-residual fwd+bwd GB/s and % of GB300 HBM peak; tokens/sec per site"
+T_TOK, D, R, N_SITES, SEED, EPS = 16384, 1024, 16, 49, 1, 1e-6
+WORKLOAD = ("S-LR-AttnRes fwd+bwd at every residual site (n_src = 1..49) of a 24-layer decoder: "
+            "T=16384 (8 x 2048), d=1024, r=16, bf16 storage, fp32 accumulate")
+FALLBACK_HBM_GBS = 6800.0
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def _kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2607_09694_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def _recorded_traffic(kernel: str):
+    """Bytes per launch from a committed ncu summary, if it was taken on the
+    current kernel sources (the summary records their hash)."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    fields = {}
+    with open(path) as f:
+        for line in f:
+            if ":" in line and not line.startswith("#"):
+                k, v = line.split(":", 1)
+                fields[k.strip()] = v.strip()
+    if fields.get("source_hash") != _kernel_source_hash():
+        return None
+    try:
+        return float(fields["dram_bytes_per_launch_avg"])
+    except (KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines: list[str] = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, flag in zip(names, parts[5:9]):
+                if flag.lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------
+# The workload
+# --------------------------------------------------------------------------
+
+
+def site_bytes():
+    """Algorithmic bytes of each forward and backward call of one step."""
+    from paper_2607_09694_gb300 import sites
+
+    fwd = [sites.forward_bytes(sites.SiteShape("sliced", t, T_TOK, D, R)) for t in range(1, N_SITES + 1)]
+    bwd = [sites.backward_bytes(sites.SiteShape("sliced", t, T_TOK, D, R, accumulate=0 if t == N_SITES else 1))
+           for t in range(1, N_SITES + 1)]
+    return fwd, bwd
+
+
+class Workload:
+    def __init__(self, device, T=T_TOK):
+        import torch
+
+        from paper_2607_09694_gb300 import lrar, synth
+
+        self.torch, self.lrar = torch, lrar
+        self.dev = device
+        self.T = T
+        self.values = synth.values(N_SITES, T, D, SEED, "bf16", (0.5, 2.0), device=device)
+        self.queries = synth.queries(N_SITES, R, SEED, device=device)      # row t-1: query of site t
+        self.dh = synth.upstream(T, D, SEED, "bf16", sites=N_SITES, device=device)  # row t-1: dL/dh_t
+        self.h = torch.empty(N_SITES, T, D, dtype=torch.bfloat16, device=device)
+        self.lse = torch.empty(N_SITES, T, dtype=torch.float32, device=device)
+        self.dvalues = torch.empty(N_SITES, T, D, dtype=torch.bfloat16, device=device)
+        self.dq = torch.empty(N_SITES, R, dtype=torch.float32, device=device)
+        self.ws = torch.empty(lrar.workspace_size("sliced", N_SITES, T, D, R) // 4, dtype=torch.float32,
+                              device=device)
+
+    def step(self, events=None):
+        """Forward sweep t = 1..49, then backward sweep t = 49..1 (49 writes, the rest accumulate)."""
+        lrar = self.lrar
+        for t in range(1, N_SITES + 1):
+            q = self.queries[t - 1] if t > 1 else None
+            if events is not None:
+                events["fwd"][t - 1][0].record()
+            lrar.forward(lrar.SLICED, self.values, None, q, self.h[t - 1], self.lse[t - 1], n_src=t, r=R, eps=EPS)
+            if events is not None:
+                events["fwd"][t - 1][1].record()
+        for t in range(N_SITES, 0, -1):
+            q = self.queries[t - 1] if t > 1 else None
+            if events is not None:
+                events["bwd"][t - 1][0].record()
+            lrar.backward(lrar.SLICED, self.values, None, q, self.dh[t - 1], self.dvalues, self.dq[t - 1], self.ws,
+                          n_src=t, r=R, accumulate=(t != N_SITES), eps=EPS)
+            if events is not None:
+                events["bwd"][t - 1][1].record()
+
+    @staticmethod
+    def launches_per_step() -> int:
+        return N_SITES + 2 * N_SITES  # forward kernel; backward kernel + dq reduction
+
+
+def _events(torch):
+    mk = lambda: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))  # noqa: E731
+    return {"fwd": [mk() for _ in range(N_SITES)], "bwd": [mk() for _ in range(N_SITES)]}
+
+
+# --------------------------------------------------------------------------
+# CPU oracle baseline (bounded sample)
+# --------------------------------------------------------------------------
+
+
+def oracle_pass(values_cpu, queries_cpu, dh_cpu, ts: int) -> float:
+    """Seconds the fp64 oracle takes for all 49 sites (fwd + bwd) on the first ts tokens."""
+    import oracle
+
+    v = values_cpu[:, :ts].contiguous()
+    d = dh_cpu[:, :ts].contiguous()
+    q0 = queries_cpu[0] * 0
+    t0 = time.perf_counter()
+    for t in range(1, N_SITES + 1):
+        q = queries_cpu[t - 1] if t > 1 else q0
+        oracle.forward(oracle.SLICED, v[:t], None, q, EPS, r=R)
+        oracle.backward(oracle.SLICED, v[:t], None, q, EPS, d[t - 1], r=R)
+    return time.perf_counter() - t0
+
+
+def sample_bytes(ts: int) -> int:
+    from paper_2607_09694_gb300 import sites
+
+    nbytes = 0
+    for t in range(1, N_SITES + 1):
+        nbytes += sites.forward_bytes(sites.SiteShape("sliced", t, ts, D, R))
+        nbytes += sites.backward_bytes(sites.SiteShape("sliced", t, ts, D, R, accumulate=0 if t == N_SITES else 1))
+    return nbytes
+
+
+def calibrate(values_cpu, queries_cpu, dh_cpu, target_s: float) -> int:
+    """Token count whose oracle pass takes about target_s seconds (capped by the sample held)."""
+    import oracle
+
+    oracle.build()
+    probe = min(32, values_cpu.shape[1])
+    per_tok = oracle_pass(values_cpu, queries_cpu, dh_cpu, probe) / probe
+    ts = int(target_s / max(per_tok, 1e-9))
+    return max(probe, min(values_cpu.shape[1], ts))
+
+
+def oracle_sample(values_cpu, queries_cpu, dh_cpu, target_s: float):
+    """(GB/s on the sample's algorithmic bytes, seconds, tokens, threads) of one timed oracle pass."""
+    import oracle
+
+    ts = calibrate(values_cpu, queries_cpu, dh_cpu, target_s)
+    el = oracle_pass(values_cpu, queries_cpu, dh_cpu, ts)
+    return sample_bytes(ts) / el / 1e9, el, ts, oracle.get_threads()
+
+
+# --------------------------------------------------------------------------
+
+
+def _dist():
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group("nccl" if _cuda() else "gloo")
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return dist if world > 1 else None, rank, local, world
+
+
+def _cuda() -> bool:
+    import torch
+
+    return torch.cuda.is_available()
+
+
+def _max_over_ranks(dist, value: float, device) -> float:
+    if dist is None:
+        return value
+    import torch
+
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def run_ours(args):
+    import torch
+
+    from __graft_entry__ import build
+
+    dist, rank, local, world = _dist()
+    build()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    peak, peak_kind = _peaks()
+    fwd_b, bwd_b = site_bytes()
+    step_bytes = sum(fwd_b) + sum(bwd_b)
+
+    wl = Workload(dev)
+    for _ in range(args.warmup):
+        wl.step()
+    torch.cuda.synchronize()
+
+    # device-resident timed region
+    ev = [_events(torch) for _ in range(args.steps)]
+    clocks = ClockSampler(torch.cuda.current_device())
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for k in range(args.steps):
+        wl.step(ev[k])
+    t1.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if dist:
+        dist.barrier()
+    elapsed = _max_over_ranks(dist, t0.elapsed_time(t1) / 1e3, dev)
+    ms_step = elapsed / args.steps * 1e3
+    value = world * step_bytes * args.steps / elapsed / 1e9
+
+    fwd_t = [sum(e["fwd"][i][0].elapsed_time(e["fwd"][i][1]) for e in ev) / args.steps for i in range(N_SITES)]
+    bwd_t = [sum(e["bwd"][i][0].elapsed_time(e["bwd"][i][1]) for e in ev) / args.steps for i in range(N_SITES)]
+    bwd_gbs = sum(bwd_b) / (sum(bwd_t) / 1e3) / 1e9
+    fwd_gbs = sum(fwd_b) / (sum(fwd_t) / 1e3) / 1e9
+    dominant, dom_gbs, dom_bytes, dom_launches = ("lrar_bwd", bwd_gbs, sum(bwd_b), N_SITES) \
+        if sum(bwd_t) >= sum(fwd_t) else ("lrar_fwd", fwd_gbs, sum(fwd_b), N_SITES)
+    traffic = _recorded_traffic(dominant)
+    site49 = {"n_src": 49, "fwd_ms": fwd_t[-1], "bwd_ms": bwd_t[-1],
+              "fwd_gbs": fwd_b[-1] / (fwd_t[-1] / 1e3) / 1e9, "bwd_gbs": bwd_b[-1] / (bwd_t[-1] / 1e3) / 1e9,
+              "fwd_bwd_gbs": (fwd_b[-1] + bwd_b[-1]) / ((fwd_t[-1] + bwd_t[-1]) / 1e3) / 1e9}
+    site49["frac"] = site49["fwd_bwd_gbs"] / peak
+    site49["tokens_per_s"] = T_TOK / ((fwd_t[-1] + bwd_t[-1]) / 1e3)
+
+    # end to end through the public API with host buffers
+    e2e = run_e2e(wl, args, dist, dev, step_bytes, world)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        vals = wl.values[:, :4096].cpu()
+        qs = wl.queries.cpu()
+        dhs = wl.dh[:, :4096].cpu()
+        gbs, secs, ts, cores = oracle_sample(vals, qs, dhs, args.cpu_seconds)
+        cpu = {"value": gbs, "unit": "GB/s", "cores": cores, "kind": "oracle",
+               "sample": f"all 49 sites fwd+bwd on {ts} of {T_TOK} tokens ({secs:.1f} s, fp64 C oracle, "
+                         f"OpenMP {cores} threads); GB/s on the sample's algorithmic bytes"}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "T": T_TOK, "d": D, "r": R, "sites": N_SITES, "variant": "sliced",
+                   "storage": "bf16", "accumulate": "f32", "parallelism": f"replicas{world}",
+                   "l2": "inputs larger than L2 (1.64 GB of values per step, L2 129 MB)",
+                   "bytes_per_step": step_bytes},
+        "hbm_frac": value / world / peak,
+        "tokens_per_s_per_site": world * T_TOK * N_SITES / (elapsed / args.steps),
+        "site49": site49,
+        "roofline": {"bound": "hbm", "achieved": dom_gbs, "peak": peak, "unit": "GB/s",
+                     "frac": dom_gbs / peak, "traffic": traffic, "kernel": dominant,
+                     "algorithmic_bytes_per_launch": dom_bytes / dom_launches,
+                     "peak_source": f"{peak_kind} hbm_gbs (copy bandwidth)",
+                     "fwd_gbs": fwd_gbs, "bwd_gbs": bwd_gbs},
+        "e2e": e2e,
+        "gpu_launches": Workload.launches_per_step() * args.steps,
+        "clocks": clk,
+    }
+    if cpu is not None:
+        line["cpu_baseline"] = cpu
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def run_e2e(wl, args, dist, dev, step_bytes, world):
+    """The step through the public API with pinned host inputs: H2D of values,
+    queries and upstream gradients, both sweeps, D2H of h, lse, dvalues, dq."""
+    import torch
+
+    hv = torch.empty_like(wl.values, device="cpu").pin_memory()
+    hq = torch.empty_like(wl.queries, device="cpu").pin_memory()
+    hdh = torch.empty_like(wl.dh, device="cpu").pin_memory()
+    hv.copy_(wl.values)
+    hq.copy_(wl.queries)
+    hdh.copy_(wl.dh)
+    oh = torch.empty_like(wl.h, device="cpu").pin_memory()
+    olse = torch.empty_like(wl.lse, device="cpu").pin_memory()
+    odv = torch.empty_like(wl.dvalues, device="cpu").pin_memory()
+    odq = torch.empty_like(wl.dq, device="cpu").pin_memory()
+    h2d = sum(x.numel() * x.element_size() for x in (hv, hq, hdh))
+    d2h = sum(x.numel() * x.element_size() for x in (oh, olse, odv, odq))
+
+    def one():
+        wl.values.copy_(hv, non_blocking=True)
+        wl.queries.copy_(hq, non_blocking=True)
+        wl.dh.copy_(hdh, non_blocking=True)
+        wl.step()
+        oh.copy_(wl.h, non_blocking=True)
+        olse.copy_(wl.lse, non_blocking=True)
+        odv.copy_(wl.dvalues, non_blocking=True)
+        odq.copy_(wl.dq, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        one()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    s = torch.cuda.Event(enable_timing=True)
+    e = torch.cuda.Event(enable_timing=True)
+    s.record()
+    for _ in range(args.steps):
+        one()
+    e.record()
+    torch.cuda.synchronize()
+    el = _max_over_ranks(dist, s.elapsed_time(e) / 1e3, dev)
+    return {"value": world * step_bytes * args.steps / el / 1e9, "unit": "GB/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": el / args.steps * 1e3}
+
+
+def run_reference(args):
+    """The fp64 CPU oracle on the same workload's config (rank 0 only): each
+    step is a bounded sample (all 49 sites on a slice of tokens)."""
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if rank != 0:
+        return
+    import oracle
+    from paper_2607_09694_gb300 import synth
+
+    ts_max = 2048
+    vals = synth.values(N_SITES, ts_max, D, SEED, "bf16", (0.5, 2.0))
+    qs = synth.queries(N_SITES, R, SEED)
+    dhs = synth.upstream(ts_max, D, SEED, "bf16", sites=N_SITES)
+    ts = calibrate(vals, qs, dhs, args.ref_step_seconds)
+    for _ in range(args.warmup):
+        oracle_pass(vals, qs, dhs, ts)
+    secs = [oracle_pass(vals, qs, dhs, ts) for _ in range(args.steps)]
+    total = sum(secs)
+    value = sample_bytes(ts) * args.steps / total / 1e9
+    cores = oracle.get_threads()
+    sample = (f"all 49 sites fwd+bwd on {ts} of {T_TOK} tokens per step (fp64 C oracle, OpenMP {cores} threads); "
+              f"GB/s on the sample's algorithmic bytes")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": total / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "T": T_TOK, "d": D, "r": R, "sites": N_SITES, "variant": "sliced",
+                       "sample_tokens": ts},
+            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target length of the CPU oracle sample")
+    ap.add_argument("--ref-step-seconds", type=float, default=4.0, help="target length of one reference step")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,156 @@
+/*
+ * lrar.h -- C ABI of liblrar.so, the GB300 (sm_103a) depth-attention mix of
+ * "Low-Rank Attention Residuals" (arxiv 2607.09694).
+ *
+ * At a residual read site every token x mixes the outputs of earlier
+ * sub-layers ("sources") i = 0..n_src-1 with a softmax over depth:
+ *
+ *   kbar_i = RMSNorm(k_i)            Eq. (8),  parameter-free (App. A.5)
+ *   alpha_i = softmax_i(q . kbar_i)  Eq. (9),  static per-site query q
+ *   h = sum_i alpha_i o_i            Eq. (10), full-width values
+ *
+ * where the routing key k_i is
+ *   LRAR_PROJECTED  a learned r-dim key from the output projection (§3.3, Eq. 12),
+ *   LRAR_SLICED     the last r coordinates of o_i (§3.4, Eq. 14),
+ *   LRAR_FULL       o_i itself with r = d, i.e. standard AttnRes (§3.1, Eq. 2).
+ *
+ * RMSNorm is k / sqrt(mean_j k_j^2 + eps); eps is an argument because the
+ * paper does not state it.  Scores carry no temperature.
+ *
+ * Layout (all row-major, all device memory owned by the caller):
+ *   values  [n_src, T, d]   source-major stack of sub-layer outputs
+ *   keys    [n_src, T, r]   P-LR keys (LRAR_PROJECTED only)
+ *   query   [r] float32     (r = d for LRAR_FULL)
+ *   h, dh   [T, d]          mixed output and its upstream gradient
+ *   lse     [T] float32     log sum_i exp(score_i), saved by the forward
+ *
+ * Conventions shared by every entry point:
+ *   - Calls are asynchronous and ordered on `stream` (a cudaStream_t; NULL is
+ *     the legacy default stream).  No call synchronises the host, allocates
+ *     memory or keeps state between calls; the library is thread-safe.
+ *   - Return value: LRAR_OK (0) or a negative LRAR_ERR_* code.  Argument
+ *     checks run before anything is launched; on error nothing is launched and
+ *     outputs are untouched.  lrar_last_error() gives a message for the
+ *     calling thread's most recent failure.
+ *   - Tensor pointers must be 16-byte aligned (query, lse and dq: 4-byte),
+ *     and d * sizeof(input element) must be a multiple of 16 bytes
+ *     (LRAR_ERR_ALIGNMENT otherwise).
+ *   - Element types: LRAR_F32 or LRAR_BF16; arithmetic is float32 throughout
+ *     and every bfloat16 store rounds to nearest even.
+ */
+#ifndef LRAR_H
+#define LRAR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define LRAR_VERSION 1
+#define LRAR_MAX_SOURCES 128
+
+enum lrar_variant { LRAR_FULL = 0, LRAR_SLICED = 1, LRAR_PROJECTED = 2 };
+enum lrar_dtype { LRAR_F32 = 0, LRAR_BF16 = 1 };
+enum lrar_status {
+    LRAR_OK = 0,
+    LRAR_ERR_INVALID_ARG = -1, /* null required pointer, bad enum, n_src < 1, r < 1, r > d,
+                                  FULL with r != d, T < 0, eps <= 0 or not finite */
+    LRAR_ERR_ALIGNMENT = -2,   /* pointer not 16-byte aligned or row size not a multiple of 16 bytes */
+    LRAR_ERR_UNSUPPORTED = -3, /* n_src > LRAR_MAX_SOURCES, d beyond the kernel's width limit */
+    LRAR_ERR_CUDA = -4,        /* a CUDA call or launch failed; lrar_last_error() has its text */
+    LRAR_ERR_WORKSPACE = -5    /* workspace NULL or smaller than lrar_backward_workspace_size() */
+};
+
+/*
+ * Forward mix at one residual site: Eq. (8)-(10) for all T tokens.
+ *
+ *   variant   LRAR_FULL / LRAR_SLICED / LRAR_PROJECTED
+ *   in_dtype  element type of values and keys
+ *   out_dtype element type of h
+ *   values    [n_src, T, d] in_dtype, read only
+ *   keys      [n_src, T, r] in_dtype, read only; LRAR_PROJECTED only, ignored otherwise
+ *   query     [r] float32; may be NULL only when n_src == 1 (the softmax is then 1)
+ *   n_src     number of sources, 1..LRAR_MAX_SOURCES (site t of Full AttnRes has t)
+ *   T         tokens (batch x sequence); T == 0 is a no-op
+ *   d, r      value width and key width; r == d for LRAR_FULL
+ *             (d <= 2048 for bfloat16 input, <= 1024 for float32)
+ *   eps       RMSNorm epsilon, > 0
+ *   h         [T, d] out_dtype, written
+ *   lse       [T] float32, written when non-NULL (LRAR_FULL's backward needs it)
+ *   stream    cudaStream_t
+ */
+int lrar_forward(int variant, int in_dtype, int out_dtype, const void *values, const void *keys,
+                 const float *query, int n_src, int64_t T, int d, int r, float eps, void *h, float *lse,
+                 void *stream);
+
+/*
+ * Bytes of device workspace lrar_backward needs: the per-CTA partial sums of
+ * dq, reduced in a fixed order so that dq is bitwise reproducible.  Depends
+ * only on the arguments (not on the device).
+ */
+size_t lrar_backward_workspace_size(int variant, int n_src, int64_t T, int d, int r);
+
+/*
+ * Backward of lrar_forward: gradients of a loss L given dh = dL/dh.
+ * The paper prints no gradient formulas; these are the chain rule through
+ * Eq. (8)-(10):
+ *   g_i = <dh, o_i>,  gbar = sum_i alpha_i g_i,  ds_i = alpha_i (g_i - gbar)
+ *   dL/do_i  = alpha_i dh  (+ the key gradient where the key lives in o_i)
+ *   dL/dk_i  = ds_i rho_i (q - (s_i / r) kbar_i),  rho_i = 1/sqrt(mean k_i^2 + eps)
+ *   dL/dq    = sum over tokens and sources of ds_i kbar_i
+ * SLICED adds dL/dk_i into the last r coordinates of dvalues; FULL adds it to
+ * all of dvalues; PROJECTED writes it to dkeys.
+ *
+ *   in_dtype   element type of values, keys and dh
+ *   grad_dtype element type of dvalues and dkeys
+ *   dh         [T, d] in_dtype
+ *   h          [T, d] h_dtype, the forward output; required for LRAR_FULL
+ *              (gbar = <dh, h> lets FULL finish in one pass), ignored otherwise
+ *   h_dtype    element type of h
+ *   lse        [T] float32 from the forward; required for LRAR_FULL, ignored otherwise
+ *   dvalues    [n_src, T, d] grad_dtype, written (accumulate = 0) or added into
+ *   dkeys      [n_src, T, r] grad_dtype; LRAR_PROJECTED only, same accumulate rule
+ *   dq         [r] float32, written or added into; summed over all T tokens
+ *   accumulate 0: overwrite dvalues/dkeys/dq; 1: add into them (a source
+ *              receives gradient from every later site)
+ *   workspace  device scratch of at least lrar_backward_workspace_size() bytes,
+ *              16-byte aligned; contents on entry are ignored
+ *   Other arguments as for lrar_forward.  values, dvalues and dkeys must not overlap.
+ */
+int lrar_backward(int variant, int in_dtype, int grad_dtype, const void *values, const void *keys,
+                  const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh,
+                  const void *h, int h_dtype, const float *lse, void *dvalues, void *dkeys, float *dq,
+                  int accumulate, void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * Block AttnRes source assembly (§3.1, Eq. 5-6) and its gradient fan-out:
+ *   dst[e] = beta * dst[e] + alpha * src[e]   for e = 0..count-1
+ * beta == 0 does not read dst (opens a new block summary: dst = alpha * src).
+ * After sub-layer j writes o_j, `dst = partial summary slot, src = o_j, beta = 1`
+ * extends the partial block; in the backward `dst = d(o_j), src = d(slot)`
+ * hands each member its summary's gradient.  For P-LR the same call sums keys
+ * (the paper does not define a summary's key; this library reads it as the
+ * sum of the members' keys).
+ *   dst_dtype, src_dtype  element types (may differ, e.g. float32 summaries of
+ *                         bfloat16 outputs)
+ *   count                 elements (T * width); 0 is a no-op
+ */
+int lrar_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *src, int64_t count,
+                          float alpha, float beta, void *stream);
+
+/* Static text for a status code. */
+const char *lrar_strerror(int code);
+
+/* Message of the calling thread's most recent failed call ("" if none). */
+const char *lrar_last_error(void);
+
+/* LRAR_VERSION of the built library. */
+int lrar_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LRAR_H */

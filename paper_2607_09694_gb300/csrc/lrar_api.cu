@@ -1,0 +1,234 @@
+// lrar_api.cu -- the exported C ABI of liblrar.so (declared in include/lrar.h):
+// argument checks, error reporting, and dispatch to the kernel launchers.
+// Nothing here allocates device memory or synchronises the host.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <mutex>
+#include <unordered_map>
+
+#include "lrar.h"
+#include "lrar_device.cuh"
+#include "lrar_launch.h"
+
+#define LRAR_API extern "C" __attribute__((visibility("default")))
+
+namespace {
+
+thread_local char g_last_error[512] = "";
+
+int fail(int code, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_last_error, sizeof g_last_error, fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char *where) {
+    return fail(LRAR_ERR_CUDA, "%s: %s (%s)", where, cudaGetErrorString(e), cudaGetErrorName(e));
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+bool aligned4(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 3) == 0; }
+bool dtype_ok(int t) { return t == LRAR_F32 || t == LRAR_BF16; }
+int esize(int t) { return t == LRAR_BF16 ? 2 : 4; }
+
+// Scalar checks shared by forward and backward.
+int check_shape(int variant, int in_dtype, int n_src, int64_t T, int d, int r, float eps) {
+    if (variant < LRAR_FULL || variant > LRAR_PROJECTED) return fail(LRAR_ERR_INVALID_ARG, "unknown variant %d", variant);
+    if (!dtype_ok(in_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown input dtype %d", in_dtype);
+    if (n_src < 1) return fail(LRAR_ERR_INVALID_ARG, "n_src must be >= 1 (got %d)", n_src);
+    if (n_src > LRAR_MAX_SOURCES)
+        return fail(LRAR_ERR_UNSUPPORTED, "n_src %d exceeds LRAR_MAX_SOURCES (%d)", n_src, LRAR_MAX_SOURCES);
+    if (T < 0) return fail(LRAR_ERR_INVALID_ARG, "T must be >= 0");
+    if (d < 1 || r < 1 || r > d) return fail(LRAR_ERR_INVALID_ARG, "need 1 <= r <= d (got d=%d r=%d)", d, r);
+    if (variant == LRAR_FULL && r != d)
+        return fail(LRAR_ERR_INVALID_ARG, "full AttnRes keys need r == d (got d=%d r=%d)", d, r);
+    if (!(eps > 0.f) || !isfinite(eps)) return fail(LRAR_ERR_INVALID_ARG, "eps must be finite and > 0");
+    if ((d * esize(in_dtype)) % 16) return fail(LRAR_ERR_ALIGNMENT, "d * element size must be a multiple of 16 bytes");
+    if (d > lrar::max_width(in_dtype))
+        return fail(LRAR_ERR_UNSUPPORTED, "d=%d exceeds the kernel width limit %d", d, lrar::max_width(in_dtype));
+    return LRAR_OK;
+}
+
+struct OccKey {
+    const void *k;
+    int dev, threads;
+    size_t smem;
+    bool operator==(const OccKey &o) const {
+        return k == o.k && dev == o.dev && threads == o.threads && smem == o.smem;
+    }
+};
+struct OccHash {
+    size_t operator()(const OccKey &o) const {
+        return std::hash<const void *>()(o.k) ^ (std::hash<size_t>()(o.smem) * 31) ^ (size_t)o.dev * 131 ^
+               (size_t)o.threads;
+    }
+};
+std::mutex g_occ_mu;
+std::unordered_map<OccKey, int, OccHash> g_occ;  // (kernel, device, block, smem) -> resident CTAs per SM x SMs
+
+}  // namespace
+
+namespace lrar {
+
+int max_width(int in_dtype) { return 32 * 8 * VecE<float>::value * (in_dtype == LRAR_BF16 ? 2 : 1); }
+
+int persistent_grid(const void *kernel, int threads, size_t smem, int64_t work_ctas, int cap) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    OccKey key{kernel, dev, threads, smem};
+    int slots = 0;
+    {
+        std::lock_guard<std::mutex> lk(g_occ_mu);
+        auto it = g_occ.find(key);
+        if (it != g_occ.end()) slots = it->second;
+    }
+    if (slots == 0) {
+        int sms = 0, occ = 0;
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kernel, threads, smem);
+        slots = (sms > 0 ? sms : 1) * (occ > 0 ? occ : 1);
+        std::lock_guard<std::mutex> lk(g_occ_mu);
+        g_occ[key] = slots;
+    }
+    int64_t g = slots;
+    if (g > work_ctas) g = work_ctas;
+    if (g > cap) g = cap;
+    if (g < 1) g = 1;
+    return (int)g;
+}
+
+}  // namespace lrar
+
+LRAR_API int lrar_version(void) { return LRAR_VERSION; }
+
+LRAR_API const char *lrar_last_error(void) { return g_last_error; }
+
+LRAR_API const char *lrar_strerror(int code) {
+    switch (code) {
+        case LRAR_OK: return "success";
+        case LRAR_ERR_INVALID_ARG: return "invalid argument";
+        case LRAR_ERR_ALIGNMENT: return "misaligned pointer or row size";
+        case LRAR_ERR_UNSUPPORTED: return "unsupported size";
+        case LRAR_ERR_CUDA: return "CUDA error";
+        case LRAR_ERR_WORKSPACE: return "workspace missing or too small";
+        default: return "unknown status code";
+    }
+}
+
+LRAR_API int lrar_forward(int variant, int in_dtype, int out_dtype, const void *values, const void *keys,
+                          const float *query, int n_src, int64_t T, int d, int r, float eps, void *h, float *lse,
+                          void *stream) {
+    int rc = check_shape(variant, in_dtype, n_src, T, d, r, eps);
+    if (rc) return rc;
+    if (!dtype_ok(out_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown output dtype %d", out_dtype);
+    if (T == 0) return LRAR_OK;
+    if (!values || !h) return fail(LRAR_ERR_INVALID_ARG, "values and h are required");
+    if (variant == LRAR_PROJECTED && !keys) return fail(LRAR_ERR_INVALID_ARG, "projected keys are required");
+    if (!query && n_src > 1) return fail(LRAR_ERR_INVALID_ARG, "query is required when n_src > 1");
+    if (!aligned16(values) || !aligned16(h) || (variant == LRAR_PROJECTED && !aligned16(keys)) ||
+        (query && !aligned4(query)) || (lse && !aligned4(lse)))
+        return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (query and lse 4-byte)");
+    lrar::FwdArgs a;
+    a.variant = variant;
+    a.in_dtype = in_dtype;
+    a.out_dtype = out_dtype;
+    a.values = values;
+    a.keys = variant == LRAR_PROJECTED ? keys : nullptr;
+    a.query = query;
+    a.n = n_src;
+    a.T = T;
+    a.d = d;
+    a.r = r;
+    a.eps = eps;
+    a.h = h;
+    a.lse = lse;
+    cudaError_t e = lrar::launch_forward(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "lrar_forward");
+    return LRAR_OK;
+}
+
+LRAR_API size_t lrar_backward_workspace_size(int variant, int n_src, int64_t T, int d, int r) {
+    (void)n_src;
+    (void)T;
+    const int rq = variant == LRAR_FULL ? d : r;
+    if (rq < 1) return 0;
+    return sizeof(float) * (size_t)lrar::kMaxPartials * (size_t)rq;
+}
+
+LRAR_API int lrar_backward(int variant, int in_dtype, int grad_dtype, const void *values, const void *keys,
+                           const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh,
+                           const void *h, int h_dtype, const float *lse, void *dvalues, void *dkeys, float *dq,
+                           int accumulate, void *workspace, size_t workspace_bytes, void *stream) {
+    int rc = check_shape(variant, in_dtype, n_src, T, d, r, eps);
+    if (rc) return rc;
+    if (!dtype_ok(grad_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown gradient dtype %d", grad_dtype);
+    if (accumulate != 0 && accumulate != 1) return fail(LRAR_ERR_INVALID_ARG, "accumulate must be 0 or 1");
+    if (variant == LRAR_FULL && !dtype_ok(h_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown h dtype %d", h_dtype);
+    if (!dq) return fail(LRAR_ERR_INVALID_ARG, "dq is required");
+    const int rq = variant == LRAR_FULL ? d : r;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (T == 0) {  // dq is a sum over no tokens
+        if (!accumulate) {
+            cudaError_t e = cudaMemsetAsync(dq, 0, sizeof(float) * (size_t)rq, s);
+            if (e != cudaSuccess) return cuda_fail(e, "lrar_backward");
+        }
+        return LRAR_OK;
+    }
+    if (!values || !dh || !dvalues) return fail(LRAR_ERR_INVALID_ARG, "values, dh and dvalues are required");
+    if (variant == LRAR_PROJECTED && (!keys || !dkeys))
+        return fail(LRAR_ERR_INVALID_ARG, "projected keys and dkeys are required");
+    if (variant == LRAR_FULL && (!h || !lse))
+        return fail(LRAR_ERR_INVALID_ARG, "full AttnRes backward needs the forward's h and lse");
+    if (!query && n_src > 1) return fail(LRAR_ERR_INVALID_ARG, "query is required when n_src > 1");
+    if (!aligned16(values) || !aligned16(dh) || !aligned16(dvalues) || !aligned4(dq) ||
+        (variant == LRAR_PROJECTED && (!aligned16(keys) || !aligned16(dkeys))) ||
+        (variant == LRAR_FULL && (!aligned16(h) || !aligned4(lse))) || (query && !aligned4(query)))
+        return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (query, lse and dq 4-byte)");
+    if (!workspace || workspace_bytes < lrar_backward_workspace_size(variant, n_src, T, d, r))
+        return fail(LRAR_ERR_WORKSPACE, "workspace needs %zu bytes (got %zu)",
+                    lrar_backward_workspace_size(variant, n_src, T, d, r), workspace ? workspace_bytes : (size_t)0);
+    if (!aligned16(workspace)) return fail(LRAR_ERR_ALIGNMENT, "workspace must be 16-byte aligned");
+    lrar::BwdArgs a;
+    a.variant = variant;
+    a.in_dtype = in_dtype;
+    a.grad_dtype = grad_dtype;
+    a.h_dtype = h_dtype;
+    a.values = values;
+    a.keys = variant == LRAR_PROJECTED ? keys : nullptr;
+    a.query = query;
+    a.n = n_src;
+    a.T = T;
+    a.d = d;
+    a.r = r;
+    a.eps = eps;
+    a.dh = dh;
+    a.h = variant == LRAR_FULL ? h : nullptr;
+    a.lse = variant == LRAR_FULL ? lse : nullptr;
+    a.dvalues = dvalues;
+    a.dkeys = variant == LRAR_PROJECTED ? dkeys : nullptr;
+    a.dq = dq;
+    a.accumulate = accumulate;
+    a.partials = static_cast<float *>(workspace);
+    cudaError_t e = lrar::launch_backward(a, s);
+    if (e != cudaSuccess) return cuda_fail(e, "lrar_backward");
+    return LRAR_OK;
+}
+
+LRAR_API int lrar_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *src, int64_t count,
+                                   float alpha, float beta, void *stream) {
+    if (!dtype_ok(dst_dtype) || !dtype_ok(src_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown dtype");
+    if (count < 0) return fail(LRAR_ERR_INVALID_ARG, "count must be >= 0");
+    if (!isfinite(alpha) || !isfinite(beta)) return fail(LRAR_ERR_INVALID_ARG, "alpha and beta must be finite");
+    if (count == 0) return LRAR_OK;
+    if (!dst || !src) return fail(LRAR_ERR_INVALID_ARG, "dst and src are required");
+    if ((reinterpret_cast<uintptr_t>(dst) % esize(dst_dtype)) || (reinterpret_cast<uintptr_t>(src) % esize(src_dtype)))
+        return fail(LRAR_ERR_ALIGNMENT, "dst and src must be aligned to their element size");
+    cudaError_t e = lrar::launch_block_accumulate(dst_dtype, dst, src_dtype, src, count, alpha, beta,
+                                                  static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "lrar_block_accumulate");
+    return LRAR_OK;
+}

@@ -1,0 +1,574 @@
+// lrar_bwd.cu -- backward of the depth-attention mix (chain rule through
+// Eq. 8-10 of arxiv 2607.09694; the paper prints no gradient formulas):
+//
+//   g_i = <dh, o_i>,  gbar = sum_i alpha_i g_i,  ds_i = alpha_i (g_i - gbar)
+//   dL/do_i = alpha_i dh,   dL/dq = sum ds_i kbar_i
+//   dL/dk_i = ds_i rho_i (q - (s_i / r) kbar_i),   rho_i = (mean k_i^2 + eps)^-1/2
+//
+// Every value row is read once and every gradient row written once.
+//
+// Low-rank keys: (1) the routing stage recomputes s, rho, alpha from the r-dim
+// keys; (2) the value pass streams o_i, forms g_i with a warp reduction and
+// writes dL/do_i = alpha_i dh (+ the old value when accumulating) for every
+// 16-byte vector that does not lie wholly in the key slice; (3) the key pass,
+// with gbar known, forms ds_i and dL/dk_i lane-per-key-coordinate, writes the
+// key slice of dvalues (SLICED: alpha_i dh + dL/dk_i in one rounding) or dkeys
+// (PROJECTED), and accumulates dq.
+//
+// Full keys (r = d): ds_i needs gbar before row i can be written, and gbar =
+// <dh, h> because h = sum_i alpha_i o_i, so a single pass needs the forward's
+// h and lse: per row, three warp reductions (g_i, |o_i|^2, q.o_i) give s_i,
+// rho_i, alpha_i = exp(s_i - lse), ds_i, and the whole gradient row
+//   alpha_i dh + ds_i rho_i q - ds_i rho_i^2 (s_i / d) o_i.
+//
+// dq: each warp accumulates its tokens, each CTA writes one partial row to the
+// workspace, and a second kernel sums the partials in CTA order, so dq is
+// bitwise reproducible on a given device.
+#include "lrar_device.cuh"
+#include "lrar_launch.h"
+
+namespace lrar {
+
+struct BwdParams {
+    const void *values, *keys, *dh, *h;
+    const float *query, *lse;
+    void *dvalues, *dkeys;
+    float *partials;
+    int64_t T;
+    int n, d, r;
+    float eps, inv_r;
+    int sliced, key_vec, accumulate, h_bf16;
+};
+
+// Routing stage, identical arithmetic to the forward's (see lrar_fwd.cu).
+template <typename Tin>
+__device__ __forceinline__ void key_stats_b(const Tin *__restrict__ kp, int r, const float *__restrict__ q_s,
+                                            bool vec, float &ss, float &qk) {
+    ss = 0.f;
+    qk = 0.f;
+    if (vec) {
+        constexpr int E = VecE<Tin>::value;
+        for (int j = 0; j < r; j += E) {
+            Frag<Tin, E> f;
+            f.load_nc(kp + j);
+            float k[E];
+            f.get(k);
+#pragma unroll
+            for (int t = 0; t < E; ++t) {
+                ss = fmaf(k[t], k[t], ss);
+                qk = fmaf(q_s[j + t], k[t], qk);
+            }
+        }
+    } else {
+        for (int j = 0; j < r; ++j) {
+            const float k = to_f(__ldg(kp + j));
+            ss = fmaf(k, k, ss);
+            qk = fmaf(q_s[j], k, qk);
+        }
+    }
+}
+
+template <typename Tin>
+__device__ __forceinline__ void lr_route_b(const BwdParams &p, const Tin *__restrict__ values,
+                                           const Tin *__restrict__ keys, int64_t x, int lane,
+                                           const float *__restrict__ q_s, float *a_s, float *s_s, float *rho_s) {
+    float s_reg[kSrcRegs];
+    float m = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < kSrcRegs; ++k) {
+        const int i = lane + 32 * k;
+        float s = -INFINITY;
+        if (i < p.n) {
+            const Tin *kp = p.sliced ? values + ((int64_t)i * p.T + x) * p.d + (p.d - p.r)
+                                     : keys + ((int64_t)i * p.T + x) * p.r;
+            float ss, qk;
+            key_stats_b<Tin>(kp, p.r, q_s, p.key_vec != 0, ss, qk);
+            const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
+            s = rho * qk;
+            s_s[i] = s;
+            rho_s[i] = rho;
+        }
+        s_reg[k] = s;
+        m = fmaxf(m, s);
+    }
+    m = warp_max(m);
+    float z = 0.f;
+#pragma unroll
+    for (int k = 0; k < kSrcRegs; ++k) {
+        const int i = lane + 32 * k;
+        const float e = (i < p.n) ? expf(s_reg[k] - m) : 0.f;
+        s_reg[k] = e;
+        z += e;
+    }
+    z = warp_sum(z);
+    const float inv_z = 1.f / z;
+#pragma unroll
+    for (int k = 0; k < kSrcRegs; ++k) {
+        const int i = lane + 32 * k;
+        if (i < p.n) a_s[i] = s_reg[k] * inv_z;
+    }
+}
+
+// One value row of the low-rank backward (phase 2): returns the lane's part of g_i.
+template <typename Tin, typename Tg, int V>
+__device__ __forceinline__ float lr_bwd_row(const Frag<Tin, VecE<Tin>::value> *f,
+                                            const Frag<Tg, VecE<Tin>::value> *old, const float *dhf, float a,
+                                            Tg *__restrict__ drow, int skip0, int lane, int accumulate) {
+    constexpr int E = VecE<Tin>::value;
+    float gp = 0.f;
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+        const int e = (lane + 32 * v) * E;
+        float o[E];
+        f[v].get(o);
+#pragma unroll
+        for (int t = 0; t < E; ++t) gp = fmaf(dhf[v * E + t], o[t], gp);
+        if (e < skip0) {  // vectors wholly inside the key slice are written by the key pass
+            float w[E];
+            if (accumulate) old[v].get(w);
+            else
+#pragma unroll
+                for (int t = 0; t < E; ++t) w[t] = 0.f;
+#pragma unroll
+            for (int t = 0; t < E; ++t) w[t] = fmaf(a, dhf[v * E + t], w[t]);
+            Frag<Tg, E> out;
+            out.set(w);
+            out.store(drow + e);
+        }
+    }
+    return gp;
+}
+
+template <typename Tin, typename Tg, int V, int U>
+__global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(const BwdParams p) {
+    constexpr int E = VecE<Tin>::value;
+    extern __shared__ float smem[];
+    const int rp = round_up(p.r, 4);
+    float *q_s = smem;                                   // [r]
+    float *dq_all = q_s + rp;                            // [kWarps][r]
+    float *tab = dq_all + kWarps * rp;                   // [kWarps][4][kMaxSources]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    float *dq_s = dq_all + warp * rp;
+    float *a_s = tab + warp * 4 * kMaxSources;
+    float *s_s = a_s + kMaxSources;
+    float *rho_s = s_s + kMaxSources;
+    float *g_s = rho_s + kMaxSources;  // g_i, then ds_i
+    for (int j = threadIdx.x; j < p.r; j += kThreads) q_s[j] = p.query ? p.query[j] : 0.f;
+    for (int j = threadIdx.x; j < kWarps * rp; j += kThreads) dq_all[j] = 0.f;
+    __syncthreads();
+
+    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
+    const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
+    const Tin *__restrict__ dh = static_cast<const Tin *>(p.dh);
+    Tg *__restrict__ dvalues = static_cast<Tg *>(p.dvalues);
+    Tg *__restrict__ dkeys = static_cast<Tg *>(p.dkeys);
+    const int64_t src_stride = p.T * (int64_t)p.d;
+    const int64_t key_stride = p.T * (int64_t)p.r;
+    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+    const int tail0 = p.sliced ? p.d - p.r : p.d;  // first key coordinate inside the value row
+    const int skip0 = round_up(tail0, E);          // vectors starting here lie wholly in the key slice
+
+    for (int64_t x = (int64_t)blockIdx.x * kWarps + warp; x < p.T; x += nwarps) {
+        // (1) routing: s_i, rho_i, alpha_i
+        lr_route_b<Tin>(p, values, keys, x, lane, q_s, a_s, s_s, rho_s);
+        __syncwarp();
+
+        // (2) value pass
+        float dhf[V * E];
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int e = (lane + 32 * v) * E;
+            Frag<Tin, E> f;
+            if (e < p.d) f.load_nc(dh + x * p.d + e);
+            else f.zero();
+            f.get(dhf + v * E);
+        }
+        const int64_t row_off = x * p.d;
+        int i = 0;
+        for (; i + U <= p.n; i += U) {
+            Frag<Tin, E> f[U][V];
+            Frag<Tg, E> old[U][V];
+#pragma unroll
+            for (int u = 0; u < U; ++u)
+#pragma unroll
+                for (int v = 0; v < V; ++v) {
+                    const int e = (lane + 32 * v) * E;
+                    const int64_t off = (int64_t)(i + u) * src_stride + row_off + e;
+                    if (e < p.d) f[u][v].load_nc(values + off);
+                    else f[u][v].zero();
+                    if (p.accumulate && e < skip0) old[u][v].load(dvalues + off);
+                    else old[u][v].zero();
+                }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const float gp = lr_bwd_row<Tin, Tg, V>(f[u], old[u], dhf, a_s[i + u],
+                                                        dvalues + (int64_t)(i + u) * src_stride + row_off,
+                                                        p.d < skip0 ? p.d : skip0, lane, p.accumulate);
+                const float g = warp_sum(gp);
+                if (lane == 0) g_s[i + u] = g;
+            }
+        }
+        for (; i < p.n; ++i) {
+            Frag<Tin, E> f[V];
+            Frag<Tg, E> old[V];
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                const int64_t off = (int64_t)i * src_stride + row_off + e;
+                if (e < p.d) f[v].load_nc(values + off);
+                else f[v].zero();
+                if (p.accumulate && e < skip0) old[v].load(dvalues + off);
+                else old[v].zero();
+            }
+            const float gp = lr_bwd_row<Tin, Tg, V>(f, old, dhf, a_s[i], dvalues + (int64_t)i * src_stride + row_off,
+                                                    p.d < skip0 ? p.d : skip0, lane, p.accumulate);
+            const float g = warp_sum(gp);
+            if (lane == 0) g_s[i] = g;
+        }
+        __syncwarp();
+
+        // (3) key pass: gbar, ds_i, dL/dk_i, dq
+        float part = 0.f;
+        for (int k = lane; k < p.n; k += 32) part = fmaf(a_s[k], g_s[k], part);
+        const float gbar = warp_sum(part);
+        __syncwarp();
+        for (int k = lane; k < p.n; k += 32) g_s[k] = a_s[k] * (g_s[k] - gbar);
+        __syncwarp();
+        for (int j = lane; j < p.r; j += 32) {
+            const float qj = q_s[j];
+            const int c = tail0 + j;  // coordinate of key element j inside the value row (SLICED)
+            const float dh_c = p.sliced ? to_f(__ldg(dh + row_off + c)) : 0.f;
+            float dqj = 0.f;
+#pragma unroll 4
+            for (int k = 0; k < p.n; ++k) {
+                const float rho = rho_s[k], s = s_s[k], ds = g_s[k];
+                float kij;
+                if (p.sliced) kij = to_f(__ldg(values + (int64_t)k * src_stride + row_off + c));
+                else kij = to_f(__ldg(keys + ((int64_t)k * p.T + x) * p.r + j));
+                const float kbar = rho * kij;
+                const float dk = ds * rho * (qj - s * p.inv_r * kbar);
+                dqj = fmaf(ds, kbar, dqj);
+                if (p.sliced) {
+                    Tg *dp = dvalues + (int64_t)k * src_stride + row_off + c;
+                    float w;
+                    if (c < skip0) w = to_f(*dp) + dk;  // written by the value pass
+                    else w = (p.accumulate ? to_f(*dp) : 0.f) + fmaf(a_s[k], dh_c, dk);
+                    *dp = from_f<Tg>(w);
+                } else {
+                    Tg *dp = dkeys + ((int64_t)k * p.T + x) * p.r + j;
+                    *dp = from_f<Tg>(p.accumulate ? to_f(*dp) + dk : dk);
+                }
+            }
+            dq_s[j] += dqj;  // coordinate j belongs to this lane alone
+        }
+        __syncwarp();
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < p.r; j += kThreads) {
+        float acc = 0.f;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) acc += dq_all[w * rp + j];
+        p.partials[(int64_t)blockIdx.x * p.r + j] = acc;
+    }
+}
+
+// -------------------------------------------------------------- full keys
+template <typename Tin, typename Tg, int V>
+__device__ __forceinline__ void full_bwd_row(const Frag<Tin, VecE<Tin>::value> *f,
+                                             const Frag<Tg, VecE<Tin>::value> *old, const float *dhf,
+                                             const float *__restrict__ q_s, float *dqf, float gbar, float lse,
+                                             float inv_d, float eps, Tg *__restrict__ drow, int d, int lane,
+                                             int accumulate) {
+    constexpr int E = VecE<Tin>::value;
+    float o[V * E];
+    float g = 0.f, ss = 0.f, qo = 0.f;
+#pragma unroll
+    for (int v = 0; v < V; ++v) f[v].get(o + v * E);
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+        const int e = (lane + 32 * v) * E;
+#pragma unroll
+        for (int t = 0; t < E; ++t) {
+            const float qv = (e < d) ? q_s[e + t] : 0.f;
+            g = fmaf(dhf[v * E + t], o[v * E + t], g);
+            ss = fmaf(o[v * E + t], o[v * E + t], ss);
+            qo = fmaf(qv, o[v * E + t], qo);
+        }
+    }
+    g = warp_sum(g);
+    ss = warp_sum(ss);
+    qo = warp_sum(qo);
+    const float rho = rsqrtf(fmaf(ss, inv_d, eps));
+    const float s = rho * qo;
+    const float a = expf(s - lse);
+    const float ds = a * (g - gbar);
+    const float c1 = ds * rho;             // coefficient of q
+    const float c2 = c1 * rho * s * inv_d;  // coefficient of o_i
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+        const int e = (lane + 32 * v) * E;
+        if (e < d) {
+            float w[E];
+            if (accumulate) old[v].get(w);
+            else
+#pragma unroll
+                for (int t = 0; t < E; ++t) w[t] = 0.f;
+#pragma unroll
+            for (int t = 0; t < E; ++t) {
+                const float ov = o[v * E + t];
+                w[t] = fmaf(a, dhf[v * E + t], w[t]);
+                w[t] = fmaf(c1, q_s[e + t], w[t]);
+                w[t] = fmaf(-c2, ov, w[t]);
+                dqf[v * E + t] = fmaf(c1, ov, dqf[v * E + t]);
+            }
+            Frag<Tg, E> out;
+            out.set(w);
+            out.store(drow + e);
+        }
+    }
+}
+
+template <typename Tin, typename Tg, int V, int U>
+__global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(const BwdParams p) {
+    constexpr int E = VecE<Tin>::value;
+    extern __shared__ float smem[];
+    const int dp4 = round_up(p.d, 4);
+    float *q_s = smem;          // [d]
+    float *dq_all = q_s + dp4;  // [kWarps][d], used once at the end
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int j = threadIdx.x; j < p.d; j += kThreads) q_s[j] = p.query ? p.query[j] : 0.f;
+    __syncthreads();
+
+    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
+    const Tin *__restrict__ dh = static_cast<const Tin *>(p.dh);
+    Tg *__restrict__ dvalues = static_cast<Tg *>(p.dvalues);
+    const int64_t src_stride = p.T * (int64_t)p.d;
+    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+    const float inv_d = 1.f / (float)p.d;
+    float dqf[V * E];
+#pragma unroll
+    for (int t = 0; t < V * E; ++t) dqf[t] = 0.f;
+
+    for (int64_t x = (int64_t)blockIdx.x * kWarps + warp; x < p.T; x += nwarps) {
+        const int64_t row_off = x * p.d;
+        float dhf[V * E];
+        float gb = 0.f;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int e = (lane + 32 * v) * E;
+            Frag<Tin, E> f;
+            if (e < p.d) f.load_nc(dh + row_off + e);
+            else f.zero();
+            f.get(dhf + v * E);
+            float hv[E];
+            if (e < p.d) {
+                if (p.h_bf16) {
+                    Frag<bf16, E> hf;
+                    hf.load_nc(static_cast<const bf16 *>(p.h) + row_off + e);
+                    hf.get(hv);
+                } else {
+                    Frag<float, E> hf;
+                    hf.load_nc(static_cast<const float *>(p.h) + row_off + e);
+                    hf.get(hv);
+                }
+            } else {
+#pragma unroll
+                for (int t = 0; t < E; ++t) hv[t] = 0.f;
+            }
+#pragma unroll
+            for (int t = 0; t < E; ++t) gb = fmaf(dhf[v * E + t], hv[t], gb);
+        }
+        const float gbar = warp_sum(gb);  // <dh, h> = sum_i alpha_i g_i
+        const float lse = __ldg(p.lse + x);
+        int i = 0;
+        for (; i + U <= p.n; i += U) {
+            Frag<Tin, E> f[U][V];
+            Frag<Tg, E> old[U][V];
+#pragma unroll
+            for (int u = 0; u < U; ++u)
+#pragma unroll
+                for (int v = 0; v < V; ++v) {
+                    const int e = (lane + 32 * v) * E;
+                    const int64_t off = (int64_t)(i + u) * src_stride + row_off + e;
+                    if (e < p.d) f[u][v].load_nc(values + off);
+                    else f[u][v].zero();
+                    if (p.accumulate && e < p.d) old[u][v].load(dvalues + off);
+                    else old[u][v].zero();
+                }
+#pragma unroll
+            for (int u = 0; u < U; ++u)
+                full_bwd_row<Tin, Tg, V>(f[u], old[u], dhf, q_s, dqf, gbar, lse, inv_d, p.eps,
+                                         dvalues + (int64_t)(i + u) * src_stride + row_off, p.d, lane, p.accumulate);
+        }
+        for (; i < p.n; ++i) {
+            Frag<Tin, E> f[V];
+            Frag<Tg, E> old[V];
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                const int64_t off = (int64_t)i * src_stride + row_off + e;
+                if (e < p.d) f[v].load_nc(values + off);
+                else f[v].zero();
+                if (p.accumulate && e < p.d) old[v].load(dvalues + off);
+                else old[v].zero();
+            }
+            full_bwd_row<Tin, Tg, V>(f, old, dhf, q_s, dqf, gbar, lse, inv_d, p.eps,
+                                     dvalues + (int64_t)i * src_stride + row_off, p.d, lane, p.accumulate);
+        }
+    }
+    // CTA partial of dq = sum ds_i rho_i o_i
+    float *dq_s = dq_all + warp * dp4;
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+        const int e = (lane + 32 * v) * E;
+        if (e < p.d)
+#pragma unroll
+            for (int t = 0; t < E; ++t) dq_s[e + t] = dqf[v * E + t];
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < p.d; j += kThreads) {
+        float acc = 0.f;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) acc += dq_all[w * dp4 + j];
+        p.partials[(int64_t)blockIdx.x * p.d + j] = acc;
+    }
+}
+
+// Fixed-order sum of the CTA partials: dq[j] (+)= sum_b partials[b][j].
+__global__ void dq_reduce_kernel(const float *__restrict__ partials, int nparts, int rq, float *dq, int accumulate) {
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= rq) return;
+    float acc = 0.f;
+    for (int b = 0; b < nparts; ++b) acc += partials[(int64_t)b * rq + j];
+    dq[j] = accumulate ? dq[j] + acc : acc;
+}
+
+// ------------------------------------------------------------- launch ----
+template <typename Tin, typename Tg, int V>
+static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
+    constexpr int U = V >= 4 ? 1 : (V == 2 ? 2 : 4);
+    BwdParams p;
+    p.values = a.values;
+    p.keys = a.keys;
+    p.dh = a.dh;
+    p.h = a.h;
+    p.query = a.query;
+    p.lse = a.lse;
+    p.dvalues = a.dvalues;
+    p.dkeys = a.dkeys;
+    p.partials = a.partials;
+    p.T = a.T;
+    p.n = a.n;
+    p.d = a.d;
+    p.r = a.r;
+    p.eps = a.eps;
+    p.inv_r = 1.f / (float)a.r;
+    p.sliced = a.variant == kSliced;
+    p.accumulate = a.accumulate;
+    p.h_bf16 = a.h_dtype == kBF16;
+    constexpr int esz = sizeof(Tin);
+    if (a.variant == kSliced)
+        p.key_vec = ((a.r * esz) % 16 == 0) && (((a.d - a.r) * esz) % 16 == 0);
+    else
+        p.key_vec = ((a.r * esz) % 16 == 0) && ((reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
+    const int64_t work = (a.T + kWarps - 1) / kWarps;
+    const void *k;
+    size_t smem;
+    int rq;
+    if (a.variant == kFull) {
+        k = (const void *)bwd_full_kernel<Tin, Tg, V, U>;
+        smem = sizeof(float) * (size_t)round_up(a.d, 4) * (1 + kWarps);
+        rq = a.d;
+    } else {
+        k = (const void *)bwd_lr_kernel<Tin, Tg, V, U>;
+        smem = sizeof(float) * ((size_t)round_up(a.r, 4) * (1 + kWarps) + (size_t)kWarps * 4 * kMaxSources);
+        rq = a.r;
+    }
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    const int grid = persistent_grid(k, kThreads, smem, work, kMaxPartials);
+    if (a.variant == kFull)
+        bwd_full_kernel<Tin, Tg, V, U><<<grid, kThreads, smem, s>>>(p);
+    else
+        bwd_lr_kernel<Tin, Tg, V, U><<<grid, kThreads, smem, s>>>(p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    dq_reduce_kernel<<<(rq + 255) / 256, 256, 0, s>>>(a.partials, grid, rq, a.dq, a.accumulate);
+    return cudaGetLastError();
+}
+
+template <typename Tin, typename Tg>
+static cudaError_t launch_bwd_w(const BwdArgs &a, cudaStream_t s) {
+    constexpr int E = VecE<Tin>::value;
+    const int vecs = (a.d + E - 1) / E;
+    if (vecs <= 32) return launch_bwd_t<Tin, Tg, 1>(a, s);
+    if (vecs <= 64) return launch_bwd_t<Tin, Tg, 2>(a, s);
+    if (vecs <= 128) return launch_bwd_t<Tin, Tg, 4>(a, s);
+    return launch_bwd_t<Tin, Tg, 8>(a, s);
+}
+
+cudaError_t launch_backward(const BwdArgs &a, cudaStream_t s) {
+    if (a.in_dtype == kBF16)
+        return a.grad_dtype == kBF16 ? launch_bwd_w<bf16, bf16>(a, s) : launch_bwd_w<bf16, float>(a, s);
+    return a.grad_dtype == kBF16 ? launch_bwd_w<float, bf16>(a, s) : launch_bwd_w<float, float>(a, s);
+}
+
+// ------------------------------------------------------ block assembly ---
+// dst = beta * dst + alpha * src over count elements, 8 per thread-step.
+template <typename Td, typename Ts>
+__global__ void block_acc_kernel(Td *__restrict__ dst, const Ts *__restrict__ src, int64_t count, float alpha,
+                                 float beta, int vec) {
+    const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t nthreads = (int64_t)gridDim.x * blockDim.x;
+    const int64_t groups = vec ? count / 8 : 0;
+    for (int64_t gi = tid; gi < groups; gi += nthreads) {
+        const int64_t e = gi * 8;
+        Frag<Ts, 8> fs;
+        fs.load_nc(src + e);
+        float sv[8], w[8];
+        fs.get(sv);
+        if (beta != 0.f) {
+            Frag<Td, 8> fd;
+            fd.load(dst + e);
+            fd.get(w);
+#pragma unroll
+            for (int t = 0; t < 8; ++t) w[t] = fmaf(alpha, sv[t], beta * w[t]);
+        } else {
+#pragma unroll
+            for (int t = 0; t < 8; ++t) w[t] = alpha * sv[t];
+        }
+        Frag<Td, 8> out;
+        out.set(w);
+        out.store(dst + e);
+    }
+    for (int64_t e = groups * 8 + tid; e < count; e += nthreads) {
+        const float sv = to_f(src[e]);
+        const float w = beta != 0.f ? fmaf(alpha, sv, beta * to_f(dst[e])) : alpha * sv;
+        dst[e] = from_f<Td>(w);
+    }
+}
+
+template <typename Td, typename Ts>
+static cudaError_t launch_acc_t(void *dst, const void *src, int64_t count, float alpha, float beta, cudaStream_t s) {
+    const int vec = ((reinterpret_cast<uintptr_t>(dst) | reinterpret_cast<uintptr_t>(src)) & 15) == 0;
+    const int threads = 256;
+    const int64_t groups = vec ? count / 8 : count;
+    const int grid = persistent_grid((const void *)block_acc_kernel<Td, Ts>, threads, 0,
+                                     (groups + threads - 1) / threads, 1 << 30);
+    block_acc_kernel<Td, Ts><<<grid, threads, 0, s>>>(static_cast<Td *>(dst), static_cast<const Ts *>(src), count,
+                                                       alpha, beta, vec);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *src, int64_t count,
+                                    float alpha, float beta, cudaStream_t s) {
+    if (dst_dtype == kBF16)
+        return src_dtype == kBF16 ? launch_acc_t<bf16, bf16>(dst, src, count, alpha, beta, s)
+                                  : launch_acc_t<bf16, float>(dst, src, count, alpha, beta, s);
+    return src_dtype == kBF16 ? launch_acc_t<float, bf16>(dst, src, count, alpha, beta, s)
+                              : launch_acc_t<float, float>(dst, src, count, alpha, beta, s);
+}
+
+}  // namespace lrar

@@ -1,0 +1,131 @@
+// lrar_device.cuh -- device helpers shared by the depth-mix kernels:
+// 16-byte streaming loads, bf16 <-> f32 packing, warp reductions.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace lrar {
+
+constexpr int kWarps = 8;                 // warps per CTA
+constexpr int kThreads = kWarps * 32;
+constexpr int kMaxSources = 128;          // LRAR_MAX_SOURCES
+constexpr int kSrcRegs = kMaxSources / 32;
+constexpr int kMaxPartials = 1024;        // CTAs whose dq partials the workspace holds
+
+typedef __nv_bfloat16 bf16;
+
+// Elements of T in one 16-byte vector.
+template <typename T> struct VecE;
+template <> struct VecE<float> { static constexpr int value = 4; };
+template <> struct VecE<bf16> { static constexpr int value = 8; };
+
+// ---------------------------------------------------------------- loads ----
+// Read-only, streamed once: bypass L1 allocation.
+__device__ __forceinline__ uint4 ld_nc16(const void *p) {
+    uint4 v;
+    asm("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+        : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+        : "l"(p));
+    return v;
+}
+__device__ __forceinline__ uint2 ld_nc8(const void *p) {
+    uint2 v;
+    asm("ld.global.nc.L1::no_allocate.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "l"(p));
+    return v;
+}
+// Coherent loads/stores (data the same kernel writes).
+__device__ __forceinline__ uint4 ld16(const void *p) { return *reinterpret_cast<const uint4 *>(p); }
+__device__ __forceinline__ uint2 ld8(const void *p) { return *reinterpret_cast<const uint2 *>(p); }
+__device__ __forceinline__ void st16(void *p, uint4 v) { *reinterpret_cast<uint4 *>(p) = v; }
+__device__ __forceinline__ void st8(void *p, uint2 v) { *reinterpret_cast<uint2 *>(p) = v; }
+
+// ------------------------------------------------------------- packing ----
+// A bfloat16 is the upper half of a binary32 word, so widening is a shift.
+__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+__device__ __forceinline__ uint32_t bf_pack(float lo, float hi) {
+    __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);  // round to nearest even
+    return *reinterpret_cast<uint32_t *>(&b);
+}
+
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(bf16 v) { return __bfloat162float(v); }
+template <typename T> __device__ __forceinline__ T from_f(float v);
+template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __float2bfloat16_rn(v); }
+
+// E consecutive elements of type T held as raw words.
+template <typename T, int E> struct Frag;
+
+template <> struct Frag<bf16, 8> {
+    uint4 a;
+    __device__ __forceinline__ void load_nc(const bf16 *p) { a = ld_nc16(p); }
+    __device__ __forceinline__ void load(const bf16 *p) { a = ld16(p); }
+    __device__ __forceinline__ void store(bf16 *p) const { st16(p, a); }
+    __device__ __forceinline__ void zero() { a = make_uint4(0, 0, 0, 0); }
+    __device__ __forceinline__ void get(float *f) const {
+        f[0] = bf_lo(a.x); f[1] = bf_hi(a.x); f[2] = bf_lo(a.y); f[3] = bf_hi(a.y);
+        f[4] = bf_lo(a.z); f[5] = bf_hi(a.z); f[6] = bf_lo(a.w); f[7] = bf_hi(a.w);
+    }
+    __device__ __forceinline__ void set(const float *f) {
+        a.x = bf_pack(f[0], f[1]); a.y = bf_pack(f[2], f[3]);
+        a.z = bf_pack(f[4], f[5]); a.w = bf_pack(f[6], f[7]);
+    }
+};
+
+template <> struct Frag<bf16, 4> {
+    uint2 a;
+    __device__ __forceinline__ void load_nc(const bf16 *p) { a = ld_nc8(p); }
+    __device__ __forceinline__ void load(const bf16 *p) { a = ld8(p); }
+    __device__ __forceinline__ void store(bf16 *p) const { st8(p, a); }
+    __device__ __forceinline__ void zero() { a = make_uint2(0, 0); }
+    __device__ __forceinline__ void get(float *f) const {
+        f[0] = bf_lo(a.x); f[1] = bf_hi(a.x); f[2] = bf_lo(a.y); f[3] = bf_hi(a.y);
+    }
+    __device__ __forceinline__ void set(const float *f) { a.x = bf_pack(f[0], f[1]); a.y = bf_pack(f[2], f[3]); }
+};
+
+template <> struct Frag<float, 4> {
+    uint4 a;
+    __device__ __forceinline__ void load_nc(const float *p) { a = ld_nc16(p); }
+    __device__ __forceinline__ void load(const float *p) { a = ld16(p); }
+    __device__ __forceinline__ void store(float *p) const { st16(p, a); }
+    __device__ __forceinline__ void zero() { a = make_uint4(0, 0, 0, 0); }
+    __device__ __forceinline__ void get(float *f) const {
+        f[0] = __uint_as_float(a.x); f[1] = __uint_as_float(a.y);
+        f[2] = __uint_as_float(a.z); f[3] = __uint_as_float(a.w);
+    }
+    __device__ __forceinline__ void set(const float *f) {
+        a.x = __float_as_uint(f[0]); a.y = __float_as_uint(f[1]);
+        a.z = __float_as_uint(f[2]); a.w = __float_as_uint(f[3]);
+    }
+};
+
+template <> struct Frag<float, 8> {
+    Frag<float, 4> lo, hi;
+    __device__ __forceinline__ void load_nc(const float *p) { lo.load_nc(p); hi.load_nc(p + 4); }
+    __device__ __forceinline__ void load(const float *p) { lo.load(p); hi.load(p + 4); }
+    __device__ __forceinline__ void store(float *p) const { lo.store(p); hi.store(p + 4); }
+    __device__ __forceinline__ void zero() { lo.zero(); hi.zero(); }
+    __device__ __forceinline__ void get(float *f) const { lo.get(f); hi.get(f + 4); }
+    __device__ __forceinline__ void set(const float *f) { lo.set(f); hi.set(f + 4); }
+};
+
+// ----------------------------------------------------------- reductions ---
+// xor butterflies leave the identical bit pattern in every lane.
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+__host__ __device__ __forceinline__ int round_up(int a, int b) { return (a + b - 1) / b * b; }
+
+}  // namespace lrar

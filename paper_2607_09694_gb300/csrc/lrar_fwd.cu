@@ -1,0 +1,334 @@
+// lrar_fwd.cu -- forward depth-attention mix, Eq. (8)-(10) of arxiv 2607.09694.
+//
+// One warp owns one token row at a time (grid-stride over tokens, persistent
+// grid sized to the resident CTAs of the device).  Lane l holds the 16-byte
+// vectors l, l+32, ... of the row, so every load instruction of a warp covers
+// 512 contiguous bytes of one source row.
+//
+// Low-rank keys (SLICED, PROJECTED): a routing stage reads the n r-dim keys
+// (lane i scores source i), takes the softmax with two warp reductions and
+// leaves alpha in shared memory; the value stage then streams the n full-width
+// value rows once and accumulates in fp32 registers.
+//
+// Full keys (AttnRes, r = d): the key is the whole value row, so the score of a
+// source is known only once its row is loaded.  The kernel streams each row
+// once with an online softmax (running max, rescaled accumulator), so the
+// values are read exactly once.
+#include "lrar_device.cuh"
+#include "lrar_launch.h"
+
+namespace lrar {
+
+struct FwdParams {
+    const void *values, *keys;
+    const float *query;
+    void *h;
+    float *lse;
+    int64_t T;
+    int n, d, r;
+    float eps, inv_r;
+    int sliced;   // key = last r coordinates of the value row
+    int key_vec;  // keys can be read as aligned 16-byte vectors
+};
+
+// sum_j k_j^2 and sum_j q_j k_j of one key of r elements.
+template <typename Tin>
+__device__ __forceinline__ void key_stats(const Tin *__restrict__ kp, int r, const float *__restrict__ q_s,
+                                          bool vec, float &ss, float &qk) {
+    ss = 0.f;
+    qk = 0.f;
+    if (vec) {
+        constexpr int E = VecE<Tin>::value;
+        for (int j = 0; j < r; j += E) {
+            Frag<Tin, E> f;
+            f.load_nc(kp + j);
+            float k[E];
+            f.get(k);
+#pragma unroll
+            for (int t = 0; t < E; ++t) {
+                ss = fmaf(k[t], k[t], ss);
+                qk = fmaf(q_s[j + t], k[t], qk);
+            }
+        }
+    } else {
+        for (int j = 0; j < r; ++j) {
+            const float k = to_f(__ldg(kp + j));
+            ss = fmaf(k, k, ss);
+            qk = fmaf(q_s[j], k, qk);
+        }
+    }
+}
+
+// Routing stage for token x (Eq. 8-9): lane owns sources lane + 32k.
+// Leaves alpha_i in a_s[i] (and s_i, rho_i in s_s, rho_s when non-null);
+// returns lse = log sum_i exp(s_i) in every lane.
+template <typename Tin>
+__device__ __forceinline__ float lr_route(const Tin *__restrict__ values, const Tin *__restrict__ keys, int64_t T,
+                                          int n, int d, int r, float eps, float inv_r, int sliced, int key_vec,
+                                          int64_t x, int lane, const float *__restrict__ q_s, float *a_s, float *s_s,
+                                          float *rho_s) {
+    float s_reg[kSrcRegs];
+    float m = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < kSrcRegs; ++k) {
+        const int i = lane + 32 * k;
+        float s = -INFINITY;
+        if (i < n) {
+            const Tin *kp = sliced ? values + ((int64_t)i * T + x) * d + (d - r) : keys + ((int64_t)i * T + x) * r;
+            float ss, qk;
+            key_stats<Tin>(kp, r, q_s, key_vec != 0, ss, qk);
+            const float rho = rsqrtf(fmaf(ss, inv_r, eps));
+            s = rho * qk;
+            if (s_s) {
+                s_s[i] = s;
+                rho_s[i] = rho;
+            }
+        }
+        s_reg[k] = s;
+        m = fmaxf(m, s);
+    }
+    m = warp_max(m);
+    float z = 0.f;
+#pragma unroll
+    for (int k = 0; k < kSrcRegs; ++k) {
+        const int i = lane + 32 * k;
+        const float e = (i < n) ? expf(s_reg[k] - m) : 0.f;
+        s_reg[k] = e;
+        z += e;
+    }
+    z = warp_sum(z);
+    const float inv_z = 1.f / z;
+#pragma unroll
+    for (int k = 0; k < kSrcRegs; ++k) {
+        const int i = lane + 32 * k;
+        if (i < n) a_s[i] = s_reg[k] * inv_z;
+    }
+    return m + logf(z);
+}
+
+template <typename Tin, typename Tout, int V>
+__device__ __forceinline__ void store_row(Tout *__restrict__ hrow, int d, int lane, const float *acc, float scale) {
+    constexpr int E = VecE<Tin>::value;
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+        const int e = (lane + 32 * v) * E;
+        if (e < d) {
+            float o[E];
+#pragma unroll
+            for (int t = 0; t < E; ++t) o[t] = acc[v * E + t] * scale;
+            Frag<Tout, E> f;
+            f.set(o);
+            f.store(hrow + e);
+        }
+    }
+}
+
+// ------------------------------------------------- low-rank keys (LR) ----
+template <typename Tin, typename Tout, int V, int U>
+__global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(const FwdParams p) {
+    constexpr int E = VecE<Tin>::value;
+    extern __shared__ float smem[];
+    float *q_s = smem;                                         // [r]
+    float *a_all = smem + round_up(p.r, 4);                    // [kWarps][kMaxSources]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    float *a_s = a_all + warp * kMaxSources;
+    for (int j = threadIdx.x; j < p.r; j += kThreads) q_s[j] = p.query ? p.query[j] : 0.f;
+    __syncthreads();
+
+    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
+    const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
+    const int64_t src_stride = p.T * (int64_t)p.d;
+    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+
+    for (int64_t x = (int64_t)blockIdx.x * kWarps + warp; x < p.T; x += nwarps) {
+        const float lse = lr_route<Tin>(values, keys, p.T, p.n, p.d, p.r, p.eps, p.inv_r, p.sliced, p.key_vec, x,
+                                        lane, q_s, a_s, nullptr, nullptr);
+        if (lane == 0 && p.lse) p.lse[x] = lse;
+        __syncwarp();
+
+        // Eq. (10): h = sum_i alpha_i o_i, fp32 accumulation.
+        float acc[V * E];
+#pragma unroll
+        for (int t = 0; t < V * E; ++t) acc[t] = 0.f;
+        const Tin *row0 = values + x * p.d;
+        int i = 0;
+        for (; i + U <= p.n; i += U) {
+            Frag<Tin, E> f[U][V];
+#pragma unroll
+            for (int u = 0; u < U; ++u)
+#pragma unroll
+                for (int v = 0; v < V; ++v) {
+                    const int e = (lane + 32 * v) * E;
+                    if (e < p.d) f[u][v].load_nc(row0 + (int64_t)(i + u) * src_stride + e);
+                    else f[u][v].zero();
+                }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const float a = a_s[i + u];
+#pragma unroll
+                for (int v = 0; v < V; ++v) {
+                    float o[E];
+                    f[u][v].get(o);
+#pragma unroll
+                    for (int t = 0; t < E; ++t) acc[v * E + t] = fmaf(a, o[t], acc[v * E + t]);
+                }
+            }
+        }
+        for (; i < p.n; ++i) {
+            const float a = a_s[i];
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                Frag<Tin, E> f;
+                if (e < p.d) f.load_nc(row0 + (int64_t)i * src_stride + e);
+                else f.zero();
+                float o[E];
+                f.get(o);
+#pragma unroll
+                for (int t = 0; t < E; ++t) acc[v * E + t] = fmaf(a, o[t], acc[v * E + t]);
+            }
+        }
+        store_row<Tin, Tout, V>(static_cast<Tout *>(p.h) + x * p.d, p.d, lane, acc, 1.f);
+        __syncwarp();  // a_s is rewritten for the next token
+    }
+}
+
+// ------------------------------------------------------- full keys -------
+template <typename Tin, int V>
+__device__ __forceinline__ void full_row_step(const Frag<Tin, VecE<Tin>::value> *f, const float *qf, float inv_d,
+                                              float eps, float &m, float &z, float *acc) {
+    constexpr int E = VecE<Tin>::value;
+    float o[V * E];
+    float ss = 0.f, qo = 0.f;
+#pragma unroll
+    for (int v = 0; v < V; ++v) f[v].get(o + v * E);
+#pragma unroll
+    for (int t = 0; t < V * E; ++t) {
+        ss = fmaf(o[t], o[t], ss);
+        qo = fmaf(qf[t], o[t], qo);
+    }
+    ss = warp_sum(ss);
+    qo = warp_sum(qo);
+    const float s = rsqrtf(fmaf(ss, inv_d, eps)) * qo;  // Eq. (2) with RMSNorm(o_i) as the key
+    if (s > m) {                                        // warp-uniform: s is identical in all lanes
+        const float c = expf(m - s);
+        z *= c;
+#pragma unroll
+        for (int t = 0; t < V * E; ++t) acc[t] *= c;
+        m = s;
+    }
+    const float w = expf(s - m);
+    z += w;
+#pragma unroll
+    for (int t = 0; t < V * E; ++t) acc[t] = fmaf(w, o[t], acc[t]);
+}
+
+template <typename Tin, typename Tout, int V, int U>
+__global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) fwd_full_kernel(const FwdParams p) {
+    constexpr int E = VecE<Tin>::value;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    float qf[V * E];
+#pragma unroll
+    for (int v = 0; v < V; ++v)
+#pragma unroll
+        for (int t = 0; t < E; ++t) {
+            const int e = (lane + 32 * v) * E + t;
+            qf[v * E + t] = (p.query && e < p.d) ? __ldg(p.query + e) : 0.f;
+        }
+    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
+    const int64_t src_stride = p.T * (int64_t)p.d;
+    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+    const float inv_d = 1.f / (float)p.d;
+
+    for (int64_t x = (int64_t)blockIdx.x * kWarps + warp; x < p.T; x += nwarps) {
+        float acc[V * E];
+#pragma unroll
+        for (int t = 0; t < V * E; ++t) acc[t] = 0.f;
+        float m = -INFINITY, z = 0.f;
+        const Tin *row0 = values + x * p.d;
+        int i = 0;
+        for (; i + U <= p.n; i += U) {
+            Frag<Tin, E> f[U][V];
+#pragma unroll
+            for (int u = 0; u < U; ++u)
+#pragma unroll
+                for (int v = 0; v < V; ++v) {
+                    const int e = (lane + 32 * v) * E;
+                    if (e < p.d) f[u][v].load_nc(row0 + (int64_t)(i + u) * src_stride + e);
+                    else f[u][v].zero();
+                }
+#pragma unroll
+            for (int u = 0; u < U; ++u) full_row_step<Tin, V>(f[u], qf, inv_d, p.eps, m, z, acc);
+        }
+        for (; i < p.n; ++i) {
+            Frag<Tin, E> f[V];
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) f[v].load_nc(row0 + (int64_t)i * src_stride + e);
+                else f[v].zero();
+            }
+            full_row_step<Tin, V>(f, qf, inv_d, p.eps, m, z, acc);
+        }
+        store_row<Tin, Tout, V>(static_cast<Tout *>(p.h) + x * p.d, p.d, lane, acc, 1.f / z);
+        if (lane == 0 && p.lse) p.lse[x] = m + logf(z);
+    }
+}
+
+// ------------------------------------------------------------- launch ----
+template <typename Tin, typename Tout, int V>
+static cudaError_t launch_fwd_t(const FwdArgs &a, cudaStream_t s) {
+    constexpr int U = V >= 8 ? 1 : (V == 4 ? 2 : 4);
+    FwdParams p;
+    p.values = a.values;
+    p.keys = a.keys;
+    p.query = a.query;
+    p.h = a.h;
+    p.lse = a.lse;
+    p.T = a.T;
+    p.n = a.n;
+    p.d = a.d;
+    p.r = a.r;
+    p.eps = a.eps;
+    p.inv_r = 1.f / (float)a.r;
+    p.sliced = a.variant == kSliced;
+    constexpr int esz = sizeof(Tin);
+    if (a.variant == kSliced)
+        p.key_vec = ((a.r * esz) % 16 == 0) && (((a.d - a.r) * esz) % 16 == 0);
+    else
+        p.key_vec = ((a.r * esz) % 16 == 0) && ((reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
+    const int64_t work = (a.T + kWarps - 1) / kWarps;
+    if (a.variant == kFull) {
+        const void *k = (const void *)fwd_full_kernel<Tin, Tout, V, U>;
+        const int grid = persistent_grid(k, kThreads, 0, work, 1 << 30);
+        fwd_full_kernel<Tin, Tout, V, U><<<grid, kThreads, 0, s>>>(p);
+    } else {
+        const size_t smem = sizeof(float) * (round_up(a.r, 4) + kWarps * kMaxSources);
+        const void *k = (const void *)fwd_lr_kernel<Tin, Tout, V, U>;
+        if (smem > 48 * 1024) {
+            cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (e != cudaSuccess) return e;
+        }
+        const int grid = persistent_grid(k, kThreads, smem, work, 1 << 30);
+        fwd_lr_kernel<Tin, Tout, V, U><<<grid, kThreads, smem, s>>>(p);
+    }
+    return cudaGetLastError();
+}
+
+template <typename Tin, typename Tout>
+static cudaError_t launch_fwd_w(const FwdArgs &a, cudaStream_t s) {
+    constexpr int E = VecE<Tin>::value;
+    const int vecs = (a.d + E - 1) / E;  // 16-byte vectors per row
+    if (vecs <= 32) return launch_fwd_t<Tin, Tout, 1>(a, s);
+    if (vecs <= 64) return launch_fwd_t<Tin, Tout, 2>(a, s);
+    if (vecs <= 128) return launch_fwd_t<Tin, Tout, 4>(a, s);
+    return launch_fwd_t<Tin, Tout, 8>(a, s);
+}
+
+cudaError_t launch_forward(const FwdArgs &a, cudaStream_t s) {
+    if (a.in_dtype == kBF16)
+        return a.out_dtype == kBF16 ? launch_fwd_w<bf16, bf16>(a, s) : launch_fwd_w<bf16, float>(a, s);
+    return a.out_dtype == kBF16 ? launch_fwd_w<float, bf16>(a, s) : launch_fwd_w<float, float>(a, s);
+}
+
+}  // namespace lrar

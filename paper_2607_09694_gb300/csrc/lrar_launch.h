@@ -1,0 +1,57 @@
+// lrar_launch.h -- host-side launch interface between the C ABI (lrar_api.cu)
+// and the kernel translation units.  Arguments arrive here already validated.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace lrar {
+
+enum { kFull = 0, kSliced = 1, kProjected = 2 };
+enum { kF32 = 0, kBF16 = 1 };
+
+struct FwdArgs {
+    int variant, in_dtype, out_dtype;
+    const void *values;
+    const void *keys;
+    const float *query;  // may be null when n == 1
+    int n;
+    int64_t T;
+    int d, r;
+    float eps;
+    void *h;
+    float *lse;  // may be null
+};
+
+struct BwdArgs {
+    int variant, in_dtype, grad_dtype, h_dtype;
+    const void *values;
+    const void *keys;
+    const float *query;
+    int n;
+    int64_t T;
+    int d, r;
+    float eps;
+    const void *dh;
+    const void *h;
+    const float *lse;
+    void *dvalues;
+    void *dkeys;
+    float *dq;
+    int accumulate;
+    float *partials;  // workspace: [kMaxPartials][rq] floats
+};
+
+// Largest d one warp covers (the kernels keep a whole token row per warp).
+int max_width(int in_dtype);
+
+cudaError_t launch_forward(const FwdArgs &a, cudaStream_t s);
+cudaError_t launch_backward(const BwdArgs &a, cudaStream_t s);
+cudaError_t launch_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *src, int64_t count,
+                                    float alpha, float beta, cudaStream_t s);
+
+// Resident CTAs of `kernel` per SM times the SM count of the current device,
+// capped by `cap`.
+int persistent_grid(const void *kernel, int threads, size_t smem, int64_t work_ctas, int cap);
+
+}  // namespace lrar

@@ -1,0 +1,152 @@
+"""Python binding of liblrar.so (include/lrar.h): argument marshalling only.
+
+Every function takes CUDA tensors (or raw integer device pointers), turns them
+into the C ABI's pointers, sizes and type codes, and calls the library on the
+current torch stream.  All arithmetic happens in the library's CUDA kernels;
+there is no fallback, and a missing or unbuilt library raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+FULL, SLICED, PROJECTED = 0, 1, 2
+F32, BF16 = 0, 1
+VARIANTS = {"full": FULL, "sliced": SLICED, "projected": PROJECTED}
+MAX_SOURCES = 128
+DEFAULT_EPS = 1e-6
+
+OK = 0
+ERR_INVALID_ARG, ERR_ALIGNMENT, ERR_UNSUPPORTED, ERR_CUDA, ERR_WORKSPACE = -1, -2, -3, -4, -5
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "liblrar.so")
+EXPORTS = ("lrar_forward", "lrar_backward", "lrar_backward_workspace_size", "lrar_block_accumulate",
+           "lrar_strerror", "lrar_last_error", "lrar_version")
+
+_lock = threading.Lock()
+_lib = None
+
+
+class LrarError(RuntimeError):
+    def __init__(self, code: int, message: str):
+        super().__init__(f"{message} (status {code})")
+        self.code = code
+
+
+def load(path: str | None = None):
+    """Load liblrar.so; raises if it has not been built."""
+    global _lib
+    with _lock:
+        if _lib is not None and path is None:
+            return _lib
+        p = path or LIB_PATH
+        if not os.path.exists(p):
+            raise RuntimeError(f"{p} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+        lib = ctypes.CDLL(p)
+        vp, i, i64, f32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+        lib.lrar_forward.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, vp]
+        lib.lrar_forward.restype = i
+        lib.lrar_backward.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, i, vp, vp, vp, vp, i, vp, sz, vp]
+        lib.lrar_backward.restype = i
+        lib.lrar_backward_workspace_size.argtypes = [i, i, i64, i, i]
+        lib.lrar_backward_workspace_size.restype = sz
+        lib.lrar_block_accumulate.argtypes = [i, vp, i, vp, i64, f32, f32, vp]
+        lib.lrar_block_accumulate.restype = i
+        lib.lrar_strerror.argtypes = [i]
+        lib.lrar_strerror.restype = ctypes.c_char_p
+        lib.lrar_last_error.argtypes = []
+        lib.lrar_last_error.restype = ctypes.c_char_p
+        lib.lrar_version.argtypes = []
+        lib.lrar_version.restype = i
+        if path is None:
+            _lib = lib
+        return lib
+
+
+def _check(rc: int) -> None:
+    if rc != OK:
+        lib = load()
+        raise LrarError(rc, lib.lrar_last_error().decode() or lib.lrar_strerror(rc).decode())
+
+
+def dtype_code(t: torch.Tensor | None, default: int = F32) -> int:
+    if t is None:
+        return default
+    if t.dtype == torch.bfloat16:
+        return BF16
+    if t.dtype == torch.float32:
+        return F32
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _ptr(t) -> int | None:
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream if torch.cuda.is_available() else None
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _variant(v) -> int:
+    return VARIANTS[v] if isinstance(v, str) else int(v)
+
+
+def forward(variant, values: torch.Tensor, keys: torch.Tensor | None, query: torch.Tensor | None,
+            h: torch.Tensor, lse: torch.Tensor | None = None, n_src: int | None = None, r: int | None = None,
+            eps: float = DEFAULT_EPS, stream=None) -> None:
+    """lrar_forward: h (and lse) of the first n_src sources of the stack `values` [*, T, d]."""
+    variant = _variant(variant)
+    _, T, d = values.shape
+    n = values.shape[0] if n_src is None else n_src
+    if r is None:
+        r = d if variant == FULL else (keys.shape[-1] if variant == PROJECTED else query.numel())
+    _check(load().lrar_forward(variant, dtype_code(values), dtype_code(h), _ptr(values), _ptr(keys), _ptr(query),
+                               n, T, d, r, eps, _ptr(h), _ptr(lse), _stream(stream)))
+
+
+def workspace_size(variant, n_src: int, T: int, d: int, r: int) -> int:
+    return int(load().lrar_backward_workspace_size(_variant(variant), n_src, T, d, r))
+
+
+def backward(variant, values: torch.Tensor, keys: torch.Tensor | None, query: torch.Tensor | None,
+             dh: torch.Tensor, dvalues: torch.Tensor, dq: torch.Tensor, workspace: torch.Tensor,
+             dkeys: torch.Tensor | None = None, h: torch.Tensor | None = None, lse: torch.Tensor | None = None,
+             n_src: int | None = None, r: int | None = None, accumulate: bool = False,
+             eps: float = DEFAULT_EPS, stream=None) -> None:
+    """lrar_backward for the first n_src sources of `values`; gradients go to the
+    first n_src slices of `dvalues` (and `dkeys`)."""
+    variant = _variant(variant)
+    _, T, d = values.shape
+    n = values.shape[0] if n_src is None else n_src
+    if r is None:
+        r = d if variant == FULL else (keys.shape[-1] if variant == PROJECTED else query.numel())
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check(load().lrar_backward(variant, dtype_code(values), dtype_code(dvalues), _ptr(values), _ptr(keys),
+                                _ptr(query), n, T, d, r, eps, _ptr(dh), _ptr(h), dtype_code(h), _ptr(lse),
+                                _ptr(dvalues), _ptr(dkeys), _ptr(dq), int(bool(accumulate)), _ptr(workspace),
+                                ws_bytes, _stream(stream)))
+
+
+def block_accumulate(dst: torch.Tensor, src: torch.Tensor, alpha: float = 1.0, beta: float = 1.0,
+                     stream=None) -> None:
+    """lrar_block_accumulate: dst = beta * dst + alpha * src (beta == 0 does not read dst)."""
+    if dst.numel() != src.numel():
+        raise ValueError("dst and src sizes differ")
+    _check(load().lrar_block_accumulate(dtype_code(dst), _ptr(dst), dtype_code(src), _ptr(src), dst.numel(),
+                                        float(alpha), float(beta), _stream(stream)))
+
+
+def version() -> int:
+    return int(load().lrar_version())

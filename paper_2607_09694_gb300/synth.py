@@ -139,13 +139,17 @@ class SiteInputs:
 
 
 def site(config: str, n: int | None = None, T: int | None = None, r: int | None = None,
-         dtype: str | None = None, device="cpu", query_std: float = Q_STD, seed: int | None = None) -> SiteInputs:
-    """One site of a named workload, optionally at a different n, T, r or dtype."""
+         dtype: str | None = None, device="cpu", query_std: float = Q_STD, seed: int | None = None,
+         variant: str | None = None, d: int | None = None) -> SiteInputs:
+    """One site of a named workload, optionally at a different n, T, r, d,
+    storage type or key variant (full keys force r = d)."""
     c = dict(CONFIGS[config])
+    if variant is not None:
+        c["variant"] = variant
     n = c["n"] if n is None else n
     T = c["T"] if T is None else T
     r = c["r"] if r is None else r
-    d = c["d"]
+    d = c["d"] if d is None else d
     if c["variant"] == "full":
         r = d
     dt = c["dtype"] if dtype is None else dtype

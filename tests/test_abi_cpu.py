@@ -1,0 +1,161 @@
+"""The C ABI library loads, exports every entry point include/lrar.h declares,
+and rejects bad arguments before touching the GPU (no compute calls here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2607_09694_gb300 import build as lrar_build
+from paper_2607_09694_gb300 import lrar
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+FAKE = 1 << 20  # a 16-byte aligned address that is never dereferenced
+EPS = 1e-6
+
+
+@pytest.fixture(scope="module")
+def lib():
+    lrar_build.build()
+    return lrar.load()
+
+
+def _declared():
+    text = open(os.path.join(ROOT, "include", "lrar.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(lrar_[a-z_]+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared()
+    assert set(names) == set(lrar.EXPORTS)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_only_declared_symbols_are_exported(lib):
+    import subprocess
+
+    out = subprocess.run(["nm", "-D", "--defined-only", lrar.LIB_PATH], capture_output=True, text=True).stdout
+    syms = {line.split()[-1] for line in out.splitlines() if " T " in line}
+    assert syms == set(_declared())
+
+
+def test_version_and_strings(lib):
+    assert lib.lrar_version() == 1
+    for code in (0, -1, -2, -3, -4, -5):
+        assert lib.lrar_strerror(code)
+    assert b"unknown" in lib.lrar_strerror(-99)
+
+
+def fwd(lib, variant=1, ind=1, outd=1, values=FAKE, keys=None, query=FAKE, n=4, T=8, d=64, r=4, eps=EPS, h=FAKE,
+        lse=None):
+    return lib.lrar_forward(variant, ind, outd, values, keys, query, n, T, d, r, eps, h, lse, None)
+
+
+def bwd(lib, variant=1, ind=1, gd=1, values=FAKE, keys=None, query=FAKE, n=4, T=8, d=64, r=4, eps=EPS, dh=FAKE,
+        h=None, hd=1, lse=None, dv=FAKE, dk=None, dq=FAKE, acc=0, ws=FAKE, wsb=None):
+    if wsb is None:
+        wsb = lib.lrar_backward_workspace_size(variant, n, T, d, r)
+    return lib.lrar_backward(variant, ind, gd, values, keys, query, n, T, d, r, eps, dh, h, hd, lse, dv, dk, dq, acc,
+                             ws, wsb, None)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(variant=3), lrar.ERR_INVALID_ARG),
+    (dict(ind=2), lrar.ERR_INVALID_ARG),
+    (dict(outd=7), lrar.ERR_INVALID_ARG),
+    (dict(n=0), lrar.ERR_INVALID_ARG),
+    (dict(n=129), lrar.ERR_UNSUPPORTED),
+    (dict(T=-1), lrar.ERR_INVALID_ARG),
+    (dict(r=0), lrar.ERR_INVALID_ARG),
+    (dict(r=65, d=64), lrar.ERR_INVALID_ARG),
+    (dict(variant=0, r=4), lrar.ERR_INVALID_ARG),
+    (dict(eps=0.0), lrar.ERR_INVALID_ARG),
+    (dict(eps=-1.0), lrar.ERR_INVALID_ARG),
+    (dict(eps=float("inf")), lrar.ERR_INVALID_ARG),
+    (dict(eps=float("nan")), lrar.ERR_INVALID_ARG),
+    (dict(values=None), lrar.ERR_INVALID_ARG),
+    (dict(h=None), lrar.ERR_INVALID_ARG),
+    (dict(query=None), lrar.ERR_INVALID_ARG),
+    (dict(variant=2, keys=None), lrar.ERR_INVALID_ARG),
+    (dict(values=FAKE + 8), lrar.ERR_ALIGNMENT),
+    (dict(h=FAKE + 4), lrar.ERR_ALIGNMENT),
+    (dict(query=FAKE + 2), lrar.ERR_ALIGNMENT),
+    (dict(d=60), lrar.ERR_ALIGNMENT),
+    (dict(d=4096, r=16), lrar.ERR_UNSUPPORTED),
+    (dict(ind=0, d=2048, r=16), lrar.ERR_UNSUPPORTED),
+])
+def test_forward_rejects(lib, kw, code):
+    assert fwd(lib, **kw) == code
+    assert lib.lrar_last_error()
+
+
+def test_forward_empty_is_noop(lib):
+    assert fwd(lib, T=0, values=None, h=None) == lrar.OK
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(gd=5), lrar.ERR_INVALID_ARG),
+    (dict(acc=2), lrar.ERR_INVALID_ARG),
+    (dict(dq=None), lrar.ERR_INVALID_ARG),
+    (dict(dv=None), lrar.ERR_INVALID_ARG),
+    (dict(dh=None), lrar.ERR_INVALID_ARG),
+    (dict(variant=2, keys=FAKE, dk=None), lrar.ERR_INVALID_ARG),
+    (dict(variant=0, d=64, r=64, h=FAKE, lse=None), lrar.ERR_INVALID_ARG),
+    (dict(variant=0, d=64, r=64, h=None, lse=FAKE), lrar.ERR_INVALID_ARG),
+    (dict(variant=0, d=64, r=64, h=FAKE, lse=FAKE, hd=3), lrar.ERR_INVALID_ARG),
+    (dict(ws=None), lrar.ERR_WORKSPACE),
+    (dict(wsb=16), lrar.ERR_WORKSPACE),
+    (dict(ws=FAKE + 8), lrar.ERR_ALIGNMENT),
+    (dict(dv=FAKE + 2), lrar.ERR_ALIGNMENT),
+    (dict(n=200), lrar.ERR_UNSUPPORTED),
+])
+def test_backward_rejects(lib, kw, code):
+    assert bwd(lib, **kw) == code
+
+
+def test_workspace_size_is_device_independent(lib):
+    assert lib.lrar_backward_workspace_size(1, 49, 16384, 1024, 16) == 1024 * 16 * 4
+    assert lib.lrar_backward_workspace_size(0, 49, 16384, 1024, 1024) == 1024 * 1024 * 4
+    assert lib.lrar_backward_workspace_size(2, 1, 1, 64, 0) == 0
+
+
+def test_block_accumulate_rejects(lib):
+    f = lib.lrar_block_accumulate
+    assert f(3, FAKE, 1, FAKE, 10, 1.0, 1.0, None) == lrar.ERR_INVALID_ARG
+    assert f(1, FAKE, 1, FAKE, -1, 1.0, 1.0, None) == lrar.ERR_INVALID_ARG
+    assert f(1, None, 1, FAKE, 10, 1.0, 1.0, None) == lrar.ERR_INVALID_ARG
+    assert f(0, FAKE + 2, 1, FAKE, 10, 1.0, 1.0, None) == lrar.ERR_ALIGNMENT
+    assert f(1, FAKE, 1, FAKE, 10, float("nan"), 1.0, None) == lrar.ERR_INVALID_ARG
+    assert f(1, None, 1, None, 0, 1.0, 1.0, None) == lrar.OK
+
+
+def test_last_error_is_per_thread(lib):
+    import threading
+
+    assert fwd(lib, n=0) == lrar.ERR_INVALID_ARG
+    seen = {}
+
+    def other():
+        seen["msg"] = lib.lrar_last_error()
+
+    t = threading.Thread(target=other)
+    t.start()
+    t.join()
+    assert seen["msg"] == b""
+    assert b"n_src" in lib.lrar_last_error()
+
+
+def test_binding_raises_typed_error(lib):
+    import torch
+
+    v = torch.zeros(2, 4, 64)
+    with pytest.raises(lrar.LrarError) as ei:
+        lrar.forward("sliced", v, None, torch.zeros(4), torch.zeros(4, 64), n_src=0)
+    assert ei.value.code == lrar.ERR_INVALID_ARG
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    with pytest.raises(RuntimeError, match="missing"):
+        lrar.load(str(tmp_path / "nope.so"))

@@ -1,0 +1,107 @@
+"""Parity at the workloads' full sizes, in the configuration the benchmark
+times (bf16 values, bf16 h, bf16 gradients accumulated into a live buffer).
+
+Every h / lse / dvalues row of a sample of tokens (edges, warp and CTA
+boundaries of the persistent grid, random tokens) is compared with the
+oracle; dq, a sum over all T tokens, is compared with the oracle's sum over
+all T tokens.
+"""
+import numpy as np
+import pytest
+import torch
+
+import gpu_helpers as H
+import oracle
+from paper_2607_09694_gb300 import lrar, synth
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+
+@pytest.fixture(scope="module")
+def slr_values():
+    c = synth.CONFIGS["slr"]
+    return synth.values(c["n"], c["T"], c["d"], c["seed"], "bf16", c["scale"])
+
+
+@pytest.fixture(scope="module")
+def plr_values():
+    c = synth.CONFIGS["plr"]
+    return synth.values(c["n"], c["T"], c["d"], c["seed"], "bf16")
+
+
+def _site(config, values, r=None, variant=None):
+    c = synth.CONFIGS[config]
+    variant = variant or c["variant"]
+    n, T, d = values.shape
+    r = d if variant == "full" else (c["r"] if r is None else r)
+    seed = c["seed"]
+    keys = synth.keys(n, T, r, seed, "bf16") if variant == "projected" else None
+    q = synth.queries(1, r, seed)[0].contiguous()
+    dh = synth.upstream(T, d, seed, "bf16")
+    return synth.SiteInputs(variant, n, T, d, r, values, keys, q, dh)
+
+
+def _bench_like(si):
+    """Accumulate into a buffer that already holds a per-source constant i/64
+    (exact in bf16), as the all-sites sweep does."""
+    n = si.n
+    dv0 = torch.empty(n, si.T, si.d, dtype=torch.bfloat16)
+    for i in range(n):
+        dv0[i].fill_(i / 64.0)
+    init = dict(dvalues=dv0, dq=torch.zeros(si.d if si.variant == "full" else si.r))
+    if si.keys is not None:
+        init["dkeys"] = torch.zeros(si.keys.shape, dtype=torch.bfloat16)
+    toks = H.sample_tokens(si.T)
+    got = H.run_gpu(si, "bf16", "bf16", accumulate=True, init=init, tokens=toks)
+    ov = H.ORACLE_VARIANT[si.variant]
+    f = oracle.forward(ov, si.values, si.keys, si.query, H.EPS, r=si.r, tokens=toks)
+    b = oracle.backward(ov, si.values, si.keys, si.query, H.EPS, si.dh, r=si.r, tokens=toks)
+    dq_all = oracle.backward(ov, si.values, si.keys, si.query, H.EPS, si.dh, r=si.r, want_dvalues=False)["dq"]
+    H.assert_bf16_rounded("h", got["h"], f["h"])
+    H.assert_abs("lse", got["lse"], f["lse"], 1e-4)
+    dv_ref = b["dvalues"] + (np.arange(si.n) / 64.0)[:, None, None]
+    H.assert_bf16_rounded("dvalues", got["dvalues"], dv_ref)
+    if si.keys is not None:
+        H.assert_bf16_rounded("dkeys", got["dkeys"], b["dkeys"])
+    H.assert_rms("dq", got["dq"], dq_all)
+    return got, f, b
+
+
+def test_slr_d1024_n49_bench_configuration(slr_values):
+    _bench_like(_site("slr", slr_values))
+
+
+def test_slr_d1024_n49_fp32_outputs(slr_values):
+    si = _site("slr", slr_values)
+    toks = H.sample_tokens(si.T, seed=1)
+    got = H.run_gpu(si, "f32", "f32", tokens=toks)
+    ref = H.run_oracle(si, tokens=toks)
+    H.assert_rms("h", got["h"], ref["h"])
+    H.assert_rms("dvalues", got["dvalues"], ref["dvalues"])
+
+
+def test_full_attnres_d1024_n49(slr_values):
+    _bench_like(_site("full", slr_values, variant="full"))
+
+
+@pytest.mark.parametrize("r", [4, 8, 16, 32, 64])
+def test_plr_d1024_n49_rank_sweep(r, plr_values):
+    _bench_like(_site("plr", plr_values, r=r))
+
+
+def test_all_sites_prefixes(slr_values):
+    """A few sites of the 24-layer sweep (n = 2, 25, 48) read prefixes of the stack."""
+    si = _site("slr", slr_values)
+    toks = H.sample_tokens(si.T, k=16, seed=2)
+    for n in (2, 25, 48):
+        got = H.run_gpu(si, "f32", "f32", n_src=n, tokens=toks)
+        ref = H.run_oracle(si, tokens=toks, n_src=n)
+        H.assert_rms(f"h[n={n}]", got["h"], ref["h"])
+        H.assert_rms(f"dvalues[n={n}]", got["dvalues"][:n], ref["dvalues"])
+        assert np.all(np.isnan(got["dvalues"][n:]))
+
+
+def test_slr_d2048_n65_t32768():
+    c = synth.CONFIGS["slr_large"]
+    vals = synth.values(c["n"], c["T"], c["d"], c["seed"], "bf16")
+    _bench_like(_site("slr_large", vals))

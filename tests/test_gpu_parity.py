@@ -1,0 +1,237 @@
+"""GPU path (C ABI -> CUDA kernels) against the fp64 oracle on the same seeded
+inputs.
+
+Tolerances: fp32 storage -> max abs error <= 1e-4 on every output; bf16
+inputs with fp32 outputs -> max abs error <= 1e-2 x RMS of the oracle tensor;
+bf16 outputs -> within one bf16 spacing of the exact value (rounding a value
+of several RMS to bf16 alone can exceed 1e-2 x RMS, so the rounding is checked
+directly).  lse is fp32 in every mode: <= 1e-4 absolute.
+"""
+import numpy as np
+import pytest
+import torch
+
+import gpu_helpers as H
+from paper_2607_09694_gb300 import lrar, synth
+
+pytestmark = pytest.mark.gpu
+
+
+def _check(si, got, ref, n, mode, toks=None, init=None, ulps=1.0):
+    sel = (lambda a: a) if toks is None else (lambda a: a[:, toks] if a.ndim == 3 else a[toks])
+    pairs = [("h", sel(got["h"]) if toks is not None else got["h"], ref["h"])]
+    dv_got = got["dvalues"][:n]
+    if toks is not None:
+        dv_got = dv_got[:, toks]
+    dv_ref = ref["dvalues"] + (0 if init is None else sel(init["dvalues"][:n].double().numpy()))
+    pairs.append(("dvalues", dv_got, dv_ref))
+    if si.variant == "projected":
+        dk_got = got["dkeys"][:n] if toks is None else got["dkeys"][:n][:, toks]
+        dk_ref = ref["dkeys"] + (0 if init is None else sel(init["dkeys"][:n].double().numpy()))
+        pairs.append(("dkeys", dk_got, dk_ref))
+    dq_ref = ref["dq"] + (0 if init is None else init["dq"].double().numpy())
+    lse_got = got["lse"] if toks is None else got["lse"][toks]
+    H.assert_abs("lse", lse_got, ref["lse"], 1e-4)
+    for name, g, r in pairs:
+        if mode == "f32":
+            H.assert_abs(name, g, r, 1e-4)
+        elif mode == "rms":
+            H.assert_rms(name, g, r)
+        else:
+            H.assert_bf16_rounded(name, g, r, ulps)
+    if mode == "f32":
+        H.assert_abs("dq", got["dq"], dq_ref, 1e-4)
+    else:
+        H.assert_rms("dq", got["dq"], dq_ref)
+
+
+def _init(si, seed=99, dtype=torch.float32):
+    g = torch.Generator().manual_seed(seed)
+    rq = si.d if si.variant == "full" else si.r
+    out = dict(dvalues=torch.randn(si.values.shape, generator=g).to(dtype),
+               dq=torch.randn(rq, generator=g))
+    if si.keys is not None:
+        out["dkeys"] = torch.randn(si.keys.shape, generator=g).to(dtype)
+    return out
+
+
+# ----------------------------------------------------------------- tiny ----
+@pytest.mark.parametrize("variant", ["sliced", "projected", "full"])
+@pytest.mark.parametrize("accumulate", [False, True])
+def test_tiny_fp32(variant, accumulate):
+    """T=256, d=64, n=8, r=4 (full: r=64), fp32 storage."""
+    si = synth.site("tiny", variant=variant)
+    init = _init(si) if accumulate else None
+    got = H.run_gpu(si, "f32", "f32", accumulate=accumulate, init=init)
+    ref = H.run_oracle(si)
+    _check(si, got, ref, si.n, "f32", init=init)
+
+
+# ------------------------------------------------- several tiles, ragged --
+@pytest.mark.parametrize("variant,r", [("sliced", 16), ("projected", 32), ("full", 1024)])
+def test_bf16_ragged_fp32_outputs(variant, r):
+    """d=1024, n=49, T=1000 (not a multiple of the 8-token CTA tile)."""
+    si = synth.site("slr", variant=variant, T=1000, r=r)
+    _check(si, H.run_gpu(si, "f32", "f32"), H.run_oracle(si), si.n, "rms")
+
+
+@pytest.mark.parametrize("variant,r", [("sliced", 16), ("projected", 32), ("full", 1024)])
+def test_bf16_outputs_round_once(variant, r):
+    si = synth.site("slr", variant=variant, T=777, r=r)
+    _check(si, H.run_gpu(si, "bf16", "bf16"), H.run_oracle(si), si.n, "ulp")
+
+
+@pytest.mark.parametrize("variant,r", [("sliced", 16), ("projected", 32), ("full", 1024)])
+def test_bf16_accumulate(variant, r):
+    si = synth.site("slr", variant=variant, T=515, r=r)
+    init = _init(si, dtype=torch.bfloat16)
+    got = H.run_gpu(si, "bf16", "bf16", accumulate=True, init=init)
+    _check(si, got, H.run_oracle(si), si.n, "ulp", init=init)
+
+
+# ------------------------------------------------------------ edge cases --
+@pytest.mark.parametrize("n", [1, 2, 17, 33, 128])
+def test_source_counts(n):
+    si = synth.site("slr", n=n, T=300)
+    _check(si, H.run_gpu(si, "f32", "f32"), H.run_oracle(si), n, "rms")
+
+
+@pytest.mark.parametrize("T", [1, 7, 33])
+def test_tiny_token_counts(T):
+    si = synth.site("slr", n=5, T=T)
+    _check(si, H.run_gpu(si, "f32", "f32"), H.run_oracle(si), si.n, "rms")
+
+
+@pytest.mark.parametrize("r", [1, 4, 8, 64, 100])
+@pytest.mark.parametrize("grad", ["f32", "bf16"])
+def test_sliced_key_widths(r, grad):
+    """r = 1, 4 and 100 put the key slice inside a 16-byte vector (scalar key reads,
+    partly-written boundary vector); 8 and 64 are vector-aligned."""
+    si = synth.site("slr", n=9, T=200, r=r)
+    got = H.run_gpu(si, "f32", grad)
+    ref = H.run_oracle(si)
+    if grad == "f32":
+        _check(si, got, ref, si.n, "rms")
+    else:
+        # the boundary vector's key elements are rounded twice (value pass, key pass)
+        _check(si, got, ref, si.n, "ulp", ulps=1.5)
+
+
+@pytest.mark.parametrize("r", [1, 4, 8, 16, 64])
+def test_projected_key_widths(r):
+    si = synth.site("plr", n=12, T=260, r=r)
+    _check(si, H.run_gpu(si, "f32", "f32"), H.run_oracle(si), si.n, "rms")
+
+
+@pytest.mark.parametrize("d", [64, 200, 1016, 2048])
+@pytest.mark.parametrize("variant", ["sliced", "full"])
+def test_widths(d, variant):
+    """Row widths that do not fill a lane's vectors, and the widest row (V = 8)."""
+    si = synth.site("slr", variant=variant, n=6, T=150, d=d, r=min(16, d))
+    _check(si, H.run_gpu(si, "f32", "f32"), H.run_oracle(si), si.n, "rms")
+
+
+@pytest.mark.parametrize("d", [128, 512, 1024])
+@pytest.mark.parametrize("variant", ["sliced", "projected", "full"])
+def test_fp32_widths(d, variant):
+    si = synth.site("tiny", variant=variant, n=6, T=70, d=d, r=min(8, d) if variant != "full" else None)
+    _check(si, H.run_gpu(si, "f32", "f32"), H.run_oracle(si), si.n, "f32")
+
+
+def test_single_source_is_exact_identity():
+    """n = 1 with no query: h = o_0 and dvalues = dh exactly, dq = 0."""
+    si = synth.site("slr", n=1, T=100)
+    dev = torch.device("cuda")
+    v, dh = si.values.to(dev), si.dh.to(dev)
+    h = torch.empty(si.T, si.d, dtype=torch.bfloat16, device=dev)
+    lrar.forward("sliced", v, None, None, h, None, r=si.r)
+    dv = torch.empty_like(v)
+    dq = torch.full((si.r,), 7.0, device=dev)
+    ws = torch.empty(lrar.workspace_size("sliced", 1, si.T, si.d, si.r) // 4, device=dev)
+    lrar.backward("sliced", v, None, None, dh, dv, dq, ws, r=si.r)
+    torch.cuda.synchronize()
+    assert torch.equal(h.cpu(), si.values[0])
+    assert torch.equal(dv[0].cpu(), si.dh)
+    assert torch.count_nonzero(dq).item() == 0
+
+
+def test_empty_batch():
+    dev = torch.device("cuda")
+    v = torch.empty(3, 0, 64, device=dev)
+    h = torch.empty(0, 64, device=dev)
+    q = torch.zeros(4, device=dev)
+    lrar.forward("sliced", v, None, q, h, r=4)
+    dq = torch.full((4,), 5.0, device=dev)
+    ws = torch.empty(lrar.workspace_size("sliced", 3, 0, 64, 4) // 4, device=dev)
+    lrar.backward("sliced", v, None, q, h, v, dq, ws, r=4, accumulate=True)
+    torch.cuda.synchronize()
+    assert torch.all(dq == 5.0)
+    lrar.backward("sliced", v, None, q, h, v, dq, ws, r=4, accumulate=False)
+    torch.cuda.synchronize()
+    assert torch.all(dq == 0.0)
+
+
+def test_sliced_rank_d_matches_full_on_gpu():
+    """§3.4: S-LR with r = d is AttnRes; the two kernels agree with each other."""
+    si_s = synth.site("slr", variant="sliced", n=7, T=90, d=256, r=256)
+    si_f = synth.site("slr", variant="full", n=7, T=90, d=256)
+    a = H.run_gpu(si_s, "f32", "f32")
+    b = H.run_gpu(si_f, "f32", "f32")
+    for k in ("h", "lse", "dvalues", "dq"):
+        H.assert_rms(k, a[k], b[k], 1e-4)
+    _check(si_s, a, H.run_oracle(si_s), si_s.n, "rms")
+
+
+def test_prefix_of_a_larger_stack():
+    """Site t reads the first t slices of the stacked buffer; later slices are untouched."""
+    si = synth.site("slr", n=20, T=128)
+    got = H.run_gpu(si, "f32", "f32", n_src=11)
+    ref = H.run_oracle(si, n_src=11)
+    _check(si, got, ref, 11, "rms")
+    assert np.all(np.isnan(got["dvalues"][11:]))
+
+
+def test_deterministic():
+    si = synth.site("slr", n=49, T=2000)
+    a = H.run_gpu(si, "bf16", "bf16")
+    b = H.run_gpu(si, "bf16", "bf16")
+    for k in ("h", "lse", "dvalues", "dq"):
+        assert np.array_equal(a[k], b[k]), k
+
+
+def test_side_stream():
+    si = synth.site("slr", n=10, T=333)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        got = H.run_gpu(si, "f32", "f32", stream=s)
+    _check(si, got, H.run_oracle(si), si.n, "rms")
+
+
+@pytest.mark.parametrize("variant", ["sliced", "projected", "full"])
+def test_guard_canaries(variant):
+    """Outputs live inside larger buffers whose margins hold a sentinel; no
+    kernel writes outside its output."""
+    si = synth.site("slr", variant=variant, n=5, T=77, d=256, r=16 if variant != "full" else None)
+    dev = torch.device("cuda")
+    pad = 4096
+    sentinel = -12345.0
+
+    def guarded(numel, dtype):
+        buf = torch.full((numel + 2 * pad,), sentinel, dtype=dtype, device=dev)
+        return buf, buf[pad:pad + numel]
+
+    T, d, r, n = si.T, si.d, si.r, si.n
+    v, q, dh = si.values.to(dev), si.query.to(dev), si.dh.to(dev)
+    k = si.keys.to(dev) if si.keys is not None else None
+    hb, h = guarded(T * d, torch.float32)
+    lb, lse = guarded(T, torch.float32)
+    vb, dv = guarded(n * T * d, torch.float32)
+    qb, dq = guarded(d if variant == "full" else r, torch.float32)
+    kb, dk = guarded(n * T * r, torch.float32)
+    ws = torch.empty(lrar.workspace_size(variant, n, T, d, r) // 4, device=dev)
+    lrar.forward(variant, v, k, q, h.view(T, d), lse, r=r)
+    lrar.backward(variant, v, k, q, dh, dv.view(n, T, d), dq, ws, dkeys=dk.view(n, T, r) if k is not None else None,
+                  h=h.view(T, d), lse=lse, r=r)
+    torch.cuda.synchronize()
+    for buf in (hb, lb, vb, qb, kb):
+        assert torch.all(buf[:pad] == sentinel) and torch.all(buf[-pad:] == sentinel)
