@@ -107,7 +107,11 @@ size_t lrar_backward_workspace_size(int variant, int n_src, int64_t T, int d, in
  *   grad_dtype element type of dvalues and dkeys
  *   dh         [T, d] in_dtype
  *   h          [T, d] h_dtype, the forward output; required for LRAR_FULL
- *              (gbar = <dh, h> lets FULL finish in one pass), ignored otherwise
+ *              (gbar = <dh, h> lets FULL finish in one pass), ignored otherwise.
+ *              gbar is exact for a float32 h; a bfloat16 h carries its rounding
+ *              into gbar (as FlashAttention's backward does with its stored
+ *              output): at most alpha_i rho_i |q - (s_i/d) kbar_i| sum_j |dh_j|
+ *              ulp(h_j)/2 per gradient element
  *   h_dtype    element type of h
  *   lse        [T] float32 from the forward; required for LRAR_FULL, ignored otherwise
  *   dvalues    [n_src, T, d] grad_dtype, written (accumulate = 0) or added into

@@ -110,10 +110,14 @@ __device__ __forceinline__ void lr_route_b(const BwdParams &p, const Tin *__rest
 }
 
 // One value row of the low-rank backward (phase 2): returns the lane's part of g_i.
+// Vectors wholly inside the key slice (e >= skip0) are left to the key pass; in
+// the one vector that straddles the slice start (tail0), the slice elements keep
+// their old value here and receive alpha_i dh + dL/dk_i in the key pass, so every
+// element is rounded once.
 template <typename Tin, typename Tg, int V>
 __device__ __forceinline__ float lr_bwd_row(const Frag<Tin, VecE<Tin>::value> *f,
                                             const Frag<Tg, VecE<Tin>::value> *old, const float *dhf, float a,
-                                            Tg *__restrict__ drow, int skip0, int lane, int accumulate) {
+                                            Tg *__restrict__ drow, int tail0, int skip0, int lane, int accumulate) {
     constexpr int E = VecE<Tin>::value;
     float gp = 0.f;
 #pragma unroll
@@ -123,14 +127,20 @@ __device__ __forceinline__ float lr_bwd_row(const Frag<Tin, VecE<Tin>::value> *f
         f[v].get(o);
 #pragma unroll
         for (int t = 0; t < E; ++t) gp = fmaf(dhf[v * E + t], o[t], gp);
-        if (e < skip0) {  // vectors wholly inside the key slice are written by the key pass
+        if (e < skip0) {
             float w[E];
             if (accumulate) old[v].get(w);
             else
 #pragma unroll
                 for (int t = 0; t < E; ++t) w[t] = 0.f;
+            if (e + E <= tail0) {
 #pragma unroll
-            for (int t = 0; t < E; ++t) w[t] = fmaf(a, dhf[v * E + t], w[t]);
+                for (int t = 0; t < E; ++t) w[t] = fmaf(a, dhf[v * E + t], w[t]);
+            } else {
+#pragma unroll
+                for (int t = 0; t < E; ++t)
+                    if (e + t < tail0) w[t] = fmaf(a, dhf[v * E + t], w[t]);
+            }
             Frag<Tg, E> out;
             out.set(w);
             out.store(drow + e);
@@ -202,7 +212,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 const float gp = lr_bwd_row<Tin, Tg, V>(f[u], old[u], dhf, a_s[i + u],
-                                                        dvalues + (int64_t)(i + u) * src_stride + row_off,
+                                                        dvalues + (int64_t)(i + u) * src_stride + row_off, tail0,
                                                         p.d < skip0 ? p.d : skip0, lane, p.accumulate);
                 const float g = warp_sum(gp);
                 if (lane == 0) g_s[i + u] = g;
@@ -221,7 +231,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
                 else old[v].zero();
             }
             const float gp = lr_bwd_row<Tin, Tg, V>(f, old, dhf, a_s[i], dvalues + (int64_t)i * src_stride + row_off,
-                                                    p.d < skip0 ? p.d : skip0, lane, p.accumulate);
+                                                    tail0, p.d < skip0 ? p.d : skip0, lane, p.accumulate);
             const float g = warp_sum(gp);
             if (lane == 0) g_s[i] = g;
         }
@@ -249,11 +259,10 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
                 const float dk = ds * rho * (qj - s * p.inv_r * kbar);
                 dqj = fmaf(ds, kbar, dqj);
                 if (p.sliced) {
+                    // c < skip0: the value pass stored the old value (or 0) here
                     Tg *dp = dvalues + (int64_t)k * src_stride + row_off + c;
-                    float w;
-                    if (c < skip0) w = to_f(*dp) + dk;  // written by the value pass
-                    else w = (p.accumulate ? to_f(*dp) : 0.f) + fmaf(a_s[k], dh_c, dk);
-                    *dp = from_f<Tg>(w);
+                    const float base = (c < skip0 || p.accumulate) ? to_f(*dp) : 0.f;
+                    *dp = from_f<Tg>(base + fmaf(a_s[k], dh_c, dk));
                 } else {
                     Tg *dp = dkeys + ((int64_t)k * p.T + x) * p.r + j;
                     *dp = from_f<Tg>(p.accumulate ? to_f(*dp) + dk : dk);

@@ -29,6 +29,15 @@ def assert_abs(name, got, ref, tol=1e-4):
     assert e <= tol, f"{name}: max abs err {e:.3e} > {tol:.1e}"
 
 
+def assert_f32(name, got, ref):
+    """fp32 storage and arithmetic: 1e-4 absolute, widened by 1e-6 relative to
+    the largest exact value for sums whose magnitude makes a flat 1e-4 finer
+    than fp32 resolution (fp32 spacing is 1.2e-7 relative)."""
+    ref = np.asarray(ref, dtype=np.float64)
+    scale = float(np.max(np.abs(ref))) if ref.size else 0.0
+    assert_abs(name, got, ref, 1e-4 + 1e-6 * scale)
+
+
 def assert_rms(name, got, ref, frac=1e-2):
     e, r = max_err(got, ref), rms(ref)
     assert e <= frac * r, f"{name}: max abs err {e:.3e} > {frac:g} x RMS {r:.3e}"
