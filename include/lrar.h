@@ -129,6 +129,33 @@ int lrar_backward(int variant, int in_dtype, int grad_dtype, const void *values,
                   int accumulate, void *workspace, size_t workspace_bytes, void *stream);
 
 /*
+ * lrar_backward for callers that cannot allocate device memory.  The paper has
+ * no counterpart: this is a deployment variant of lrar_backward.
+ *
+ * Some callers cannot hand lrar_backward a workspace: plugin callbacks of
+ * inference or training runtimes that must not allocate while they run,
+ * services held to a fixed device-memory budget, and C hosts that receive
+ * device pointers from another component and have no device allocator.  This
+ * call takes the same arguments minus the workspace and allocates nothing: its
+ * scratch is a fixed 4 MiB array compiled into the library, which every GPU
+ * that loads the library holds until the process exits.
+ *   - Problems whose workspace would exceed 4 MiB (lrar_backward_workspace_size()
+ *     > 4 MiB, i.e. a dq width -- r, or d for LRAR_FULL -- above 1024) are
+ *     rejected with LRAR_ERR_UNSUPPORTED before anything runs.
+ *   - The first call on each device looks up the scratch's device address with
+ *     that device current; make that first call before any stream capture.
+ *   - All calls on a device share the one scratch array.  None of it needs to
+ *     start at zero (every partial sum is written before it is read), but calls
+ *     that may run at the same time on the GPU (different streams, or host
+ *     threads without ordering between them) race on it: serialise them.
+ * Results, errors and all other rules are those of lrar_backward.
+ */
+int lrar_backward_noalloc(int variant, int in_dtype, int grad_dtype, const void *values, const void *keys,
+                          const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh,
+                          const void *h, int h_dtype, const float *lse, void *dvalues, void *dkeys, float *dq,
+                          int accumulate, void *stream);
+
+/*
  * Block AttnRes source assembly (§3.1, Eq. 5-6) and its gradient fan-out:
  *   dst[e] = beta * dst[e] + alpha * src[e]   for e = 0..count-1
  * beta == 0 does not read dst (opens a new block summary: dst = alpha * src).

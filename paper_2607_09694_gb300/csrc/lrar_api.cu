@@ -74,6 +74,8 @@ std::unordered_map<OccKey, int, OccHash> g_occ;  // (kernel, device, block, smem
 
 namespace lrar {
 
+int record_error(int code, const char *message) { return fail(code, "%s", message); }
+
 int max_width(int in_dtype) { return 32 * 8 * VecE<float>::value * (in_dtype == LRAR_BF16 ? 2 : 1); }
 
 int persistent_grid(const void *kernel, int threads, size_t smem, int64_t work_ctas, int cap) {

@@ -42,6 +42,9 @@ struct BwdArgs {
     float *partials;  // workspace: [kMaxPartials][rq] floats
 };
 
+// Sets the calling thread's lrar_last_error() message; returns `code`.
+int record_error(int code, const char *message);
+
 // Largest d one warp covers (the kernels keep a whole token row per warp).
 int max_width(int in_dtype);
 

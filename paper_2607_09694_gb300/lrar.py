@@ -25,7 +25,7 @@ ERR_INVALID_ARG, ERR_ALIGNMENT, ERR_UNSUPPORTED, ERR_CUDA, ERR_WORKSPACE = -1, -
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "liblrar.so")
 EXPORTS = ("lrar_forward", "lrar_backward", "lrar_backward_workspace_size", "lrar_block_accumulate",
-           "lrar_strerror", "lrar_last_error", "lrar_version")
+           "lrar_strerror", "lrar_last_error", "lrar_version", "lrar_backward_noalloc")
 
 _lock = threading.Lock()
 _lib = None
@@ -52,6 +52,8 @@ def load(path: str | None = None):
         lib.lrar_forward.restype = i
         lib.lrar_backward.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, i, vp, vp, vp, vp, i, vp, sz, vp]
         lib.lrar_backward.restype = i
+        lib.lrar_backward_noalloc.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, i, vp, vp, vp, vp, i, vp]
+        lib.lrar_backward_noalloc.restype = i
         lib.lrar_backward_workspace_size.argtypes = [i, i, i64, i, i]
         lib.lrar_backward_workspace_size.restype = sz
         lib.lrar_block_accumulate.argtypes = [i, vp, i, vp, i64, f32, f32, vp]
@@ -137,6 +139,24 @@ def backward(variant, values: torch.Tensor, keys: torch.Tensor | None, query: to
                                 _ptr(query), n, T, d, r, eps, _ptr(dh), _ptr(h), dtype_code(h), _ptr(lse),
                                 _ptr(dvalues), _ptr(dkeys), _ptr(dq), int(bool(accumulate)), _ptr(workspace),
                                 ws_bytes, _stream(stream)))
+
+
+def backward_noalloc(variant, values: torch.Tensor, keys: torch.Tensor | None, query: torch.Tensor | None,
+                     dh: torch.Tensor, dvalues: torch.Tensor, dq: torch.Tensor, dkeys: torch.Tensor | None = None,
+                     h: torch.Tensor | None = None, lse: torch.Tensor | None = None, n_src: int | None = None,
+                     r: int | None = None, accumulate: bool = False, eps: float = DEFAULT_EPS, stream=None) -> None:
+    """lrar_backward_noalloc: lrar_backward without a workspace, for callers
+    that cannot allocate device memory (scratch is the library's fixed 4 MiB
+    array per device; calls that may overlap on the GPU race on it)."""
+    variant = _variant(variant)
+    _, T, d = values.shape
+    n = values.shape[0] if n_src is None else n_src
+    if r is None:
+        r = d if variant == FULL else (keys.shape[-1] if variant == PROJECTED else query.numel())
+    _check(load().lrar_backward_noalloc(variant, dtype_code(values), dtype_code(dvalues), _ptr(values), _ptr(keys),
+                                        _ptr(query), n, T, d, r, eps, _ptr(dh), _ptr(h), dtype_code(h), _ptr(lse),
+                                        _ptr(dvalues), _ptr(dkeys), _ptr(dq), int(bool(accumulate)),
+                                        _stream(stream)))
 
 
 def block_accumulate(dst: torch.Tensor, src: torch.Tensor, alpha: float = 1.0, beta: float = 1.0,
