@@ -150,7 +150,7 @@ def site_bytes():
 
 
 class Workload:
-    def __init__(self, device, T=T_TOK):
+    def __init__(self, device, T=T_TOK, n_sites=N_SITES):
         import torch
 
         from paper_2607_09694_gb300 import lrar, synth
@@ -158,14 +158,15 @@ class Workload:
         self.torch, self.lrar = torch, lrar
         self.dev = device
         self.T = T
-        self.values = synth.values(N_SITES, T, D, SEED, "bf16", (0.5, 2.0), device=device)
-        self.queries = synth.queries(N_SITES, R, SEED, device=device)      # row t-1: query of site t
-        self.dh = synth.upstream(T, D, SEED, "bf16", sites=N_SITES, device=device)  # row t-1: dL/dh_t
-        self.h = torch.empty(N_SITES, T, D, dtype=torch.bfloat16, device=device)
-        self.lse = torch.empty(N_SITES, T, dtype=torch.float32, device=device)
-        self.dvalues = torch.empty(N_SITES, T, D, dtype=torch.bfloat16, device=device)
-        self.dq = torch.empty(N_SITES, R, dtype=torch.float32, device=device)
-        self.ws = torch.empty(lrar.workspace_size("sliced", N_SITES, T, D, R) // 4, dtype=torch.float32,
+        ns = n_sites
+        self.values = synth.values(ns, T, D, SEED, "bf16", (0.5, 2.0), device=device)
+        self.queries = synth.queries(ns, R, SEED, device=device)      # row t-1: query of site t
+        self.dh = synth.upstream(T, D, SEED, "bf16", sites=ns, device=device)  # row t-1: dL/dh_t
+        self.h = torch.empty(ns, T, D, dtype=torch.bfloat16, device=device)
+        self.lse = torch.empty(ns, T, dtype=torch.float32, device=device)
+        self.dvalues = torch.zeros(ns, T, D, dtype=torch.bfloat16, device=device)
+        self.dq = torch.empty(ns, R, dtype=torch.float32, device=device)
+        self.ws = torch.empty(lrar.workspace_size("sliced", ns, T, D, R) // 4, dtype=torch.float32,
                               device=device)
 
     def step(self, events=None):
@@ -329,6 +330,17 @@ def run_ours(args):
     site49["frac"] = site49["fwd_bwd_gbs"] / peak
     site49["tokens_per_s"] = T_TOK / ((fwd_t[-1] + bwd_t[-1]) / 1e3)
 
+    # the headline site on its own: n = 49, accumulate = 1 (every site but the
+    # last accumulates), forward and backward each timed with CUDA events
+    hf, hb = time_site(wl, N_SITES, True, 20)
+    from paper_2607_09694_gb300 import sites as _sites
+
+    hfb = _sites.forward_bytes(_sites.SiteShape("sliced", N_SITES, T_TOK, D, R))
+    hbb = _sites.backward_bytes(_sites.SiteShape("sliced", N_SITES, T_TOK, D, R, accumulate=1))
+    headline = {"n_src": N_SITES, "accumulate": 1, "fwd_ms": hf, "bwd_ms": hb, "fwd_gbs": hfb / hf / 1e6,
+                "bwd_gbs": hbb / hb / 1e6, "fwd_bwd_gbs": (hfb + hbb) / (hf + hb) / 1e6,
+                "frac": (hfb + hbb) / (hf + hb) / 1e6 / peak, "tokens_per_s": T_TOK / ((hf + hb) / 1e3)}
+
     # end to end through the public API with host buffers
     e2e = run_e2e(wl, args, dist, dev, step_bytes, world)
 
@@ -352,7 +364,8 @@ def run_ours(args):
                    "bytes_per_step": step_bytes},
         "hbm_frac": value / world / peak,
         "tokens_per_s_per_site": world * T_TOK * N_SITES / (elapsed / args.steps),
-        "site49": site49,
+        "site49_in_sweep": site49,
+        "headline_site": headline,
         "roofline": {"bound": "hbm", "achieved": dom_gbs, "peak": peak, "unit": "GB/s",
                      "frac": dom_gbs / peak, "traffic": traffic, "kernel": dominant,
                      "algorithmic_bytes_per_launch": dom_bytes / dom_launches,
@@ -368,6 +381,47 @@ def run_ours(args):
         print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()
+
+
+def time_site(wl, n: int, accumulate: bool, reps: int):
+    """Median ms of one site's forward and backward (first n sources), timed
+    separately with CUDA events on the launching stream."""
+    import torch
+
+    lrar = wl.lrar
+    q = wl.queries[n - 1] if n > 1 else None
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(reps)]
+    for e in evs:  # back to back: the host stays ahead of the GPU, so no launch gaps are timed
+        e[0].record()
+        lrar.forward(lrar.SLICED, wl.values, None, q, wl.h[n - 1], wl.lse[n - 1], n_src=n, r=R, eps=EPS)
+        e[1].record()
+        lrar.backward(lrar.SLICED, wl.values, None, q, wl.dh[n - 1], wl.dvalues, wl.dq[n - 1], wl.ws, n_src=n, r=R,
+                      accumulate=accumulate, eps=EPS)
+        e[2].record()
+    torch.cuda.synchronize()
+    f_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    b_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    return statistics.median(f_ms), statistics.median(b_ms)
+
+
+def run_profile_site(args):
+    """Small single-site case for profilers: --profile-site n, --tokens T."""
+    import torch
+
+    from __graft_entry__ import build
+    from paper_2607_09694_gb300 import sites
+
+    build()
+    torch.cuda.set_device(0)
+    wl = Workload(torch.device("cuda", 0), T=args.tokens, n_sites=args.profile_site)
+    n = args.profile_site
+    for _ in range(args.warmup):
+        time_site(wl, n, True, 1)
+    f, b = time_site(wl, n, True, args.steps)
+    fb = sites.forward_bytes(sites.SiteShape("sliced", n, args.tokens, D, R))
+    bb = sites.backward_bytes(sites.SiteShape("sliced", n, args.tokens, D, R, accumulate=1))
+    print(json.dumps({"profile_site": n, "T": args.tokens, "fwd_ms": f, "bwd_ms": b,
+                      "fwd_gbs": fb / f / 1e6, "bwd_gbs": bb / b / 1e6}), flush=True)
 
 
 def run_e2e(wl, args, dist, dev, step_bytes, world):
@@ -451,16 +505,20 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target length of the CPU oracle sample")
     ap.add_argument("--ref-step-seconds", type=float, default=4.0, help="target length of one reference step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-site", type=int, default=0, help="time one site with this many sources (profiling)")
+    ap.add_argument("--tokens", type=int, default=4096, help="tokens of the --profile-site case")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
-    if args.impl == "reference":
+    if args.profile_site:
+        run_profile_site(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)

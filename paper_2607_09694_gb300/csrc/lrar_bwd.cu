@@ -114,32 +114,34 @@ __device__ __forceinline__ void lr_route_b(const BwdParams &p, const Tin *__rest
 // the one vector that straddles the slice start (tail0), the slice elements keep
 // their old value here and receive alpha_i dh + dL/dk_i in the key pass, so every
 // element is rounded once.
-template <typename Tin, typename Tg, int V>
+template <typename Tin, typename Tg, int V, bool ACC>
 __device__ __forceinline__ float lr_bwd_row(const Frag<Tin, VecE<Tin>::value> *f,
-                                            const Frag<Tg, VecE<Tin>::value> *old, const float *dhf, float a,
-                                            Tg *__restrict__ drow, int tail0, int skip0, int lane, int accumulate) {
+                                            const Frag<Tg, VecE<Tin>::value> *old,
+                                            const Frag<Tin, VecE<Tin>::value> *dhr, float a, Tg *__restrict__ drow,
+                                            int tail0, int skip0, int lane) {
     constexpr int E = VecE<Tin>::value;
     float gp = 0.f;
 #pragma unroll
     for (int v = 0; v < V; ++v) {
         const int e = (lane + 32 * v) * E;
-        float o[E];
+        float o[E], dhv[E];
         f[v].get(o);
+        dhr[v].get(dhv);
 #pragma unroll
-        for (int t = 0; t < E; ++t) gp = fmaf(dhf[v * E + t], o[t], gp);
+        for (int t = 0; t < E; ++t) gp = fmaf(dhv[t], o[t], gp);
         if (e < skip0) {
             float w[E];
-            if (accumulate) old[v].get(w);
+            if (ACC) old[v].get(w);
             else
 #pragma unroll
                 for (int t = 0; t < E; ++t) w[t] = 0.f;
             if (e + E <= tail0) {
 #pragma unroll
-                for (int t = 0; t < E; ++t) w[t] = fmaf(a, dhf[v * E + t], w[t]);
+                for (int t = 0; t < E; ++t) w[t] = fmaf(a, dhv[t], w[t]);
             } else {
 #pragma unroll
                 for (int t = 0; t < E; ++t)
-                    if (e + t < tail0) w[t] = fmaf(a, dhf[v * E + t], w[t]);
+                    if (e + t < tail0) w[t] = fmaf(a, dhv[t], w[t]);
             }
             Frag<Tg, E> out;
             out.set(w);
@@ -149,7 +151,7 @@ __device__ __forceinline__ float lr_bwd_row(const Frag<Tin, VecE<Tin>::value> *f
     return gp;
 }
 
-template <typename Tin, typename Tg, int V, int U>
+template <typename Tin, typename Tg, int V, int U, bool ACC>
 __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(const BwdParams p) {
     constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
@@ -183,17 +185,16 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
         lr_route_b<Tin>(p, values, keys, x, lane, q_s, a_s, s_s, rho_s);
         __syncwarp();
 
-        // (2) value pass
-        float dhf[V * E];
+        // (2) value pass; dh stays packed in registers and widens per use
+        Frag<Tin, E> dhr[V];
 #pragma unroll
         for (int v = 0; v < V; ++v) {
             const int e = (lane + 32 * v) * E;
-            Frag<Tin, E> f;
-            if (e < p.d) f.load_nc(dh + x * p.d + e);
-            else f.zero();
-            f.get(dhf + v * E);
+            if (e < p.d) dhr[v].load_nc(dh + x * p.d + e);
+            else dhr[v].zero();
         }
         const int64_t row_off = x * p.d;
+        const int wend = p.d < skip0 ? p.d : skip0;
         int i = 0;
         for (; i + U <= p.n; i += U) {
             Frag<Tin, E> f[U][V];
@@ -206,14 +207,14 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
                     const int64_t off = (int64_t)(i + u) * src_stride + row_off + e;
                     if (e < p.d) f[u][v].load_nc(values + off);
                     else f[u][v].zero();
-                    if (p.accumulate && e < skip0) old[u][v].load(dvalues + off);
+                    if (ACC && e < skip0) old[u][v].load(dvalues + off);
                     else old[u][v].zero();
                 }
 #pragma unroll
             for (int u = 0; u < U; ++u) {
-                const float gp = lr_bwd_row<Tin, Tg, V>(f[u], old[u], dhf, a_s[i + u],
-                                                        dvalues + (int64_t)(i + u) * src_stride + row_off, tail0,
-                                                        p.d < skip0 ? p.d : skip0, lane, p.accumulate);
+                const float gp = lr_bwd_row<Tin, Tg, V, ACC>(f[u], old[u], dhr, a_s[i + u],
+                                                             dvalues + (int64_t)(i + u) * src_stride + row_off, tail0,
+                                                             wend, lane);
                 const float g = warp_sum(gp);
                 if (lane == 0) g_s[i + u] = g;
             }
@@ -227,11 +228,12 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
                 const int64_t off = (int64_t)i * src_stride + row_off + e;
                 if (e < p.d) f[v].load_nc(values + off);
                 else f[v].zero();
-                if (p.accumulate && e < skip0) old[v].load(dvalues + off);
+                if (ACC && e < skip0) old[v].load(dvalues + off);
                 else old[v].zero();
             }
-            const float gp = lr_bwd_row<Tin, Tg, V>(f, old, dhf, a_s[i], dvalues + (int64_t)i * src_stride + row_off,
-                                                    tail0, p.d < skip0 ? p.d : skip0, lane, p.accumulate);
+            const float gp = lr_bwd_row<Tin, Tg, V, ACC>(f, old, dhr, a_s[i],
+                                                         dvalues + (int64_t)i * src_stride + row_off, tail0, wend,
+                                                         lane);
             const float g = warp_sum(gp);
             if (lane == 0) g_s[i] = g;
         }
@@ -443,19 +445,38 @@ __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(co
     }
 }
 
-// Fixed-order sum of the CTA partials: dq[j] (+)= sum_b partials[b][j].
+// Fixed-order sum of the CTA partials, dq[j] (+)= sum_b partials[b][j]: one
+// warp per coordinate, lane l sums partials l, l+32, ... and a fixed butterfly
+// combines the lanes, so the result depends only on the number of partials.
 __global__ void dq_reduce_kernel(const float *__restrict__ partials, int nparts, int rq, float *dq, int accumulate) {
-    const int j = blockIdx.x * blockDim.x + threadIdx.x;
-    if (j >= rq) return;
+    const int j = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
+    const int lane = threadIdx.x & 31;
+    if (j >= rq) return;  // whole warps leave together (blockDim is a multiple of 32)
     float acc = 0.f;
-    for (int b = 0; b < nparts; ++b) acc += partials[(int64_t)b * rq + j];
-    dq[j] = accumulate ? dq[j] + acc : acc;
+    for (int b = lane; b < nparts; b += 32) acc += partials[(int64_t)b * rq + j];
+    acc = warp_sum(acc);
+    if (lane == 0) dq[j] = accumulate ? dq[j] + acc : acc;
 }
 
 // ------------------------------------------------------------- launch ----
+// Rows in flight per lane in the low-rank value pass (registers: V vectors of
+// values, and as many of old gradients when accumulating, per row).
+#ifndef LRAR_BWD_U_ACC
+#define LRAR_BWD_U_ACC 2
+#endif
+#ifndef LRAR_BWD_U_NOACC
+#define LRAR_BWD_U_NOACC 4
+#endif
+template <int V, bool ACC> struct BwdRows {
+    static constexpr int value = V >= 8 ? (ACC ? 1 : 2)
+                                        : V == 4 ? (ACC ? LRAR_BWD_U_ACC : LRAR_BWD_U_NOACC) : (ACC ? 4 : 8);
+};
+
 template <typename Tin, typename Tg, int V>
 static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     constexpr int U = V >= 4 ? 1 : (V == 2 ? 2 : 4);
+    // wider gradients than inputs double the old-gradient registers per row
+    constexpr int UA = sizeof(Tg) > sizeof(Tin) ? (BwdRows<V, true>::value + 1) / 2 : BwdRows<V, true>::value;
     BwdParams p;
     p.values = a.values;
     p.keys = a.keys;
@@ -489,7 +510,8 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
         smem = sizeof(float) * (size_t)round_up(a.d, 4) * (1 + kWarps);
         rq = a.d;
     } else {
-        k = (const void *)bwd_lr_kernel<Tin, Tg, V, U>;
+        k = a.accumulate ? (const void *)bwd_lr_kernel<Tin, Tg, V, UA, true>
+                         : (const void *)bwd_lr_kernel<Tin, Tg, V, BwdRows<V, false>::value, false>;
         smem = sizeof(float) * ((size_t)round_up(a.r, 4) * (1 + kWarps) + (size_t)kWarps * 4 * kMaxSources);
         rq = a.r;
     }
@@ -500,11 +522,13 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     const int grid = persistent_grid(k, kThreads, smem, work, kMaxPartials);
     if (a.variant == kFull)
         bwd_full_kernel<Tin, Tg, V, U><<<grid, kThreads, smem, s>>>(p);
+    else if (a.accumulate)
+        bwd_lr_kernel<Tin, Tg, V, UA, true><<<grid, kThreads, smem, s>>>(p);
     else
-        bwd_lr_kernel<Tin, Tg, V, U><<<grid, kThreads, smem, s>>>(p);
+        bwd_lr_kernel<Tin, Tg, V, BwdRows<V, false>::value, false><<<grid, kThreads, smem, s>>>(p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    dq_reduce_kernel<<<(rq + 255) / 256, 256, 0, s>>>(a.partials, grid, rq, a.dq, a.accumulate);
+    dq_reduce_kernel<<<(rq + 7) / 8, 256, 0, s>>>(a.partials, grid, rq, a.dq, a.accumulate);
     return cudaGetLastError();
 }
 
