@@ -45,7 +45,8 @@ def _load():
     global _lib
     with _lock:
         if _lib is None:
-            lib = ctypes.CDLL(build())
+            # LRAR_ORACLE_LIB points the tests' mutation check at a deliberately broken build.
+            lib = ctypes.CDLL(os.environ.get("LRAR_ORACLE_LIB") or build())
             vp, i64p, dp = ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p
             i, i64, dbl = ctypes.c_int, ctypes.c_int64, ctypes.c_double
             lib.oracle_forward.argtypes = [i, i, vp, vp, dp, i, i64, i, i, dbl, i64p, i64, dp, dp, dp]
