@@ -252,30 +252,15 @@ def oracle_sample(values_cpu, queries_cpu, dh_cpu, target_s: float):
 
 
 def _dist():
-    import torch.distributed as dist
+    from paper_2607_09694_gb300 import replicas
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    if world > 1 and not dist.is_initialized():
-        dist.init_process_group("nccl" if _cuda() else "gloo")
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    return dist if world > 1 else None, rank, local, world
-
-
-def _cuda() -> bool:
-    import torch
-
-    return torch.cuda.is_available()
+    return replicas.init_from_env()
 
 
 def _max_over_ranks(dist, value: float, device) -> float:
-    if dist is None:
-        return value
-    import torch
+    from paper_2607_09694_gb300 import replicas
 
-    t = torch.tensor([value], dtype=torch.float64, device=device)
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    return float(t.item())
+    return replicas.max_over_ranks(dist, value, device)
 
 
 def run_ours(args):
