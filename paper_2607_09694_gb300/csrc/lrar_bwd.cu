@@ -24,6 +24,8 @@
 // dq: each warp accumulates its tokens, each CTA writes one partial row to the
 // workspace, and a second kernel sums the partials in CTA order, so dq is
 // bitwise reproducible on a given device.
+#include <type_traits>
+
 #include "lrar_device.cuh"
 #include "lrar_launch.h"
 
@@ -175,7 +177,6 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
     Tg *__restrict__ dvalues = static_cast<Tg *>(p.dvalues);
     Tg *__restrict__ dkeys = static_cast<Tg *>(p.dkeys);
     const int64_t src_stride = p.T * (int64_t)p.d;
-    const int64_t key_stride = p.T * (int64_t)p.r;
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     const int tail0 = p.sliced ? p.d - p.r : p.d;  // first key coordinate inside the value row
     const int skip0 = round_up(tail0, E);          // vectors starting here lie wholly in the key slice
@@ -274,6 +275,157 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
         }
         __syncwarp();
     }
+    __syncthreads();
+    for (int j = threadIdx.x; j < p.r; j += kThreads) {
+        float acc = 0.f;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) acc += dq_all[w * rp + j];
+        p.partials[(int64_t)blockIdx.x * p.r + j] = acc;
+    }
+}
+
+// Low-rank keys with a per-lane async-copy ring (gradient type = input type):
+// the value pass reads rows of o (and, when accumulating, of the old gradient)
+// from shared memory, filled by cp.async S - 1 rows ahead across token
+// boundaries, so the loads in flight no longer drain between rows and cost no
+// registers.  Routing and key pass are those of bwd_lr_kernel.
+#ifndef LRAR_BWD_PIPE
+#define LRAR_BWD_PIPE 1
+#endif
+template <int V, bool ACC> struct BwdStages {
+#ifdef LRAR_BWD_STAGES
+    static constexpr int value = LRAR_BWD_STAGES;
+#else
+    static constexpr int value = V >= 8 ? (ACC ? 2 : 3) : (ACC ? 3 : 5);
+#endif
+};
+
+template <typename T, int V, int S, bool ACC>
+__global__ void __launch_bounds__(kThreads, 2) bwd_lr_pipe_kernel(const BwdParams p) {
+    constexpr int E = VecE<T>::value;
+    constexpr int P = ACC ? 2 : 1;  // planes per stage: o, old gradient
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int rp = round_up(p.r, 4);
+    uint4 *ring = reinterpret_cast<uint4 *>(smem_raw);  // [kWarps][S][P][V][32] cells
+    float *q_s = reinterpret_cast<float *>(smem_raw + (size_t)kWarps * S * P * V * 32 * 16);
+    float *dq_all = q_s + rp;             // [kWarps][r]
+    float *tab = dq_all + kWarps * rp;    // [kWarps][4][kMaxSources]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    float *dq_s = dq_all + warp * rp;
+    float *a_s = tab + warp * 4 * kMaxSources;
+    float *s_s = a_s + kMaxSources;
+    float *rho_s = s_s + kMaxSources;
+    float *g_s = rho_s + kMaxSources;  // g_i, then ds_i
+    const uint32_t ring_w = smem_u32(ring + (size_t)warp * S * P * V * 32) + 16u * lane;
+    for (int j = threadIdx.x; j < p.r; j += kThreads) q_s[j] = p.query ? p.query[j] : 0.f;
+    for (int j = threadIdx.x; j < kWarps * rp; j += kThreads) dq_all[j] = 0.f;
+    __syncthreads();
+
+    const T *__restrict__ values = static_cast<const T *>(p.values);
+    const T *__restrict__ keys = static_cast<const T *>(p.keys);
+    const T *__restrict__ dh = static_cast<const T *>(p.dh);
+    T *__restrict__ dvalues = static_cast<T *>(p.dvalues);
+    T *__restrict__ dkeys = static_cast<T *>(p.dkeys);
+    const int64_t src_stride = p.T * (int64_t)p.d;
+    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+    const int tail0 = p.sliced ? p.d - p.r : p.d;
+    const int skip0 = round_up(tail0, E);
+    const int wend = p.d < skip0 ? p.d : skip0;  // vectors below wend are written by the value pass
+    const int64_t x0 = (int64_t)blockIdx.x * kWarps + warp;
+
+    int64_t ix = x0;  // next row to copy: source ii of token ix
+    int ii = 0;
+    auto cell = [&](int st, int plane, int v) -> uint32_t {
+        return ring_w + (uint32_t)((((st * P + plane) * V + v) * 32) * 16);
+    };
+    auto issue = [&](int st) {
+        if (ix < p.T) {
+            const int64_t off = ((int64_t)ii * p.T + ix) * p.d;
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) cp_async16(cell(st, 0, v), values + off + e);
+                if (ACC && e < wend) cp_async16(cell(st, P - 1, v), dvalues + off + e);
+            }
+            if (++ii == p.n) {
+                ii = 0;
+                ix += nwarps;
+            }
+        }
+        cp_async_commit();
+    };
+#pragma unroll
+    for (int st = 0; st < S - 1; ++st) issue(st);
+    int st_c = 0, st_i = S - 1;
+
+    for (int64_t x = x0; x < p.T; x += nwarps) {
+        lr_route_b<T>(p, values, keys, x, lane, q_s, a_s, s_s, rho_s);
+        __syncwarp();
+
+        Frag<T, E> dhr[V];
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int e = (lane + 32 * v) * E;
+            if (e < p.d) dhr[v].load_nc(dh + x * p.d + e);
+            else dhr[v].zero();
+        }
+        const int64_t row_off = x * p.d;
+        for (int i = 0; i < p.n; ++i) {
+            issue(st_i);
+            cp_async_wait<S - 1>();  // this lane's copies of row i have landed
+            Frag<T, E> f[V];
+            Frag<T, E> old[V];
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) f[v].a = ld_shared16(cell(st_c, 0, v));
+                else f[v].zero();
+                if (ACC && e < wend) old[v].a = ld_shared16(cell(st_c, P - 1, v));
+                else old[v].zero();
+            }
+            const float gp = lr_bwd_row<T, T, V, ACC>(f, old, dhr, a_s[i], dvalues + (int64_t)i * src_stride + row_off,
+                                                      tail0, wend, lane);
+            const float g = warp_sum(gp);
+            if (lane == 0) g_s[i] = g;
+            st_c = (st_c + 1 == S) ? 0 : st_c + 1;
+            st_i = (st_i + 1 == S) ? 0 : st_i + 1;
+        }
+        __syncwarp();
+
+        float part = 0.f;
+        for (int k = lane; k < p.n; k += 32) part = fmaf(a_s[k], g_s[k], part);
+        const float gbar = warp_sum(part);
+        __syncwarp();
+        for (int k = lane; k < p.n; k += 32) g_s[k] = a_s[k] * (g_s[k] - gbar);
+        __syncwarp();
+        for (int j = lane; j < p.r; j += 32) {
+            const float qj = q_s[j];
+            const int c = tail0 + j;
+            const float dh_c = p.sliced ? to_f(__ldg(dh + row_off + c)) : 0.f;
+            float dqj = 0.f;
+#pragma unroll 4
+            for (int k = 0; k < p.n; ++k) {
+                const float rho = rho_s[k], s = s_s[k], ds = g_s[k];
+                float kij;
+                if (p.sliced) kij = to_f(__ldg(values + (int64_t)k * src_stride + row_off + c));
+                else kij = to_f(__ldg(keys + ((int64_t)k * p.T + x) * p.r + j));
+                const float kbar = rho * kij;
+                const float dk = ds * rho * (qj - s * p.inv_r * kbar);
+                dqj = fmaf(ds, kbar, dqj);
+                if (p.sliced) {
+                    T *dp = dvalues + (int64_t)k * src_stride + row_off + c;
+                    const float base = (c < skip0 || ACC) ? to_f(*dp) : 0.f;
+                    *dp = from_f<T>(base + fmaf(a_s[k], dh_c, dk));
+                } else {
+                    T *dp = dkeys + ((int64_t)k * p.T + x) * p.r + j;
+                    *dp = from_f<T>(ACC ? to_f(*dp) + dk : dk);
+                }
+            }
+            dq_s[j] += dqj;
+        }
+        __syncwarp();
+    }
+    cp_async_wait_all();
     __syncthreads();
     for (int j = threadIdx.x; j < p.r; j += kThreads) {
         float acc = 0.f;
@@ -505,10 +657,18 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     const void *k;
     size_t smem;
     int rq;
+    constexpr bool kPipe = LRAR_BWD_PIPE && std::is_same<Tin, Tg>::value;
+    constexpr int SA = BwdStages<V, true>::value, SN = BwdStages<V, false>::value;
     if (a.variant == kFull) {
         k = (const void *)bwd_full_kernel<Tin, Tg, V, U>;
         smem = sizeof(float) * (size_t)round_up(a.d, 4) * (1 + kWarps);
         rq = a.d;
+    } else if (kPipe) {
+        k = a.accumulate ? (const void *)bwd_lr_pipe_kernel<Tin, V, SA, true>
+                         : (const void *)bwd_lr_pipe_kernel<Tin, V, SN, false>;
+        smem = (size_t)kWarps * (a.accumulate ? SA * 2 : SN) * V * 32 * 16 +
+               sizeof(float) * ((size_t)round_up(a.r, 4) * (1 + kWarps) + (size_t)kWarps * 4 * kMaxSources);
+        rq = a.r;
     } else {
         k = a.accumulate ? (const void *)bwd_lr_kernel<Tin, Tg, V, UA, true>
                          : (const void *)bwd_lr_kernel<Tin, Tg, V, BwdRows<V, false>::value, false>;
@@ -522,6 +682,10 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     const int grid = persistent_grid(k, kThreads, smem, work, kMaxPartials);
     if (a.variant == kFull)
         bwd_full_kernel<Tin, Tg, V, U><<<grid, kThreads, smem, s>>>(p);
+    else if (kPipe && a.accumulate)
+        bwd_lr_pipe_kernel<Tin, V, SA, true><<<grid, kThreads, smem, s>>>(p);
+    else if (kPipe)
+        bwd_lr_pipe_kernel<Tin, V, SN, false><<<grid, kThreads, smem, s>>>(p);
     else if (a.accumulate)
         bwd_lr_kernel<Tin, Tg, V, UA, true><<<grid, kThreads, smem, s>>>(p);
     else
