@@ -292,6 +292,10 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
 #ifndef LRAR_BWD_PIPE
 #define LRAR_BWD_PIPE 1
 #endif
+#ifndef LRAR_KEY_BATCH
+#define LRAR_KEY_BATCH 8
+#endif
+constexpr int kKeyBatch = LRAR_KEY_BATCH;  // key-pass loads a lane keeps in flight
 template <int V, bool ACC> struct BwdStages {
 #ifdef LRAR_BWD_STAGES
     static constexpr int value = LRAR_BWD_STAGES;
@@ -398,30 +402,77 @@ __global__ void __launch_bounds__(kThreads, 2) bwd_lr_pipe_kernel(const BwdParam
         __syncwarp();
         for (int k = lane; k < p.n; k += 32) g_s[k] = a_s[k] * (g_s[k] - gbar);
         __syncwarp();
-        for (int j = lane; j < p.r; j += 32) {
+        if ((32 % p.r) == 0) {
+            // Key pass in batches: lane l owns key coordinate j = l mod r, the
+            // 32/r lanes that share j split the sources, and each lane keeps
+            // kKeyBatch (key, old gradient) loads in flight at once.
+            const int j = lane % p.r;
+            const int kstep = 32 / p.r;
             const float qj = q_s[j];
             const int c = tail0 + j;
             const float dh_c = p.sliced ? to_f(__ldg(dh + row_off + c)) : 0.f;
+            const bool rd_old = p.sliced ? (c < skip0 || ACC) : ACC;
             float dqj = 0.f;
-#pragma unroll 4
-            for (int k = 0; k < p.n; ++k) {
-                const float rho = rho_s[k], s = s_s[k], ds = g_s[k];
-                float kij;
-                if (p.sliced) kij = to_f(__ldg(values + (int64_t)k * src_stride + row_off + c));
-                else kij = to_f(__ldg(keys + ((int64_t)k * p.T + x) * p.r + j));
-                const float kbar = rho * kij;
-                const float dk = ds * rho * (qj - s * p.inv_r * kbar);
-                dqj = fmaf(ds, kbar, dqj);
-                if (p.sliced) {
-                    T *dp = dvalues + (int64_t)k * src_stride + row_off + c;
-                    const float base = (c < skip0 || ACC) ? to_f(*dp) : 0.f;
-                    *dp = from_f<T>(base + fmaf(a_s[k], dh_c, dk));
-                } else {
-                    T *dp = dkeys + ((int64_t)k * p.T + x) * p.r + j;
-                    *dp = from_f<T>(ACC ? to_f(*dp) + dk : dk);
+            for (int kb = lane / p.r; kb < p.n; kb += kstep * kKeyBatch) {
+                float kv[kKeyBatch], ov[kKeyBatch];
+#pragma unroll
+                for (int m = 0; m < kKeyBatch; ++m) {
+                    const int k = kb + m * kstep;
+                    kv[m] = ov[m] = 0.f;
+                    if (k < p.n) {
+                        if (p.sliced) {
+                            kv[m] = to_f(__ldg(values + (int64_t)k * src_stride + row_off + c));
+                            if (rd_old) ov[m] = to_f(dvalues[(int64_t)k * src_stride + row_off + c]);
+                        } else {
+                            kv[m] = to_f(__ldg(keys + ((int64_t)k * p.T + x) * p.r + j));
+                            if (rd_old) ov[m] = to_f(dkeys[((int64_t)k * p.T + x) * p.r + j]);
+                        }
+                    }
+                }
+#pragma unroll
+                for (int m = 0; m < kKeyBatch; ++m) {
+                    const int k = kb + m * kstep;
+                    if (k < p.n) {
+                        const float rho = rho_s[k], s = s_s[k], ds = g_s[k];
+                        const float kbar = rho * kv[m];
+                        const float dk = ds * rho * (qj - s * p.inv_r * kbar);
+                        dqj = fmaf(ds, kbar, dqj);
+                        if (p.sliced)
+                            dvalues[(int64_t)k * src_stride + row_off + c] = from_f<T>(ov[m] + fmaf(a_s[k], dh_c, dk));
+                        else
+                            dkeys[((int64_t)k * p.T + x) * p.r + j] = from_f<T>(ov[m] + dk);
+                    }
                 }
             }
-            dq_s[j] += dqj;
+            // lanes l and l ^ (r, 2r, ..., 16) share j: fixed-order butterfly
+            for (int off = p.r; off < 32; off <<= 1) dqj += __shfl_xor_sync(0xffffffffu, dqj, off);
+            if (lane < p.r) dq_s[j] += dqj;
+        } else {
+            for (int j = lane; j < p.r; j += 32) {
+                const float qj = q_s[j];
+                const int c = tail0 + j;
+                const float dh_c = p.sliced ? to_f(__ldg(dh + row_off + c)) : 0.f;
+                float dqj = 0.f;
+#pragma unroll 4
+                for (int k = 0; k < p.n; ++k) {
+                    const float rho = rho_s[k], s = s_s[k], ds = g_s[k];
+                    float kij;
+                    if (p.sliced) kij = to_f(__ldg(values + (int64_t)k * src_stride + row_off + c));
+                    else kij = to_f(__ldg(keys + ((int64_t)k * p.T + x) * p.r + j));
+                    const float kbar = rho * kij;
+                    const float dk = ds * rho * (qj - s * p.inv_r * kbar);
+                    dqj = fmaf(ds, kbar, dqj);
+                    if (p.sliced) {
+                        T *dp = dvalues + (int64_t)k * src_stride + row_off + c;
+                        const float base = (c < skip0 || ACC) ? to_f(*dp) : 0.f;
+                        *dp = from_f<T>(base + fmaf(a_s[k], dh_c, dk));
+                    } else {
+                        T *dp = dkeys + ((int64_t)k * p.T + x) * p.r + j;
+                        *dp = from_f<T>(ACC ? to_f(*dp) + dk : dk);
+                    }
+                }
+                dq_s[j] += dqj;
+            }
         }
         __syncwarp();
     }
