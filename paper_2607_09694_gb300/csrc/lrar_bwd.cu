@@ -304,8 +304,101 @@ template <int V, bool ACC> struct BwdStages {
 #endif
 };
 
+// Key pass of one token (low-rank keys), with ds_i already in ds_s: writes the
+// key slice of dvalues (S-LR: old + alpha_i dh + dL/dk_i, one rounding) or the
+// key gradients (P-LR), and adds sum_i ds_i kbar_i into dq_s.  When r divides
+// 32 or is a multiple of 32, every lane works and keeps kKeyBatch (key, old
+// gradient) loads in flight; lanes that share a coordinate combine their dq
+// parts with a fixed butterfly.  Other widths take one coordinate per lane.
+template <typename T, bool ACC>
+__device__ __forceinline__ void key_pass(const BwdParams &p, const T *__restrict__ values,
+                                         const T *__restrict__ keys, const T *__restrict__ dh,
+                                         T *__restrict__ dvalues, T *__restrict__ dkeys, int64_t x, int lane,
+                                         int tail0, int skip0, const float *__restrict__ q_s, const float *a_s,
+                                         const float *s_s, const float *rho_s, const float *ds_s, float *dq_s) {
+    const int64_t src_stride = p.T * (int64_t)p.d;
+    const int64_t row_off = x * p.d;
+    const bool shared_j = (32 % p.r) == 0;  // 32/r lanes per coordinate
+    const bool multi_j = (p.r % 32) == 0;   // r/32 coordinates per lane
+    if (shared_j || multi_j) {
+        const int kstep = shared_j ? 32 / p.r : 1;
+        const int jn = shared_j ? 1 : p.r / 32;
+        for (int t = 0; t < jn; ++t) {
+            const int j = shared_j ? lane % p.r : lane + 32 * t;
+            const float qj = q_s[j];
+            const int c = tail0 + j;
+            const float dh_c = p.sliced ? to_f(__ldg(dh + row_off + c)) : 0.f;
+            const bool rd_old = p.sliced ? (c < skip0 || ACC) : ACC;
+            float dqj = 0.f;
+            for (int kb = shared_j ? lane / p.r : 0; kb < p.n; kb += kstep * kKeyBatch) {
+                float kv[kKeyBatch], ov[kKeyBatch];
+#pragma unroll
+                for (int m = 0; m < kKeyBatch; ++m) {
+                    const int k = kb + m * kstep;
+                    kv[m] = ov[m] = 0.f;
+                    if (k < p.n) {
+                        if (p.sliced) {
+                            kv[m] = to_f(__ldg(values + (int64_t)k * src_stride + row_off + c));
+                            if (rd_old) ov[m] = to_f(dvalues[(int64_t)k * src_stride + row_off + c]);
+                        } else {
+                            kv[m] = to_f(__ldg(keys + ((int64_t)k * p.T + x) * p.r + j));
+                            if (rd_old) ov[m] = to_f(dkeys[((int64_t)k * p.T + x) * p.r + j]);
+                        }
+                    }
+                }
+#pragma unroll
+                for (int m = 0; m < kKeyBatch; ++m) {
+                    const int k = kb + m * kstep;
+                    if (k < p.n) {
+                        const float rho = rho_s[k], s = s_s[k], ds = ds_s[k];
+                        const float kbar = rho * kv[m];
+                        const float dk = ds * rho * (qj - s * p.inv_r * kbar);
+                        dqj = fmaf(ds, kbar, dqj);
+                        if (p.sliced)
+                            dvalues[(int64_t)k * src_stride + row_off + c] = from_f<T>(ov[m] + fmaf(a_s[k], dh_c, dk));
+                        else
+                            dkeys[((int64_t)k * p.T + x) * p.r + j] = from_f<T>(ov[m] + dk);
+                    }
+                }
+            }
+            if (shared_j) {  // lanes l and l ^ (r, 2r, ..., 16) share j: fixed-order butterfly
+                for (int off = p.r; off < 32; off <<= 1) dqj += __shfl_xor_sync(0xffffffffu, dqj, off);
+                if (lane < p.r) dq_s[j] += dqj;
+            } else {
+                dq_s[j] += dqj;
+            }
+        }
+    } else {
+        for (int j = lane; j < p.r; j += 32) {
+            const float qj = q_s[j];
+            const int c = tail0 + j;
+            const float dh_c = p.sliced ? to_f(__ldg(dh + row_off + c)) : 0.f;
+            float dqj = 0.f;
+#pragma unroll 4
+            for (int k = 0; k < p.n; ++k) {
+                const float rho = rho_s[k], s = s_s[k], ds = ds_s[k];
+                float kij;
+                if (p.sliced) kij = to_f(__ldg(values + (int64_t)k * src_stride + row_off + c));
+                else kij = to_f(__ldg(keys + ((int64_t)k * p.T + x) * p.r + j));
+                const float kbar = rho * kij;
+                const float dk = ds * rho * (qj - s * p.inv_r * kbar);
+                dqj = fmaf(ds, kbar, dqj);
+                if (p.sliced) {
+                    T *dp = dvalues + (int64_t)k * src_stride + row_off + c;
+                    const float base = (c < skip0 || ACC) ? to_f(*dp) : 0.f;
+                    *dp = from_f<T>(base + fmaf(a_s[k], dh_c, dk));
+                } else {
+                    T *dp = dkeys + ((int64_t)k * p.T + x) * p.r + j;
+                    *dp = from_f<T>(ACC ? to_f(*dp) + dk : dk);
+                }
+            }
+            dq_s[j] += dqj;
+        }
+    }
+}
+
 template <typename T, int V, int S, bool ACC>
-__global__ void __launch_bounds__(kThreads, 2) bwd_lr_pipe_kernel(const BwdParams p) {
+__global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(const BwdParams p) {
     constexpr int E = VecE<T>::value;
     constexpr int P = ACC ? 2 : 1;  // planes per stage: o, old gradient
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -358,6 +451,16 @@ __global__ void __launch_bounds__(kThreads, 2) bwd_lr_pipe_kernel(const BwdParam
         }
         cp_async_commit();
     };
+    Frag<T, E> dhr[V];  // dh of the token being processed (loaded one token ahead)
+    auto load_dh = [&](int64_t xx) {
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int e = (lane + 32 * v) * E;
+            if (e < p.d && xx < p.T) dhr[v].load_nc(dh + xx * p.d + e);
+            else dhr[v].zero();
+        }
+    };
+    load_dh(x0);
 #pragma unroll
     for (int st = 0; st < S - 1; ++st) issue(st);
     int st_c = 0, st_i = S - 1;
@@ -366,13 +469,6 @@ __global__ void __launch_bounds__(kThreads, 2) bwd_lr_pipe_kernel(const BwdParam
         lr_route_b<T>(p, values, keys, x, lane, q_s, a_s, s_s, rho_s);
         __syncwarp();
 
-        Frag<T, E> dhr[V];
-#pragma unroll
-        for (int v = 0; v < V; ++v) {
-            const int e = (lane + 32 * v) * E;
-            if (e < p.d) dhr[v].load_nc(dh + x * p.d + e);
-            else dhr[v].zero();
-        }
         const int64_t row_off = x * p.d;
         for (int i = 0; i < p.n; ++i) {
             issue(st_i);
@@ -394,6 +490,8 @@ __global__ void __launch_bounds__(kThreads, 2) bwd_lr_pipe_kernel(const BwdParam
             st_c = (st_c + 1 == S) ? 0 : st_c + 1;
             st_i = (st_i + 1 == S) ? 0 : st_i + 1;
         }
+        // this token's dh is dead now: the next token's travels during the key pass
+        load_dh(x + nwarps);
         __syncwarp();
 
         float part = 0.f;
@@ -402,78 +500,7 @@ __global__ void __launch_bounds__(kThreads, 2) bwd_lr_pipe_kernel(const BwdParam
         __syncwarp();
         for (int k = lane; k < p.n; k += 32) g_s[k] = a_s[k] * (g_s[k] - gbar);
         __syncwarp();
-        if ((32 % p.r) == 0) {
-            // Key pass in batches: lane l owns key coordinate j = l mod r, the
-            // 32/r lanes that share j split the sources, and each lane keeps
-            // kKeyBatch (key, old gradient) loads in flight at once.
-            const int j = lane % p.r;
-            const int kstep = 32 / p.r;
-            const float qj = q_s[j];
-            const int c = tail0 + j;
-            const float dh_c = p.sliced ? to_f(__ldg(dh + row_off + c)) : 0.f;
-            const bool rd_old = p.sliced ? (c < skip0 || ACC) : ACC;
-            float dqj = 0.f;
-            for (int kb = lane / p.r; kb < p.n; kb += kstep * kKeyBatch) {
-                float kv[kKeyBatch], ov[kKeyBatch];
-#pragma unroll
-                for (int m = 0; m < kKeyBatch; ++m) {
-                    const int k = kb + m * kstep;
-                    kv[m] = ov[m] = 0.f;
-                    if (k < p.n) {
-                        if (p.sliced) {
-                            kv[m] = to_f(__ldg(values + (int64_t)k * src_stride + row_off + c));
-                            if (rd_old) ov[m] = to_f(dvalues[(int64_t)k * src_stride + row_off + c]);
-                        } else {
-                            kv[m] = to_f(__ldg(keys + ((int64_t)k * p.T + x) * p.r + j));
-                            if (rd_old) ov[m] = to_f(dkeys[((int64_t)k * p.T + x) * p.r + j]);
-                        }
-                    }
-                }
-#pragma unroll
-                for (int m = 0; m < kKeyBatch; ++m) {
-                    const int k = kb + m * kstep;
-                    if (k < p.n) {
-                        const float rho = rho_s[k], s = s_s[k], ds = g_s[k];
-                        const float kbar = rho * kv[m];
-                        const float dk = ds * rho * (qj - s * p.inv_r * kbar);
-                        dqj = fmaf(ds, kbar, dqj);
-                        if (p.sliced)
-                            dvalues[(int64_t)k * src_stride + row_off + c] = from_f<T>(ov[m] + fmaf(a_s[k], dh_c, dk));
-                        else
-                            dkeys[((int64_t)k * p.T + x) * p.r + j] = from_f<T>(ov[m] + dk);
-                    }
-                }
-            }
-            // lanes l and l ^ (r, 2r, ..., 16) share j: fixed-order butterfly
-            for (int off = p.r; off < 32; off <<= 1) dqj += __shfl_xor_sync(0xffffffffu, dqj, off);
-            if (lane < p.r) dq_s[j] += dqj;
-        } else {
-            for (int j = lane; j < p.r; j += 32) {
-                const float qj = q_s[j];
-                const int c = tail0 + j;
-                const float dh_c = p.sliced ? to_f(__ldg(dh + row_off + c)) : 0.f;
-                float dqj = 0.f;
-#pragma unroll 4
-                for (int k = 0; k < p.n; ++k) {
-                    const float rho = rho_s[k], s = s_s[k], ds = g_s[k];
-                    float kij;
-                    if (p.sliced) kij = to_f(__ldg(values + (int64_t)k * src_stride + row_off + c));
-                    else kij = to_f(__ldg(keys + ((int64_t)k * p.T + x) * p.r + j));
-                    const float kbar = rho * kij;
-                    const float dk = ds * rho * (qj - s * p.inv_r * kbar);
-                    dqj = fmaf(ds, kbar, dqj);
-                    if (p.sliced) {
-                        T *dp = dvalues + (int64_t)k * src_stride + row_off + c;
-                        const float base = (c < skip0 || ACC) ? to_f(*dp) : 0.f;
-                        *dp = from_f<T>(base + fmaf(a_s[k], dh_c, dk));
-                    } else {
-                        T *dp = dkeys + ((int64_t)k * p.T + x) * p.r + j;
-                        *dp = from_f<T>(ACC ? to_f(*dp) + dk : dk);
-                    }
-                }
-                dq_s[j] += dqj;
-            }
-        }
+        key_pass<T, ACC>(p, values, keys, dh, dvalues, dkeys, x, lane, tail0, skip0, q_s, a_s, s_s, rho_s, g_s, dq_s);
         __syncwarp();
     }
     cp_async_wait_all();
