@@ -171,6 +171,24 @@ int lrar_backward_noalloc(int variant, int in_dtype, int grad_dtype, const void 
 int lrar_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *src, int64_t count,
                           float alpha, float beta, void *stream);
 
+/*
+ * Routing diagnostics of one site (§4.5-4.6): the effective number of sources
+ * of every token, N_eff = exp(H(alpha)) with H = -sum_i alpha_i log alpha_i
+ * (Eq. 16; 0 log 0 = 0), and alpha averaged over the T tokens (one row of the
+ * mean-attention heatmap).  alpha is that of lrar_forward with the same
+ * arguments (Eq. 8-9); for low-rank keys only the keys are read.
+ *   neff        [T] float32, written; may be NULL
+ *   mean_alpha  [n_src] float32, written; may be NULL (then no workspace is needed)
+ *   workspace   >= lrar_diagnostics_workspace_size(n_src) bytes, 16-byte aligned,
+ *               when mean_alpha is requested; contents on entry are ignored.
+ *               The mean is summed in a fixed order (bitwise reproducible).
+ * Other arguments, layouts and errors as for lrar_forward; T == 0 sets mean_alpha to 0.
+ */
+size_t lrar_diagnostics_workspace_size(int n_src);
+int lrar_diagnostics(int variant, int in_dtype, const void *values, const void *keys, const float *query,
+                     int n_src, int64_t T, int d, int r, float eps, float *neff, float *mean_alpha, void *workspace,
+                     size_t workspace_bytes, void *stream);
+
 /* Static text for a status code. */
 const char *lrar_strerror(int code);
 

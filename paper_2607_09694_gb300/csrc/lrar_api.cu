@@ -220,6 +220,53 @@ LRAR_API int lrar_backward(int variant, int in_dtype, int grad_dtype, const void
     return LRAR_OK;
 }
 
+LRAR_API size_t lrar_diagnostics_workspace_size(int n_src) {
+    return n_src < 1 ? 0 : sizeof(float) * (size_t)lrar::kMaxPartials * (size_t)n_src;
+}
+
+LRAR_API int lrar_diagnostics(int variant, int in_dtype, const void *values, const void *keys, const float *query,
+                              int n_src, int64_t T, int d, int r, float eps, float *neff, float *mean_alpha,
+                              void *workspace, size_t workspace_bytes, void *stream) {
+    int rc = check_shape(variant, in_dtype, n_src, T, d, r, eps);
+    if (rc) return rc;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (T == 0) {  // no tokens: the mean over them is defined here as 0
+        if (mean_alpha) {
+            cudaError_t e = cudaMemsetAsync(mean_alpha, 0, sizeof(float) * (size_t)n_src, s);
+            if (e != cudaSuccess) return cuda_fail(e, "lrar_diagnostics");
+        }
+        return LRAR_OK;
+    }
+    if (!values) return fail(LRAR_ERR_INVALID_ARG, "values are required");
+    if (variant == LRAR_PROJECTED && !keys) return fail(LRAR_ERR_INVALID_ARG, "projected keys are required");
+    if (!query && n_src > 1) return fail(LRAR_ERR_INVALID_ARG, "query is required when n_src > 1");
+    if (!aligned16(values) || (variant == LRAR_PROJECTED && !aligned16(keys)) || (query && !aligned4(query)) ||
+        (neff && !aligned4(neff)) || (mean_alpha && !aligned4(mean_alpha)))
+        return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (query, neff and mean_alpha 4-byte)");
+    if (mean_alpha && (!workspace || workspace_bytes < lrar_diagnostics_workspace_size(n_src)))
+        return fail(LRAR_ERR_WORKSPACE, "mean_alpha needs a workspace of %zu bytes",
+                    lrar_diagnostics_workspace_size(n_src));
+    if (mean_alpha && !aligned16(workspace)) return fail(LRAR_ERR_ALIGNMENT, "workspace must be 16-byte aligned");
+    if (!neff && !mean_alpha) return LRAR_OK;
+    lrar::FwdArgs a;
+    a.variant = variant;
+    a.in_dtype = in_dtype;
+    a.out_dtype = in_dtype;
+    a.values = values;
+    a.keys = variant == LRAR_PROJECTED ? keys : nullptr;
+    a.query = query;
+    a.n = n_src;
+    a.T = T;
+    a.d = d;
+    a.r = r;
+    a.eps = eps;
+    a.h = nullptr;
+    a.lse = nullptr;
+    cudaError_t e = lrar::launch_diagnostics(a, neff, mean_alpha, static_cast<float *>(workspace), s);
+    if (e != cudaSuccess) return cuda_fail(e, "lrar_diagnostics");
+    return LRAR_OK;
+}
+
 LRAR_API int lrar_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *src, int64_t count,
                                    float alpha, float beta, void *stream) {
     if (!dtype_ok(dst_dtype) || !dtype_ok(src_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown dtype");

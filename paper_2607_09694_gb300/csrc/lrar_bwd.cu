@@ -688,6 +688,12 @@ __global__ void dq_reduce_kernel(const float *__restrict__ partials, int nparts,
     if (lane == 0) dq[j] = accumulate ? dq[j] + acc : acc;
 }
 
+cudaError_t launch_partial_sum(const float *partials, int nparts, int width, float *out, int accumulate,
+                               cudaStream_t s) {
+    dq_reduce_kernel<<<(width + 7) / 8, 256, 0, s>>>(partials, nparts, width, out, accumulate);
+    return cudaGetLastError();
+}
+
 // ------------------------------------------------------------- launch ----
 // Rows in flight per lane in the low-rank value pass (registers: V vectors of
 // values, and as many of old gradients when accumulating, per row).

@@ -325,6 +325,136 @@ static cudaError_t launch_fwd_w(const FwdArgs &a, cudaStream_t s) {
     return launch_fwd_t<Tin, Tout, 8>(a, s);
 }
 
+// ------------------------------------------------- routing diagnostics ----
+// §4.5-4.6: per token, N_eff = exp(H(alpha)) with H = -sum_i alpha_i log alpha_i
+// (Eq. 16, 0 log 0 = 0); per site, alpha averaged over the T tokens.  Routing is
+// that of the forward (low-rank keys: lr_route; full keys: each value row is
+// read once for its score).  Each CTA writes one row of mean partials (already
+// divided by T) for a fixed-order sum.
+template <typename Tin, int V>
+__global__ void __launch_bounds__(kThreads) diag_kernel(const FwdParams p, float *neff, float *partials, int full) {
+    constexpr int E = VecE<Tin>::value;
+    extern __shared__ float smem[];
+    float *q_s = smem;                                    // [r]
+    float *a_all = smem + round_up(p.r, 4);               // [kWarps][kMaxSources]
+    float *m_all = a_all + kWarps * kMaxSources;          // [kWarps][kMaxSources] running mean
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    float *a_s = a_all + warp * kMaxSources;
+    float *m_s = m_all + warp * kMaxSources;
+    for (int j = threadIdx.x; j < p.r; j += kThreads) q_s[j] = p.query ? p.query[j] : 0.f;
+    for (int j = threadIdx.x; j < kWarps * kMaxSources; j += kThreads) m_all[j] = 0.f;
+    __syncthreads();
+
+    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
+    const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
+    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+    const float inv_T = 1.f / (float)p.T;
+    for (int64_t x = (int64_t)blockIdx.x * kWarps + warp; x < p.T; x += nwarps) {
+        if (!full) {
+            lr_route<Tin>(values, keys, p.T, p.n, p.d, p.r, p.eps, p.inv_r, p.sliced, p.key_vec, x, lane, q_s, a_s,
+                          nullptr, nullptr);
+        } else {
+            for (int i = 0; i < p.n; ++i) {  // score of source i from its whole row (r = d)
+                const Tin *row = values + ((int64_t)i * p.T + x) * p.d;
+                float ss = 0.f, qo = 0.f;
+#pragma unroll
+                for (int v = 0; v < V; ++v) {
+                    const int e = (lane + 32 * v) * E;
+                    if (e < p.d) {
+                        Frag<Tin, E> f;
+                        f.load_nc(row + e);
+                        float o[E];
+                        f.get(o);
+#pragma unroll
+                        for (int t = 0; t < E; ++t) {
+                            ss = fmaf(o[t], o[t], ss);
+                            qo = fmaf(q_s[e + t], o[t], qo);
+                        }
+                    }
+                }
+                ss = warp_sum(ss);
+                qo = warp_sum(qo);
+                if (lane == 0) a_s[i] = rsqrtf(fmaf(ss, p.inv_r, p.eps)) * qo;  // score, softmax below
+            }
+            __syncwarp();
+            float m = -INFINITY;
+            for (int i = lane; i < p.n; i += 32) m = fmaxf(m, a_s[i]);
+            m = warp_max(m);
+            float z = 0.f;
+            for (int i = lane; i < p.n; i += 32) z += expf(a_s[i] - m);
+            z = warp_sum(z);
+            __syncwarp();
+            for (int i = lane; i < p.n; i += 32) a_s[i] = expf(a_s[i] - m) / z;
+        }
+        __syncwarp();
+        float hp = 0.f;
+        for (int i = lane; i < p.n; i += 32) {
+            const float a = a_s[i];
+            if (a > 0.f) hp -= a * logf(a);
+            m_s[i] = fmaf(a, inv_T, m_s[i]);  // coordinate i belongs to this lane alone
+        }
+        const float H = warp_sum(hp);
+        if (lane == 0 && neff) neff[x] = expf(H);
+        __syncwarp();
+    }
+    __syncthreads();
+    if (partials)
+        for (int i = threadIdx.x; i < p.n; i += kThreads) {
+            float acc = 0.f;
+#pragma unroll
+            for (int w = 0; w < kWarps; ++w) acc += m_all[w * kMaxSources + i];
+            partials[(int64_t)blockIdx.x * p.n + i] = acc;
+        }
+}
+
+template <typename Tin, int V>
+static cudaError_t launch_diag_t(const FwdArgs &a, float *neff, float *mean_alpha, float *partials, cudaStream_t s) {
+    FwdParams p;
+    p.values = a.values;
+    p.keys = a.keys;
+    p.query = a.query;
+    p.h = nullptr;
+    p.lse = nullptr;
+    p.T = a.T;
+    p.n = a.n;
+    p.d = a.d;
+    p.r = a.r;
+    p.eps = a.eps;
+    p.inv_r = 1.f / (float)a.r;
+    p.sliced = a.variant == kSliced;
+    constexpr int esz = sizeof(Tin);
+    if (a.variant == kSliced)
+        p.key_vec = ((a.r * esz) % 16 == 0) && (((a.d - a.r) * esz) % 16 == 0);
+    else
+        p.key_vec = ((a.r * esz) % 16 == 0) && ((reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
+    const size_t smem = sizeof(float) * (round_up(a.r, 4) + 2 * kWarps * kMaxSources);
+    const void *k = (const void *)diag_kernel<Tin, V>;
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    const int grid = persistent_grid(k, kThreads, smem, (a.T + kWarps - 1) / kWarps, kMaxPartials);
+    diag_kernel<Tin, V><<<grid, kThreads, smem, s>>>(p, neff, mean_alpha ? partials : nullptr, a.variant == kFull);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess || !mean_alpha) return e;
+    return launch_partial_sum(partials, grid, a.n, mean_alpha, 0, s);
+}
+
+template <typename Tin>
+static cudaError_t launch_diag_w(const FwdArgs &a, float *neff, float *mean_alpha, float *partials, cudaStream_t s) {
+    constexpr int E = VecE<Tin>::value;
+    const int vecs = (a.d + E - 1) / E;
+    if (vecs <= 32) return launch_diag_t<Tin, 1>(a, neff, mean_alpha, partials, s);
+    if (vecs <= 64) return launch_diag_t<Tin, 2>(a, neff, mean_alpha, partials, s);
+    if (vecs <= 128) return launch_diag_t<Tin, 4>(a, neff, mean_alpha, partials, s);
+    return launch_diag_t<Tin, 8>(a, neff, mean_alpha, partials, s);
+}
+
+cudaError_t launch_diagnostics(const FwdArgs &a, float *neff, float *mean_alpha, float *partials, cudaStream_t s) {
+    return a.in_dtype == kBF16 ? launch_diag_w<bf16>(a, neff, mean_alpha, partials, s)
+                               : launch_diag_w<float>(a, neff, mean_alpha, partials, s);
+}
+
 cudaError_t launch_forward(const FwdArgs &a, cudaStream_t s) {
     if (a.in_dtype == kBF16)
         return a.out_dtype == kBF16 ? launch_fwd_w<bf16, bf16>(a, s) : launch_fwd_w<bf16, float>(a, s);

@@ -49,6 +49,12 @@ int record_error(int code, const char *message);
 int max_width(int in_dtype);
 
 cudaError_t launch_forward(const FwdArgs &a, cudaStream_t s);
+// Routing diagnostics (a.h unused): neff [T] and/or mean_alpha [n] (the latter
+// through `partials`, [kMaxPartials][n] floats).
+cudaError_t launch_diagnostics(const FwdArgs &a, float *neff, float *mean_alpha, float *partials, cudaStream_t s);
+// out[j] (+)= sum_b partials[b][j] for b < nparts, in a fixed order.
+cudaError_t launch_partial_sum(const float *partials, int nparts, int width, float *out, int accumulate,
+                               cudaStream_t s);
 cudaError_t launch_backward(const BwdArgs &a, cudaStream_t s);
 cudaError_t launch_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *src, int64_t count,
                                     float alpha, float beta, cudaStream_t s);

@@ -25,7 +25,8 @@ ERR_INVALID_ARG, ERR_ALIGNMENT, ERR_UNSUPPORTED, ERR_CUDA, ERR_WORKSPACE = -1, -
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "liblrar.so")
 EXPORTS = ("lrar_forward", "lrar_backward", "lrar_backward_workspace_size", "lrar_block_accumulate",
-           "lrar_strerror", "lrar_last_error", "lrar_version", "lrar_backward_noalloc")
+           "lrar_strerror", "lrar_last_error", "lrar_version", "lrar_backward_noalloc", "lrar_diagnostics",
+           "lrar_diagnostics_workspace_size")
 
 _lock = threading.Lock()
 _lib = None
@@ -54,6 +55,10 @@ def load(path: str | None = None):
         lib.lrar_backward.restype = i
         lib.lrar_backward_noalloc.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, i, vp, vp, vp, vp, i, vp]
         lib.lrar_backward_noalloc.restype = i
+        lib.lrar_diagnostics.argtypes = [i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, vp, sz, vp]
+        lib.lrar_diagnostics.restype = i
+        lib.lrar_diagnostics_workspace_size.argtypes = [i]
+        lib.lrar_diagnostics_workspace_size.restype = sz
         lib.lrar_backward_workspace_size.argtypes = [i, i, i64, i, i]
         lib.lrar_backward_workspace_size.restype = sz
         lib.lrar_block_accumulate.argtypes = [i, vp, i, vp, i64, f32, f32, vp]
@@ -157,6 +162,25 @@ def backward_noalloc(variant, values: torch.Tensor, keys: torch.Tensor | None, q
                                         _ptr(query), n, T, d, r, eps, _ptr(dh), _ptr(h), dtype_code(h), _ptr(lse),
                                         _ptr(dvalues), _ptr(dkeys), _ptr(dq), int(bool(accumulate)),
                                         _stream(stream)))
+
+
+def diagnostics(variant, values: torch.Tensor, keys: torch.Tensor | None, query: torch.Tensor | None,
+                neff: torch.Tensor | None = None, mean_alpha: torch.Tensor | None = None,
+                workspace: torch.Tensor | None = None, n_src: int | None = None, r: int | None = None,
+                eps: float = DEFAULT_EPS, stream=None) -> None:
+    """lrar_diagnostics: per-token N_eff [T] and the token-mean of alpha [n_src] (Eq. 16, §4.5-4.6)."""
+    variant = _variant(variant)
+    _, T, d = values.shape
+    n = values.shape[0] if n_src is None else n_src
+    if r is None:
+        r = d if variant == FULL else (keys.shape[-1] if variant == PROJECTED else query.numel())
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(load().lrar_diagnostics(variant, dtype_code(values), _ptr(values), _ptr(keys), _ptr(query), n, T, d, r,
+                                   eps, _ptr(neff), _ptr(mean_alpha), _ptr(workspace), ws_bytes, _stream(stream)))
+
+
+def diagnostics_workspace_size(n_src: int) -> int:
+    return int(load().lrar_diagnostics_workspace_size(n_src))
 
 
 def block_accumulate(dst: torch.Tensor, src: torch.Tensor, alpha: float = 1.0, beta: float = 1.0,

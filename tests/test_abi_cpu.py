@@ -121,6 +121,19 @@ def test_workspace_size_is_device_independent(lib):
     assert lib.lrar_backward_workspace_size(2, 1, 1, 64, 0) == 0
 
 
+def test_diagnostics_rejects(lib):
+    f = lib.lrar_diagnostics
+    ws = lib.lrar_diagnostics_workspace_size(4)
+    assert ws == 1024 * 4 * 4
+    assert f(1, 1, FAKE, None, FAKE, 0, 8, 64, 4, EPS, FAKE, FAKE, FAKE, ws, None) == lrar.ERR_INVALID_ARG
+    assert f(1, 1, None, None, FAKE, 4, 8, 64, 4, EPS, FAKE, None, None, 0, None) == lrar.ERR_INVALID_ARG
+    assert f(2, 1, FAKE, None, FAKE, 4, 8, 64, 4, EPS, FAKE, None, None, 0, None) == lrar.ERR_INVALID_ARG
+    assert f(1, 1, FAKE, None, FAKE, 4, 8, 64, 4, EPS, FAKE, FAKE, None, 0, None) == lrar.ERR_WORKSPACE
+    assert f(1, 1, FAKE, None, FAKE, 4, 8, 64, 4, EPS, FAKE, FAKE, FAKE, 16, None) == lrar.ERR_WORKSPACE
+    assert f(1, 1, FAKE + 8, None, FAKE, 4, 8, 64, 4, EPS, FAKE, None, None, 0, None) == lrar.ERR_ALIGNMENT
+    assert f(1, 1, FAKE, None, FAKE, 4, 8, 64, 4, EPS, None, None, None, 0, None) == lrar.OK  # nothing asked
+
+
 def test_block_accumulate_rejects(lib):
     f = lib.lrar_block_accumulate
     assert f(3, FAKE, 1, FAKE, 10, 1.0, 1.0, None) == lrar.ERR_INVALID_ARG
