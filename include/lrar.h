@@ -50,6 +50,7 @@ extern "C" {
 
 #define LRAR_VERSION 1
 #define LRAR_MAX_SOURCES 128
+#define LRAR_MAX_BLOCK_SITES 64
 
 enum lrar_variant { LRAR_FULL = 0, LRAR_SLICED = 1, LRAR_PROJECTED = 2 };
 enum lrar_dtype { LRAR_F32 = 0, LRAR_BF16 = 1 };
@@ -170,6 +171,41 @@ int lrar_backward_noalloc(int variant, int in_dtype, int grad_dtype, const void 
  */
 int lrar_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *src, int64_t count,
                           float alpha, float beta, void *stream);
+
+/*
+ * Block AttnRes two-phase batched sites (§3.5), low-rank keys only.  The
+ * n_sites read sites inside one block all see the block's completed sources
+ * (the embedding and the completed block summaries, Eq. 5) plus a partial
+ * summary that grows by one output per site (Eq. 6).  Because the queries are
+ * static, one pass over the completed sources serves every site of the block
+ * (phase 1), and each site then folds in its partial summary with an
+ * online-softmax update (phase 2).  The completed sources are read once per
+ * block instead of once per site; the result equals lrar_forward over
+ * [completed sources, partial summary].
+ *
+ * Phase 1:
+ *   values      [n_completed, T, d] in_dtype: the completed sources (a stack prefix)
+ *   keys        [n_completed, T, r] in_dtype, LRAR_PROJECTED only
+ *   queries     [n_sites, r] float32, one static query per site
+ *   h_pre       [n_sites, T, d] pre_dtype, written: softmax mix over the completed
+ *               sources only (float32 keeps phase 2 exact; bfloat16 rounds it)
+ *   lse_pre     [n_sites, T] float32, written: log sum_i exp(score) over them
+ *   n_sites     1..LRAR_MAX_BLOCK_SITES
+ * Phase 2 (one site):
+ *   h_pre, lse_pre  that site's rows of the phase-1 outputs ([T, d], [T])
+ *   partial     [T, d] in_dtype: the partial-block summary (for the first site
+ *               of a block the partial block is empty: use h_pre as h directly)
+ *   partial_key [T, r] in_dtype: its projected key (LRAR_PROJECTED), else ignored
+ *   query       [r] float32: the site's query
+ *   h           [T, d] out_dtype, written; lse [T] float32, written when non-NULL
+ * Other arguments and errors as for lrar_forward; LRAR_FULL is LRAR_ERR_UNSUPPORTED.
+ */
+int lrar_block_phase1(int variant, int in_dtype, int pre_dtype, const void *values, const void *keys,
+                      const float *queries, int n_completed, int n_sites, int64_t T, int d, int r, float eps,
+                      void *h_pre, float *lse_pre, void *stream);
+int lrar_block_phase2(int variant, int in_dtype, int pre_dtype, int out_dtype, const void *h_pre,
+                      const float *lse_pre, const void *partial, const void *partial_key, const float *query,
+                      int64_t T, int d, int r, float eps, void *h, float *lse, void *stream);
 
 /*
  * Routing diagnostics of one site (§4.5-4.6): the effective number of sources

@@ -267,6 +267,81 @@ LRAR_API int lrar_diagnostics(int variant, int in_dtype, const void *values, con
     return LRAR_OK;
 }
 
+LRAR_API int lrar_block_phase1(int variant, int in_dtype, int pre_dtype, const void *values, const void *keys,
+                               const float *queries, int n_completed, int n_sites, int64_t T, int d, int r, float eps,
+                               void *h_pre, float *lse_pre, void *stream) {
+    if (variant == LRAR_FULL)
+        return fail(LRAR_ERR_UNSUPPORTED, "the two-phase block path serves low-rank keys (sliced, projected)");
+    int rc = check_shape(variant, in_dtype, n_completed, T, d, r, eps);
+    if (rc) return rc;
+    if (!dtype_ok(pre_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown phase-1 output dtype %d", pre_dtype);
+    if (n_sites < 1 || n_sites > LRAR_MAX_BLOCK_SITES)
+        return fail(LRAR_ERR_INVALID_ARG, "n_sites must be in 1..%d (got %d)", LRAR_MAX_BLOCK_SITES, n_sites);
+    if (T == 0) return LRAR_OK;
+    if (!values || !queries || !h_pre || !lse_pre)
+        return fail(LRAR_ERR_INVALID_ARG, "values, queries, h_pre and lse_pre are required");
+    if (variant == LRAR_PROJECTED && !keys) return fail(LRAR_ERR_INVALID_ARG, "projected keys are required");
+    if (!aligned16(values) || !aligned16(h_pre) || (variant == LRAR_PROJECTED && !aligned16(keys)) ||
+        !aligned4(queries) || !aligned4(lse_pre))
+        return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (queries and lse_pre 4-byte)");
+    lrar::BlockPh1Args a;
+    a.variant = variant;
+    a.in_dtype = in_dtype;
+    a.pre_dtype = pre_dtype;
+    a.values = values;
+    a.keys = variant == LRAR_PROJECTED ? keys : nullptr;
+    a.queries = queries;
+    a.n = n_completed;
+    a.c = n_sites;
+    a.T = T;
+    a.d = d;
+    a.r = r;
+    a.eps = eps;
+    a.h_pre = h_pre;
+    a.lse_pre = lse_pre;
+    cudaError_t e = lrar::launch_block_phase1(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "lrar_block_phase1");
+    return LRAR_OK;
+}
+
+LRAR_API int lrar_block_phase2(int variant, int in_dtype, int pre_dtype, int out_dtype, const void *h_pre,
+                               const float *lse_pre, const void *partial, const void *partial_key,
+                               const float *query, int64_t T, int d, int r, float eps, void *h, float *lse,
+                               void *stream) {
+    if (variant == LRAR_FULL)
+        return fail(LRAR_ERR_UNSUPPORTED, "the two-phase block path serves low-rank keys (sliced, projected)");
+    int rc = check_shape(variant, in_dtype, 1, T, d, r, eps);
+    if (rc) return rc;
+    if (!dtype_ok(pre_dtype) || !dtype_ok(out_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown dtype");
+    if (T == 0) return LRAR_OK;
+    if (!h_pre || !lse_pre || !partial || !query || !h)
+        return fail(LRAR_ERR_INVALID_ARG, "h_pre, lse_pre, partial, query and h are required");
+    if (variant == LRAR_PROJECTED && !partial_key)
+        return fail(LRAR_ERR_INVALID_ARG, "the partial summary's projected key is required");
+    if (!aligned16(h_pre) || !aligned16(partial) || !aligned16(h) || !aligned4(lse_pre) || !aligned4(query) ||
+        (lse && !aligned4(lse)) || (variant == LRAR_PROJECTED && !aligned4(partial_key)))
+        return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (lse, query and keys 4-byte)");
+    lrar::BlockPh2Args a;
+    a.variant = variant;
+    a.in_dtype = in_dtype;
+    a.pre_dtype = pre_dtype;
+    a.out_dtype = out_dtype;
+    a.h_pre = h_pre;
+    a.lse_pre = lse_pre;
+    a.partial = partial;
+    a.pkeys = variant == LRAR_PROJECTED ? partial_key : nullptr;
+    a.query = query;
+    a.T = T;
+    a.d = d;
+    a.r = r;
+    a.eps = eps;
+    a.h = h;
+    a.lse = lse;
+    cudaError_t e = lrar::launch_block_phase2(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "lrar_block_phase2");
+    return LRAR_OK;
+}
+
 LRAR_API int lrar_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *src, int64_t count,
                                    float alpha, float beta, void *stream) {
     if (!dtype_ok(dst_dtype) || !dtype_ok(src_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown dtype");

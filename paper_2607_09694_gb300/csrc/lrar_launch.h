@@ -42,6 +42,36 @@ struct BwdArgs {
     float *partials;  // workspace: [kMaxPartials][rq] floats
 };
 
+struct BlockPh1Args {
+    int variant, in_dtype, pre_dtype;
+    const void *values;   // completed sources [n, T, d]
+    const void *keys;     // P-LR keys [n, T, r]
+    const float *queries; // [c, r]
+    int n, c;
+    int64_t T;
+    int d, r;
+    float eps;
+    void *h_pre;     // [c, T, d]
+    float *lse_pre;  // [c, T]
+};
+
+struct BlockPh2Args {
+    int variant, in_dtype, pre_dtype, out_dtype;
+    const void *h_pre;     // [T, d] of one site
+    const float *lse_pre;  // [T]
+    const void *partial;   // partial-block summary [T, d]
+    const void *pkeys;     // its P-LR key [T, r]
+    const float *query;    // [r]
+    int64_t T;
+    int d, r;
+    float eps;
+    void *h;     // [T, d]
+    float *lse;  // [T] or null
+};
+
+cudaError_t launch_block_phase1(const BlockPh1Args &a, cudaStream_t s);
+cudaError_t launch_block_phase2(const BlockPh2Args &a, cudaStream_t s);
+
 // Sets the calling thread's lrar_last_error() message; returns `code`.
 int record_error(int code, const char *message);
 

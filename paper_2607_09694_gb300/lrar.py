@@ -26,7 +26,8 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "liblrar.so")
 EXPORTS = ("lrar_forward", "lrar_backward", "lrar_backward_workspace_size", "lrar_block_accumulate",
            "lrar_strerror", "lrar_last_error", "lrar_version", "lrar_backward_noalloc", "lrar_diagnostics",
-           "lrar_diagnostics_workspace_size")
+           "lrar_diagnostics_workspace_size", "lrar_block_phase1", "lrar_block_phase2")
+MAX_BLOCK_SITES = 64
 
 _lock = threading.Lock()
 _lib = None
@@ -55,6 +56,10 @@ def load(path: str | None = None):
         lib.lrar_backward.restype = i
         lib.lrar_backward_noalloc.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, i, vp, vp, vp, vp, i, vp]
         lib.lrar_backward_noalloc.restype = i
+        lib.lrar_block_phase1.argtypes = [i, i, i, vp, vp, vp, i, i, i64, i, i, f32, vp, vp, vp]
+        lib.lrar_block_phase1.restype = i
+        lib.lrar_block_phase2.argtypes = [i, i, i, i, vp, vp, vp, vp, vp, i64, i, i, f32, vp, vp, vp]
+        lib.lrar_block_phase2.restype = i
         lib.lrar_diagnostics.argtypes = [i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, vp, sz, vp]
         lib.lrar_diagnostics.restype = i
         lib.lrar_diagnostics_workspace_size.argtypes = [i]
@@ -162,6 +167,31 @@ def backward_noalloc(variant, values: torch.Tensor, keys: torch.Tensor | None, q
                                         _ptr(query), n, T, d, r, eps, _ptr(dh), _ptr(h), dtype_code(h), _ptr(lse),
                                         _ptr(dvalues), _ptr(dkeys), _ptr(dq), int(bool(accumulate)),
                                         _stream(stream)))
+
+
+def block_phase1(variant, values: torch.Tensor, keys: torch.Tensor | None, queries: torch.Tensor,
+                 h_pre: torch.Tensor, lse_pre: torch.Tensor, n_completed: int | None = None,
+                 eps: float = DEFAULT_EPS, stream=None) -> None:
+    """lrar_block_phase1: mixes of the first n_completed sources of `values` for
+    every query row of `queries` [n_sites, r] -> h_pre [n_sites, T, d], lse_pre [n_sites, T]."""
+    variant = _variant(variant)
+    _, T, d = values.shape
+    n = values.shape[0] if n_completed is None else n_completed
+    c, r = queries.shape
+    _check(load().lrar_block_phase1(variant, dtype_code(values), dtype_code(h_pre), _ptr(values), _ptr(keys),
+                                    _ptr(queries), n, c, T, d, r, eps, _ptr(h_pre), _ptr(lse_pre), _stream(stream)))
+
+
+def block_phase2(variant, h_pre: torch.Tensor, lse_pre: torch.Tensor, partial: torch.Tensor,
+                 partial_key: torch.Tensor | None, query: torch.Tensor, h: torch.Tensor,
+                 lse: torch.Tensor | None = None, eps: float = DEFAULT_EPS, stream=None) -> None:
+    """lrar_block_phase2: one site's mix = phase-1 result (+) its partial-block summary."""
+    variant = _variant(variant)
+    T, d = partial.shape
+    r = query.numel()
+    _check(load().lrar_block_phase2(variant, dtype_code(partial), dtype_code(h_pre), dtype_code(h), _ptr(h_pre),
+                                    _ptr(lse_pre), _ptr(partial), _ptr(partial_key), _ptr(query), T, d, r, eps,
+                                    _ptr(h), _ptr(lse), _stream(stream)))
 
 
 def diagnostics(variant, values: torch.Tensor, keys: torch.Tensor | None, query: torch.Tensor | None,
