@@ -409,6 +409,113 @@ def run_profile_site(args):
                       "fwd_gbs": fb / f / 1e6, "bwd_gbs": bb / b / 1e6}), flush=True)
 
 
+def _median_ms(torch, fn, reps):
+    """Median CUDA-event time of fn() over reps back-to-back repetitions (after one warm-up)."""
+    fn()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    for a, b in evs:
+        a.record()
+        fn()
+        b.record()
+    torch.cuda.synchronize()
+    return statistics.median(a.elapsed_time(b) for a, b in evs)
+
+
+def run_suite(args):
+    """Every workload's headline site (not only the benchmark's): P-LR and its
+    rank sweep, full AttnRes keys, the d = 2048 decoder, and the Block AttnRes
+    forward sweep site by site against the two-phase path.  One JSON line each."""
+    import torch
+
+    from __graft_entry__ import build
+    from paper_2607_09694_gb300 import lrar, sites, synth
+
+    build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    peak, _ = _peaks()
+    reps = max(5, args.steps // 5)
+
+    def emit(d):
+        d["peak_gbs"] = peak
+        for k in list(d):
+            if k.endswith("_gbs") and k != "peak_gbs":
+                d[k.replace("_gbs", "_frac")] = d[k] / peak
+        print(json.dumps(d), flush=True)
+
+    def fwd_bwd(name, variant, T, d, r, n, seed, scale=None, h_dtype=torch.bfloat16):
+        vals = synth.values(n, T, d, seed, "bf16", scale, device=dev)
+        keys = synth.keys(n, T, r, seed, "bf16", device=dev) if variant == "projected" else None
+        q = synth.queries(1, r, seed, device=dev)[0].contiguous()
+        dh = synth.upstream(T, d, seed, "bf16", device=dev)
+        h = torch.empty(T, d, dtype=h_dtype, device=dev)
+        lse = torch.empty(T, device=dev)
+        dv = torch.zeros(n, T, d, dtype=torch.bfloat16, device=dev)
+        dk = torch.zeros(n, T, r, dtype=torch.bfloat16, device=dev) if keys is not None else None
+        dq = torch.empty(r, device=dev)
+        ws = torch.empty(lrar.workspace_size(variant, n, T, d, r) // 4, device=dev)
+        f = _median_ms(torch, lambda: lrar.forward(variant, vals, keys, q, h, lse, r=r), reps)
+        b = _median_ms(torch, lambda: lrar.backward(variant, vals, keys, q, dh, dv, dq, ws, dkeys=dk, h=h, lse=lse,
+                                                    r=r, accumulate=True), reps)
+        hb = 4 if h_dtype == torch.float32 else 2
+        shp = sites.SiteShape(variant, n, T, d, r, out_bytes=hb)
+        fb, bb = sites.forward_bytes(shp), sites.backward_bytes(shp)
+        emit({"suite": name, "variant": variant, "T": T, "d": d, "r": r, "n_src": n, "h_bytes": hb,
+              "fwd_ms": f, "bwd_ms": b, "fwd_gbs": fb / f / 1e6, "bwd_gbs": bb / b / 1e6,
+              "fwd_bwd_gbs": (fb + bb) / (f + b) / 1e6, "tokens_per_s": T / ((f + b) / 1e3)})
+        del vals, keys, dh, h, dv, dk
+        torch.cuda.empty_cache()
+
+    fwd_bwd("S-LR d1024 n49 r16 (reference for the rows below)", "sliced", 16384, 1024, 16, 49, 1, (0.5, 2.0))
+    for r in (4, 8, 16, 32, 64):
+        fwd_bwd(f"P-LR d1024 n49 r{r}", "projected", 16384, 1024, r, 49, 2)
+    fwd_bwd("full AttnRes keys d1024 n49 (fp32 h: exact gbar)", "full", 16384, 1024, 1024, 49, 1, (0.5, 2.0),
+            torch.float32)
+    fwd_bwd("full AttnRes keys d1024 n49 (bf16 h)", "full", 16384, 1024, 1024, 49, 1, (0.5, 2.0))
+    fwd_bwd("S-LR d2048 n65 r64 T32768", "sliced", 32768, 2048, 64, 65, 3)
+    fwd_bwd("Block S-LR site d2048 n9 r64 T32768", "sliced", 32768, 2048, 64, 9, 3)
+
+    # Block AttnRes forward sweep of the 32-layer decoder (64 outputs, c = 8):
+    # every site on its own versus the two-phase path.
+    T, d, r, c, M = 32768, 2048, 64, 8, 64
+    stack = synth.values(1 + M // c, T, d, 3, "bf16", device=dev)
+    qs = synth.queries(M + 1, r, 3, device=dev)
+    h = torch.empty(T, d, dtype=torch.bfloat16, device=dev)
+    lse = torch.empty(T, device=dev)
+
+    def naive():
+        for t in range(1, M + 2):
+            n = sites.block_num_sources(t, c)
+            lrar.forward("sliced", stack, None, qs[t - 1] if n > 1 else None, h, lse, n_src=n, r=r)
+
+    naive_bytes = sum(sites.forward_bytes(sites.SiteShape("sliced", sites.block_num_sources(t, c), T, d, r))
+                      for t in range(1, M + 2))
+    for pre_dtype, pb in ((torch.float32, 4), (torch.bfloat16, 2)):
+        h_pre = torch.empty(c, T, d, dtype=pre_dtype, device=dev)
+        lse_pre = torch.empty(c, T, device=dev)
+
+        def two_phase():
+            for b in range(M // c + 1):
+                ns = c if b < M // c else 1  # the final read site forms a block of one
+                t0 = b * c + 1
+                lrar.block_phase1("sliced", stack, None, qs[t0 - 1:t0 - 1 + ns], h_pre[:ns], lse_pre[:ns],
+                                  n_completed=1 + b)
+                for j in range(1, ns):
+                    lrar.block_phase2("sliced", h_pre[j], lse_pre[j], stack[1 + b], None, qs[t0 - 1 + j], h, lse)
+
+        tp_bytes = 0
+        for b in range(M // c + 1):
+            ns = c if b < M // c else 1
+            tp_bytes += T * ((1 + b) * d * 2 + ns * (d * pb + 4))
+            tp_bytes += (ns - 1) * T * (d * pb + 4 + d * 2 + d * 2 + 4 + 2 * r)
+        tn = _median_ms(torch, naive, max(3, reps // 2))
+        tt = _median_ms(torch, two_phase, max(3, reps // 2))
+        emit({"suite": "Block S-LR forward sweep, 65 sites, d2048 r64 c8 T32768", "h_pre_bytes": pb,
+              "per_site_ms": tn, "two_phase_ms": tt, "speedup": tn / tt, "per_site_bytes": naive_bytes,
+              "two_phase_bytes": tp_bytes, "per_site_gbs": naive_bytes / tn / 1e6,
+              "two_phase_gbs": tp_bytes / tt / 1e6})
+
+
 def run_e2e(wl, args, dist, dev, step_bytes, world):
     """The step through the public API with pinned host buffers: H2D of values,
     queries and upstream gradients, both sweeps, D2H of h, lse, dvalues and dq,
@@ -555,10 +662,13 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-site", type=int, default=0, help="time one site with this many sources (profiling)")
     ap.add_argument("--tokens", type=int, default=4096, help="tokens of the --profile-site case")
+    ap.add_argument("--suite", action="store_true", help="time every workload's headline site (JSON line each)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
-    if args.profile_site:
+    if args.suite:
+        run_suite(args)
+    elif args.profile_site:
         run_profile_site(args)
     elif args.impl == "reference":
         run_reference(args)

@@ -296,6 +296,10 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
 #define LRAR_KEY_BATCH 8
 #endif
 constexpr int kKeyBatch = LRAR_KEY_BATCH;  // key-pass loads a lane keeps in flight
+#ifndef LRAR_VEC_KEYPASS
+#define LRAR_VEC_KEYPASS 1
+#endif
+constexpr bool kVecKeyPass = LRAR_VEC_KEYPASS;
 template <int V, bool ACC> struct BwdStages {
 #ifdef LRAR_BWD_STAGES
     static constexpr int value = LRAR_BWD_STAGES;
@@ -303,6 +307,84 @@ template <int V, bool ACC> struct BwdStages {
     static constexpr int value = V >= 8 ? (ACC ? 2 : 3) : (ACC ? 3 : 5);
 #endif
 };
+
+// Key pass with 16-byte vectors, for keys that are whole aligned vectors
+// (key_vec) and whose row of NV = r / E vectors divides 32: lane l owns vector
+// jv = l mod NV of the key rows of sources l / NV, l / NV + 32 / NV, ...; it
+// loads a key vector and an old-gradient vector per source, writes the new
+// gradient vector, and keeps E dq parts that the lanes sharing jv combine with
+// a fixed butterfly.  S-LR slices are vector-aligned here, so no element of
+// the slice was touched by the value pass.
+template <typename T, bool ACC>
+__device__ __forceinline__ void key_pass_vec(const BwdParams &p, const T *__restrict__ values,
+                                             const T *__restrict__ keys, const T *__restrict__ dh,
+                                             T *__restrict__ dvalues, T *__restrict__ dkeys, int64_t x, int lane,
+                                             int tail0, const float *__restrict__ q_s, const float *a_s,
+                                             const float *s_s, const float *rho_s, const float *ds_s, float *dq_s) {
+    constexpr int E = VecE<T>::value;
+    constexpr int B = 4;  // sources per batch and lane
+    const int NV = p.r / E;
+    const int jv = lane % NV, kst = 32 / NV;
+    const int j0 = jv * E;
+    const int64_t src_stride = p.T * (int64_t)p.d;
+    const int64_t row_off = x * p.d;
+    float dqv[E];
+#pragma unroll
+    for (int t = 0; t < E; ++t) dqv[t] = 0.f;
+    for (int kb = lane / NV; kb < p.n; kb += kst * B) {
+        Frag<T, E> kf[B], of[B];
+#pragma unroll
+        for (int m = 0; m < B; ++m) {
+            const int k = kb + m * kst;
+            if (k < p.n) {
+                if (p.sliced) {
+                    const int64_t off = (int64_t)k * src_stride + row_off + tail0 + j0;
+                    kf[m].load_nc(values + off);
+                    if (ACC) of[m].load(dvalues + off);
+                    else of[m].zero();
+                } else {
+                    const int64_t off = ((int64_t)k * p.T + x) * p.r + j0;
+                    kf[m].load_nc(keys + off);
+                    if (ACC) of[m].load(dkeys + off);
+                    else of[m].zero();
+                }
+            }
+        }
+#pragma unroll
+        for (int m = 0; m < B; ++m) {
+            const int k = kb + m * kst;
+            if (k < p.n) {
+                const float rho = rho_s[k], s = s_s[k], ds = ds_s[k], a = a_s[k];
+                const float c1 = ds * rho, c2 = s * p.inv_r;
+                float kv[E], w[E], dhv[E];
+                kf[m].get(kv);
+                of[m].get(w);
+                if (p.sliced) {  // dh of the slice, re-read from L1 per source
+                    Frag<T, E> f;
+                    f.a = __ldg(reinterpret_cast<const uint4 *>(dh + row_off + tail0 + j0));
+                    f.get(dhv);
+                }
+#pragma unroll
+                for (int t = 0; t < E; ++t) {
+                    const float kbar = rho * kv[t];
+                    const float dk = c1 * (q_s[j0 + t] - c2 * kbar);
+                    dqv[t] = fmaf(ds, kbar, dqv[t]);
+                    w[t] += p.sliced ? fmaf(a, dhv[t], dk) : dk;
+                }
+                Frag<T, E> out;
+                out.set(w);
+                if (p.sliced) out.store(dvalues + (int64_t)k * src_stride + row_off + tail0 + j0);
+                else out.store(dkeys + ((int64_t)k * p.T + x) * p.r + j0);
+            }
+        }
+    }
+#pragma unroll
+    for (int t = 0; t < E; ++t) {
+        float v = dqv[t];
+        for (int off = NV; off < 32; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+        if (lane < NV) dq_s[j0 + t] += v;
+    }
+}
 
 // Key pass of one token (low-rank keys), with ds_i already in ds_s: writes the
 // key slice of dvalues (S-LR: old + alpha_i dh + dL/dk_i, one rounding) or the
@@ -397,7 +479,7 @@ __device__ __forceinline__ void key_pass(const BwdParams &p, const T *__restrict
     }
 }
 
-template <typename T, int V, int S, bool ACC>
+template <typename T, int V, int S, bool ACC, bool VK>
 __global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(const BwdParams p) {
     constexpr int E = VecE<T>::value;
     constexpr int P = ACC ? 2 : 1;  // planes per stage: o, old gradient
@@ -500,7 +582,12 @@ __global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(c
         __syncwarp();
         for (int k = lane; k < p.n; k += 32) g_s[k] = a_s[k] * (g_s[k] - gbar);
         __syncwarp();
-        key_pass<T, ACC>(p, values, keys, dh, dvalues, dkeys, x, lane, tail0, skip0, q_s, a_s, s_s, rho_s, g_s, dq_s);
+        if (VK)  // chosen on the host (vector_key_pass): only one pass is compiled in
+            key_pass_vec<T, ACC>(p, values, keys, dh, dvalues, dkeys, x, lane, tail0, q_s, a_s, s_s, rho_s, g_s,
+                                 dq_s);
+        else
+            key_pass<T, ACC>(p, values, keys, dh, dvalues, dkeys, x, lane, tail0, skip0, q_s, a_s, s_s, rho_s, g_s,
+                             dq_s);
         __syncwarp();
     }
     cp_async_wait_all();
@@ -737,6 +824,11 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
         p.key_vec = ((a.r * esz) % 16 == 0) && (((a.d - a.r) * esz) % 16 == 0);
     else
         p.key_vec = ((a.r * esz) % 16 == 0) && ((reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
+    // Vector key pass (key_pass_vec) when the keys are whole aligned vectors whose
+    // row divides a warp, except for accumulating keys of fewer than four vectors,
+    // where the scalar batches measured slightly faster.
+    constexpr int E = VecE<Tin>::value;
+    const bool vk = kVecKeyPass && p.key_vec && a.r % E == 0 && 32 % (a.r / E) == 0 && (!a.accumulate || a.r / E >= 4);
     const int64_t work = (a.T + kWarps - 1) / kWarps;
     const void *k;
     size_t smem;
@@ -748,8 +840,12 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
         smem = sizeof(float) * (size_t)round_up(a.d, 4) * (1 + kWarps);
         rq = a.d;
     } else if (kPipe) {
-        k = a.accumulate ? (const void *)bwd_lr_pipe_kernel<Tin, V, SA, true>
-                         : (const void *)bwd_lr_pipe_kernel<Tin, V, SN, false>;
+        if (vk)
+            k = a.accumulate ? (const void *)bwd_lr_pipe_kernel<Tin, V, SA, true, true>
+                             : (const void *)bwd_lr_pipe_kernel<Tin, V, SN, false, true>;
+        else
+            k = a.accumulate ? (const void *)bwd_lr_pipe_kernel<Tin, V, SA, true, false>
+                             : (const void *)bwd_lr_pipe_kernel<Tin, V, SN, false, false>;
         smem = (size_t)kWarps * (a.accumulate ? SA * 2 : SN) * V * 32 * 16 +
                sizeof(float) * ((size_t)round_up(a.r, 4) * (1 + kWarps) + (size_t)kWarps * 4 * kMaxSources);
         rq = a.r;
@@ -766,10 +862,14 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     const int grid = persistent_grid(k, kThreads, smem, work, kMaxPartials);
     if (a.variant == kFull)
         bwd_full_kernel<Tin, Tg, V, U><<<grid, kThreads, smem, s>>>(p);
+    else if (kPipe && a.accumulate && vk)
+        bwd_lr_pipe_kernel<Tin, V, SA, true, true><<<grid, kThreads, smem, s>>>(p);
     else if (kPipe && a.accumulate)
-        bwd_lr_pipe_kernel<Tin, V, SA, true><<<grid, kThreads, smem, s>>>(p);
+        bwd_lr_pipe_kernel<Tin, V, SA, true, false><<<grid, kThreads, smem, s>>>(p);
+    else if (kPipe && vk)
+        bwd_lr_pipe_kernel<Tin, V, SN, false, true><<<grid, kThreads, smem, s>>>(p);
     else if (kPipe)
-        bwd_lr_pipe_kernel<Tin, V, SN, false><<<grid, kThreads, smem, s>>>(p);
+        bwd_lr_pipe_kernel<Tin, V, SN, false, false><<<grid, kThreads, smem, s>>>(p);
     else if (a.accumulate)
         bwd_lr_kernel<Tin, Tg, V, UA, true><<<grid, kThreads, smem, s>>>(p);
     else
