@@ -601,26 +601,32 @@ __global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(c
 }
 
 // -------------------------------------------------------------- full keys
-template <typename Tin, typename Tg, int V>
+// One source row of the full-key backward, with lse and gbar = <dh, h> known:
+// alpha_i, g_i = <dh, o_i>, ds_i (Eq. 11-12), and the value gradient
+// alpha_i dh + ds_i rho_i (q - (s_i / d) kbar_i) written in one pass (the key
+// is the value, Eq. 13).  Operands stay packed and are unpacked one vector at
+// a time; q_s is zero past d.  dq accumulates in dqf: V * E registers, or with
+// DQS the warp's d floats in shared memory.
+template <typename Tin, typename Tg, int V, bool DQS = false>
 __device__ __forceinline__ void full_bwd_row(const Frag<Tin, VecE<Tin>::value> *f,
-                                             const Frag<Tg, VecE<Tin>::value> *old, const float *dhf,
+                                             const Frag<Tg, VecE<Tin>::value> *old,
+                                             const Frag<Tin, VecE<Tin>::value> *dhr,
                                              const float *__restrict__ q_s, float *dqf, float gbar, float lse,
                                              float inv_d, float eps, Tg *__restrict__ drow, int d, int lane,
-                                             int accumulate) {
+                                             bool accumulate) {
     constexpr int E = VecE<Tin>::value;
-    float o[V * E];
     float g = 0.f, ss = 0.f, qo = 0.f;
-#pragma unroll
-    for (int v = 0; v < V; ++v) f[v].get(o + v * E);
 #pragma unroll
     for (int v = 0; v < V; ++v) {
         const int e = (lane + 32 * v) * E;
+        float o[E], dv[E];
+        f[v].get(o);
+        dhr[v].get(dv);
 #pragma unroll
         for (int t = 0; t < E; ++t) {
-            const float qv = (e < d) ? q_s[e + t] : 0.f;
-            g = fmaf(dhf[v * E + t], o[v * E + t], g);
-            ss = fmaf(o[v * E + t], o[v * E + t], ss);
-            qo = fmaf(qv, o[v * E + t], qo);
+            g = fmaf(dv[t], o[t], g);
+            ss = fmaf(o[t], o[t], ss);
+            qo = fmaf(q_s[e + t], o[t], qo);
         }
     }
     g = warp_sum(g);
@@ -636,18 +642,20 @@ __device__ __forceinline__ void full_bwd_row(const Frag<Tin, VecE<Tin>::value> *
     for (int v = 0; v < V; ++v) {
         const int e = (lane + 32 * v) * E;
         if (e < d) {
-            float w[E];
+            float o[E], dv[E], w[E];
+            f[v].get(o);
+            dhr[v].get(dv);
             if (accumulate) old[v].get(w);
             else
 #pragma unroll
                 for (int t = 0; t < E; ++t) w[t] = 0.f;
 #pragma unroll
             for (int t = 0; t < E; ++t) {
-                const float ov = o[v * E + t];
-                w[t] = fmaf(a, dhf[v * E + t], w[t]);
+                w[t] = fmaf(a, dv[t], w[t]);
                 w[t] = fmaf(c1, q_s[e + t], w[t]);
-                w[t] = fmaf(-c2, ov, w[t]);
-                dqf[v * E + t] = fmaf(c1, ov, dqf[v * E + t]);
+                w[t] = fmaf(-c2, o[t], w[t]);
+                if (DQS) dqf[e + t] = fmaf(c1, o[t], dqf[e + t]);  // this warp's row in shared memory
+                else dqf[v * E + t] = fmaf(c1, o[t], dqf[v * E + t]);
             }
             Frag<Tg, E> out;
             out.set(w);
@@ -656,15 +664,170 @@ __device__ __forceinline__ void full_bwd_row(const Frag<Tin, VecE<Tin>::value> *
     }
 }
 
+// gbar = <dh, h> = sum_i alpha_i g_i for one token, from the saved output.
+template <typename Tin, int V>
+__device__ __forceinline__ float full_gbar(const BwdParams &p, const Frag<Tin, VecE<Tin>::value> *dhr, int64_t x,
+                                           int lane) {
+    constexpr int E = VecE<Tin>::value;
+    float gb = 0.f;
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+        const int e = (lane + 32 * v) * E;
+        if (e >= p.d) continue;
+        float dv[E], hv[E];
+        dhr[v].get(dv);
+        if (p.h_bf16) {
+            Frag<bf16, E> hf;
+            hf.load_nc(static_cast<const bf16 *>(p.h) + x * p.d + e);
+            hf.get(hv);
+        } else {
+            Frag<float, E> hf;
+            hf.load_nc(static_cast<const float *>(p.h) + x * p.d + e);
+            hf.get(hv);
+        }
+#pragma unroll
+        for (int t = 0; t < E; ++t) gb = fmaf(dv[t], hv[t], gb);
+    }
+    return warp_sum(gb);
+}
+
+// Write the CTA's dq partial (sum over its warps, fixed order) from each warp's
+// register accumulator dqf; scratch holds kWarps * round_up(d, 4) floats.
+template <typename Tin, int V, bool DQS = false>
+__device__ __forceinline__ void full_dq_partial(const BwdParams &p, const float *dqf, float *scratch, int lane,
+                                                int warp) {
+    constexpr int E = VecE<Tin>::value;
+    const int dp4 = DQS ? 32 * V * E : round_up(p.d, 4);  // with DQS the rows are already in scratch
+    float *dq_s = scratch + warp * dp4;
+    if (!DQS)
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int e = (lane + 32 * v) * E;
+            if (e < p.d)
+#pragma unroll
+                for (int t = 0; t < E; ++t) dq_s[e + t] = dqf[v * E + t];
+        }
+    __syncthreads();
+    for (int j = threadIdx.x; j < p.d; j += kThreads) {
+        float acc = 0.f;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) acc += scratch[w * dp4 + j];
+        p.partials[(int64_t)blockIdx.x * p.d + j] = acc;
+    }
+}
+
+// Bytes of the per-warp rings (cells of 16 bytes per lane), at least the dq
+// scratch of full_dq_partial that reuses them.
+__host__ __device__ inline size_t full_ring_bytes(int cells, int d) {
+    const size_t ring = (size_t)kWarps * cells * 32 * 16, dq = sizeof(float) * (size_t)kWarps * round_up(d, 4);
+    return ring > dq ? ring : dq;
+}
+
+// Full keys, one dtype for inputs and gradients: one warp per token, source
+// rows (and old gradients when accumulating) streamed through the per-lane
+// cp.async ring of the forward, S - 1 rows ahead and across tokens.  One CTA
+// per SM: dq, dh and a row stay in registers, and the deep ring keeps enough
+// bytes in flight for eight warps.
+template <typename T, int V, int S, bool ACC>
+__global__ void __launch_bounds__(kThreads, 1) bwd_full_pipe_kernel(const BwdParams p) {
+    constexpr int E = VecE<T>::value;
+    constexpr int P = ACC ? 2 : 1;
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    constexpr bool DQS = V * E > 32;  // dq in shared memory past 32 registers
+    const size_t ring_bytes = full_ring_bytes(S * P * V, p.d);
+    float *q_s = reinterpret_cast<float *>(smem_raw + ring_bytes);  // [32 V E], zero past d
+    // dq partials: per warp rows of 32 V E floats after q_s (DQS), else the drained ring
+    float *scratch = DQS ? q_s + 32 * V * E : reinterpret_cast<float *>(smem_raw);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int j = threadIdx.x; j < 32 * V * E; j += kThreads) q_s[j] = (p.query && j < p.d) ? p.query[j] : 0.f;
+    if (DQS)
+        for (int j = threadIdx.x; j < kWarps * 32 * V * E; j += kThreads) scratch[j] = 0.f;
+    __syncthreads();
+    const uint32_t ring_w = smem_u32(smem_raw) + (uint32_t)(warp * S * P * V * 32 * 16) + 16u * lane;
+
+    const T *__restrict__ values = static_cast<const T *>(p.values);
+    const T *__restrict__ dh = static_cast<const T *>(p.dh);
+    T *__restrict__ dvalues = static_cast<T *>(p.dvalues);
+    const int64_t src_stride = p.T * (int64_t)p.d;
+    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+    const float inv_d = 1.f / (float)p.d;
+    const int64_t x0 = (int64_t)blockIdx.x * kWarps + warp;
+
+    int64_t ix = x0;
+    int ii = 0;
+    auto cell = [&](int st, int plane, int v) -> uint32_t {
+        return ring_w + (uint32_t)((((st * P + plane) * V + v) * 32) * 16);
+    };
+    auto issue = [&](int st) {
+        if (ix < p.T) {
+            const int64_t off = ((int64_t)ii * p.T + ix) * p.d;
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) {
+                    cp_async16(cell(st, 0, v), values + off + e);
+                    if (ACC) cp_async16(cell(st, P - 1, v), dvalues + off + e);
+                }
+            }
+            if (++ii == p.n) {
+                ii = 0;
+                ix += nwarps;
+            }
+        }
+        cp_async_commit();
+    };
+#pragma unroll
+    for (int st = 0; st < S - 1; ++st) issue(st);
+    int st_c = 0, st_i = S - 1;
+    float dq_r[DQS ? 1 : V * E];
+#pragma unroll
+    for (int t = 0; t < (DQS ? 1 : V * E); ++t) dq_r[t] = 0.f;
+    float *dqf = DQS ? scratch + warp * 32 * V * E : dq_r;
+
+    for (int64_t x = x0; x < p.T; x += nwarps) {
+        const int64_t row_off = x * p.d;
+        Frag<T, E> dhr[V];
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int e = (lane + 32 * v) * E;
+            if (e < p.d) dhr[v].load_nc(dh + row_off + e);
+            else dhr[v].zero();
+        }
+        const float gbar = full_gbar<T, V>(p, dhr, x, lane);
+        const float lse = __ldg(p.lse + x);
+        for (int i = 0; i < p.n; ++i) {
+            issue(st_i);
+            cp_async_wait<S - 1>();
+            Frag<T, E> f[V], old[V];
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) f[v].a = ld_shared16(cell(st_c, 0, v));
+                else f[v].zero();
+                if (ACC && e < p.d) old[v].a = ld_shared16(cell(st_c, P - 1, v));
+                else old[v].zero();
+            }
+            full_bwd_row<T, T, V, DQS>(f, old, dhr, q_s, dqf, gbar, lse, inv_d, p.eps,
+                                       dvalues + (int64_t)i * src_stride + row_off, p.d, lane, ACC);
+            st_c = (st_c + 1 == S) ? 0 : st_c + 1;
+            st_i = (st_i + 1 == S) ? 0 : st_i + 1;
+        }
+    }
+    cp_async_wait_all();
+    __syncthreads();  // every warp is done with the ring before it becomes dq scratch
+    full_dq_partial<T, V, DQS>(p, dqf, scratch, lane, warp);
+}
+
+// Full keys with gradients in another dtype than the inputs: rows loaded into
+// registers, U at a time.
 template <typename Tin, typename Tg, int V, int U>
 __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(const BwdParams p) {
     constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
-    const int dp4 = round_up(p.d, 4);
-    float *q_s = smem;          // [d]
-    float *dq_all = q_s + dp4;  // [kWarps][d], used once at the end
+    float *q_s = smem;                    // [32 V E], zero past d
+    float *scratch = q_s + 32 * V * E;    // [kWarps][round_up(d, 4)], used once at the end
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int j = threadIdx.x; j < p.d; j += kThreads) q_s[j] = p.query ? p.query[j] : 0.f;
+    for (int j = threadIdx.x; j < 32 * V * E; j += kThreads) q_s[j] = (p.query && j < p.d) ? p.query[j] : 0.f;
     __syncthreads();
 
     const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
@@ -679,34 +842,14 @@ __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(co
 
     for (int64_t x = (int64_t)blockIdx.x * kWarps + warp; x < p.T; x += nwarps) {
         const int64_t row_off = x * p.d;
-        float dhf[V * E];
-        float gb = 0.f;
+        Frag<Tin, E> dhr[V];
 #pragma unroll
         for (int v = 0; v < V; ++v) {
             const int e = (lane + 32 * v) * E;
-            Frag<Tin, E> f;
-            if (e < p.d) f.load_nc(dh + row_off + e);
-            else f.zero();
-            f.get(dhf + v * E);
-            float hv[E];
-            if (e < p.d) {
-                if (p.h_bf16) {
-                    Frag<bf16, E> hf;
-                    hf.load_nc(static_cast<const bf16 *>(p.h) + row_off + e);
-                    hf.get(hv);
-                } else {
-                    Frag<float, E> hf;
-                    hf.load_nc(static_cast<const float *>(p.h) + row_off + e);
-                    hf.get(hv);
-                }
-            } else {
-#pragma unroll
-                for (int t = 0; t < E; ++t) hv[t] = 0.f;
-            }
-#pragma unroll
-            for (int t = 0; t < E; ++t) gb = fmaf(dhf[v * E + t], hv[t], gb);
+            if (e < p.d) dhr[v].load_nc(dh + row_off + e);
+            else dhr[v].zero();
         }
-        const float gbar = warp_sum(gb);  // <dh, h> = sum_i alpha_i g_i
+        const float gbar = full_gbar<Tin, V>(p, dhr, x, lane);
         const float lse = __ldg(p.lse + x);
         int i = 0;
         for (; i + U <= p.n; i += U) {
@@ -725,7 +868,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(co
                 }
 #pragma unroll
             for (int u = 0; u < U; ++u)
-                full_bwd_row<Tin, Tg, V>(f[u], old[u], dhf, q_s, dqf, gbar, lse, inv_d, p.eps,
+                full_bwd_row<Tin, Tg, V>(f[u], old[u], dhr, q_s, dqf, gbar, lse, inv_d, p.eps,
                                          dvalues + (int64_t)(i + u) * src_stride + row_off, p.d, lane, p.accumulate);
         }
         for (; i < p.n; ++i) {
@@ -740,26 +883,11 @@ __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(co
                 if (p.accumulate && e < p.d) old[v].load(dvalues + off);
                 else old[v].zero();
             }
-            full_bwd_row<Tin, Tg, V>(f, old, dhf, q_s, dqf, gbar, lse, inv_d, p.eps,
+            full_bwd_row<Tin, Tg, V>(f, old, dhr, q_s, dqf, gbar, lse, inv_d, p.eps,
                                      dvalues + (int64_t)i * src_stride + row_off, p.d, lane, p.accumulate);
         }
     }
-    // CTA partial of dq = sum ds_i rho_i o_i
-    float *dq_s = dq_all + warp * dp4;
-#pragma unroll
-    for (int v = 0; v < V; ++v) {
-        const int e = (lane + 32 * v) * E;
-        if (e < p.d)
-#pragma unroll
-            for (int t = 0; t < E; ++t) dq_s[e + t] = dqf[v * E + t];
-    }
-    __syncthreads();
-    for (int j = threadIdx.x; j < p.d; j += kThreads) {
-        float acc = 0.f;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) acc += dq_all[w * dp4 + j];
-        p.partials[(int64_t)blockIdx.x * p.d + j] = acc;
-    }
+    full_dq_partial<Tin, V>(p, dqf, scratch, lane, warp);
 }
 
 // Fixed-order sum of the CTA partials, dq[j] (+)= sum_b partials[b][j]: one
@@ -835,9 +963,19 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     int rq;
     constexpr bool kPipe = LRAR_BWD_PIPE && std::is_same<Tin, Tg>::value;
     constexpr int SA = BwdStages<V, true>::value, SN = BwdStages<V, false>::value;
+    // with dq in shared memory (V E > 32) the rings leave it room
+    constexpr int FB = V * E > 32 ? 32 : 48;
+    constexpr int FSA = FullStages<V, 2, FB>::value, FSN = FullStages<V, 1, FB>::value;
     if (a.variant == kFull) {
-        k = (const void *)bwd_full_kernel<Tin, Tg, V, U>;
-        smem = sizeof(float) * (size_t)round_up(a.d, 4) * (1 + kWarps);
+        if (kPipe) {
+            k = a.accumulate ? (const void *)bwd_full_pipe_kernel<Tin, V, FSA, true>
+                             : (const void *)bwd_full_pipe_kernel<Tin, V, FSN, false>;
+            smem = full_ring_bytes(a.accumulate ? FSA * 2 * V : FSN * V, a.d) +
+                   sizeof(float) * 32 * V * E * (V * E > 32 ? 1 + kWarps : 1);
+        } else {
+            k = (const void *)bwd_full_kernel<Tin, Tg, V, U>;
+            smem = sizeof(float) * (32 * V * E + (size_t)kWarps * round_up(a.d, 4));
+        }
         rq = a.d;
     } else if (kPipe) {
         if (vk)
@@ -860,7 +998,11 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
         if (e != cudaSuccess) return e;
     }
     const int grid = persistent_grid(k, kThreads, smem, work, kMaxPartials);
-    if (a.variant == kFull)
+    if (a.variant == kFull && kPipe && a.accumulate)
+        bwd_full_pipe_kernel<Tin, V, FSA, true><<<grid, kThreads, smem, s>>>(p);
+    else if (a.variant == kFull && kPipe)
+        bwd_full_pipe_kernel<Tin, V, FSN, false><<<grid, kThreads, smem, s>>>(p);
+    else if (a.variant == kFull)
         bwd_full_kernel<Tin, Tg, V, U><<<grid, kThreads, smem, s>>>(p);
     else if (kPipe && a.accumulate && vk)
         bwd_lr_pipe_kernel<Tin, V, SA, true, true><<<grid, kThreads, smem, s>>>(p);

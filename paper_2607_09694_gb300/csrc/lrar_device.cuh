@@ -151,4 +151,12 @@ __device__ __forceinline__ float warp_max(float v) {
 
 __host__ __device__ __forceinline__ int round_up(int a, int b) { return (a + b - 1) / b * b; }
 
+// Ring stages per warp for the full-key passes: about B * 4 KB of rows in
+// flight per CTA (P planes of V 16-byte vectors per lane and stage), at least
+// two.  B = 24 for two CTAs per SM, 48 for one.
+template <int V, int P, int B> struct FullStages {
+    static constexpr int raw = B / (V * P);
+    static constexpr int value = raw < 2 ? 2 : (raw > 8 ? 8 : raw);
+};
+
 }  // namespace lrar

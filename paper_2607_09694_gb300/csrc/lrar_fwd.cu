@@ -29,6 +29,7 @@ struct FwdParams {
     float eps, inv_r;
     int sliced;   // key = last r coordinates of the value row
     int key_vec;  // keys can be read as aligned 16-byte vectors
+    int chunks;   // warps per token row (low-rank forward): each mixes one 32 x V-vector chunk
 };
 
 // sum_j k_j^2 and sum_j q_j k_j of one key of r elements.
@@ -139,18 +140,24 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
     const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
     const int64_t src_stride = p.T * (int64_t)p.d;
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+    const int64_t items = p.T * p.chunks;
 
-    for (int64_t x = (int64_t)blockIdx.x * kWarps + warp; x < p.T; x += nwarps) {
+    // item = (token, chunk): rows wider than one warp's V vectors are split
+    // across warps, each of which recomputes the (cheap) routing of its token
+    for (int64_t it = (int64_t)blockIdx.x * kWarps + warp; it < items; it += nwarps) {
+        const int64_t x = it / p.chunks;
+        const int e0 = (int)(it - x * p.chunks) * 32 * V * E;  // first element of this chunk
+        const int dc = p.d - e0;                               // elements from the chunk start to the row end
         const float lse = lr_route<Tin>(values, keys, p.T, p.n, p.d, p.r, p.eps, p.inv_r, p.sliced, p.key_vec, x,
                                         lane, q_s, a_s, nullptr, nullptr);
-        if (lane == 0 && p.lse) p.lse[x] = lse;
+        if (lane == 0 && p.lse && e0 == 0) p.lse[x] = lse;
         __syncwarp();
 
         // Eq. (10): h = sum_i alpha_i o_i, fp32 accumulation.
         float acc[V * E];
 #pragma unroll
         for (int t = 0; t < V * E; ++t) acc[t] = 0.f;
-        const Tin *row0 = values + x * p.d;
+        const Tin *row0 = values + x * p.d + e0;
         int i = 0;
         for (; i + U <= p.n; i += U) {
             Frag<Tin, E> f[U][V];
@@ -159,7 +166,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
 #pragma unroll
                 for (int v = 0; v < V; ++v) {
                     const int e = (lane + 32 * v) * E;
-                    if (e < p.d) f[u][v].load_nc(row0 + (int64_t)(i + u) * src_stride + e);
+                    if (e < dc) f[u][v].load_nc(row0 + (int64_t)(i + u) * src_stride + e);
                     else f[u][v].zero();
                 }
 #pragma unroll
@@ -180,7 +187,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
             for (int v = 0; v < V; ++v) {
                 const int e = (lane + 32 * v) * E;
                 Frag<Tin, E> f;
-                if (e < p.d) f.load_nc(row0 + (int64_t)i * src_stride + e);
+                if (e < dc) f.load_nc(row0 + (int64_t)i * src_stride + e);
                 else f.zero();
                 float o[E];
                 f.get(o);
@@ -188,25 +195,27 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
                 for (int t = 0; t < E; ++t) acc[v * E + t] = fmaf(a, o[t], acc[v * E + t]);
             }
         }
-        store_row<Tin, Tout, V>(static_cast<Tout *>(p.h) + x * p.d, p.d, lane, acc, 1.f);
+        store_row<Tin, Tout, V>(static_cast<Tout *>(p.h) + x * p.d + e0, dc, lane, acc, 1.f);
         __syncwarp();  // a_s is rewritten for the next token
     }
 }
 
 // ------------------------------------------------------- full keys -------
 template <typename Tin, int V>
-__device__ __forceinline__ void full_row_step(const Frag<Tin, VecE<Tin>::value> *f, const float *qf, float inv_d,
-                                              float eps, float &m, float &z, float *acc) {
+__device__ __forceinline__ void full_row_step(const Frag<Tin, VecE<Tin>::value> *f, const float *__restrict__ q_s,
+                                              int lane, float inv_d, float eps, float &m, float &z, float *acc) {
     constexpr int E = VecE<Tin>::value;
     float o[V * E];
     float ss = 0.f, qo = 0.f;
 #pragma unroll
     for (int v = 0; v < V; ++v) f[v].get(o + v * E);
 #pragma unroll
-    for (int t = 0; t < V * E; ++t) {
-        ss = fmaf(o[t], o[t], ss);
-        qo = fmaf(qf[t], o[t], qo);
-    }
+    for (int v = 0; v < V; ++v)
+#pragma unroll
+        for (int t = 0; t < E; ++t) {
+            ss = fmaf(o[v * E + t], o[v * E + t], ss);
+            qo = fmaf(q_s[(lane + 32 * v) * E + t], o[v * E + t], qo);  // q is zero past d
+        }
     ss = warp_sum(ss);
     qo = warp_sum(qo);
     const float s = rsqrtf(fmaf(ss, inv_d, eps)) * qo;  // Eq. (2) with RMSNorm(o_i) as the key
@@ -223,61 +232,75 @@ __device__ __forceinline__ void full_row_step(const Frag<Tin, VecE<Tin>::value> 
     for (int t = 0; t < V * E; ++t) acc[t] = fmaf(w, o[t], acc[t]);
 }
 
-template <typename Tin, typename Tout, int V, int U>
-__global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) fwd_full_kernel(const FwdParams p) {
+// One warp per token; each lane streams its own 16-byte vectors of the source
+// rows through a per-lane cp.async ring in shared memory (it reads back only
+// what it copied, so the wait_group alone orders the two), S - 1 rows ahead.
+// The ring runs across tokens: the next token's first rows travel while this
+// one finishes.  Scores and the mix use the online softmax of full_row_step.
+template <typename Tin, typename Tout, int V, int S>
+__global__ void __launch_bounds__(kThreads, (V * VecE<Tin>::value <= 32 ? 2 : 1)) fwd_full_kernel(const FwdParams p) {
     constexpr int E = VecE<Tin>::value;
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    float *q_s = reinterpret_cast<float *>(smem_raw + (size_t)kWarps * S * V * 32 * 16);  // [32 V E], zero past d
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    float qf[V * E];
-#pragma unroll
-    for (int v = 0; v < V; ++v)
-#pragma unroll
-        for (int t = 0; t < E; ++t) {
-            const int e = (lane + 32 * v) * E + t;
-            qf[v * E + t] = (p.query && e < p.d) ? __ldg(p.query + e) : 0.f;
-        }
+    for (int j = threadIdx.x; j < 32 * V * E; j += kThreads) q_s[j] = (p.query && j < p.d) ? p.query[j] : 0.f;
+    __syncthreads();
+    const uint32_t ring_w = smem_u32(smem_raw) + (uint32_t)(warp * S * V * 32 * 16) + 16u * lane;
     const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
-    const int64_t src_stride = p.T * (int64_t)p.d;
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     const float inv_d = 1.f / (float)p.d;
+    const int64_t x0 = (int64_t)blockIdx.x * kWarps + warp;
 
-    for (int64_t x = (int64_t)blockIdx.x * kWarps + warp; x < p.T; x += nwarps) {
+    int64_t ix = x0;  // next row to copy: source ii of token ix
+    int ii = 0;
+    auto cell = [&](int st, int v) -> uint32_t { return ring_w + (uint32_t)((st * V + v) * 32 * 16); };
+    auto issue = [&](int st) {
+        if (ix < p.T) {
+            const int64_t off = ((int64_t)ii * p.T + ix) * p.d;
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) cp_async16(cell(st, v), values + off + e);
+            }
+            if (++ii == p.n) {
+                ii = 0;
+                ix += nwarps;
+            }
+        }
+        cp_async_commit();
+    };
+#pragma unroll
+    for (int st = 0; st < S - 1; ++st) issue(st);
+    int st_c = 0, st_i = S - 1;
+
+    for (int64_t x = x0; x < p.T; x += nwarps) {
         float acc[V * E];
 #pragma unroll
         for (int t = 0; t < V * E; ++t) acc[t] = 0.f;
         float m = -INFINITY, z = 0.f;
-        const Tin *row0 = values + x * p.d;
-        int i = 0;
-        for (; i + U <= p.n; i += U) {
-            Frag<Tin, E> f[U][V];
-#pragma unroll
-            for (int u = 0; u < U; ++u)
-#pragma unroll
-                for (int v = 0; v < V; ++v) {
-                    const int e = (lane + 32 * v) * E;
-                    if (e < p.d) f[u][v].load_nc(row0 + (int64_t)(i + u) * src_stride + e);
-                    else f[u][v].zero();
-                }
-#pragma unroll
-            for (int u = 0; u < U; ++u) full_row_step<Tin, V>(f[u], qf, inv_d, p.eps, m, z, acc);
-        }
-        for (; i < p.n; ++i) {
+        for (int i = 0; i < p.n; ++i) {
+            issue(st_i);
+            cp_async_wait<S - 1>();  // this lane's copies of row i have landed
             Frag<Tin, E> f[V];
 #pragma unroll
             for (int v = 0; v < V; ++v) {
                 const int e = (lane + 32 * v) * E;
-                if (e < p.d) f[v].load_nc(row0 + (int64_t)i * src_stride + e);
+                if (e < p.d) f[v].a = ld_shared16(cell(st_c, v));
                 else f[v].zero();
             }
-            full_row_step<Tin, V>(f, qf, inv_d, p.eps, m, z, acc);
+            full_row_step<Tin, V>(f, q_s, lane, inv_d, p.eps, m, z, acc);
+            st_c = (st_c + 1 == S) ? 0 : st_c + 1;
+            st_i = (st_i + 1 == S) ? 0 : st_i + 1;
         }
         store_row<Tin, Tout, V>(static_cast<Tout *>(p.h) + x * p.d, p.d, lane, acc, 1.f / z);
         if (lane == 0 && p.lse) p.lse[x] = m + logf(z);
     }
+    cp_async_wait_all();
 }
 
 // ------------------------------------------------------------- launch ----
 template <typename Tin, typename Tout, int V>
-static cudaError_t launch_fwd_t(const FwdArgs &a, cudaStream_t s) {
+static cudaError_t launch_fwd_t(const FwdArgs &a, cudaStream_t s, int chunks = 1) {
     constexpr int U = V >= 8 ? 1 : (V == 4 ? 2 : 4);
     FwdParams p;
     p.values = a.values;
@@ -292,16 +315,23 @@ static cudaError_t launch_fwd_t(const FwdArgs &a, cudaStream_t s) {
     p.eps = a.eps;
     p.inv_r = 1.f / (float)a.r;
     p.sliced = a.variant == kSliced;
+    p.chunks = chunks;
     constexpr int esz = sizeof(Tin);
     if (a.variant == kSliced)
         p.key_vec = ((a.r * esz) % 16 == 0) && (((a.d - a.r) * esz) % 16 == 0);
     else
         p.key_vec = ((a.r * esz) % 16 == 0) && ((reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
-    const int64_t work = (a.T + kWarps - 1) / kWarps;
+    const int64_t work = (a.T * chunks + kWarps - 1) / kWarps;
     if (a.variant == kFull) {
-        const void *k = (const void *)fwd_full_kernel<Tin, Tout, V, U>;
-        const int grid = persistent_grid(k, kThreads, 0, work, 1 << 30);
-        fwd_full_kernel<Tin, Tout, V, U><<<grid, kThreads, 0, s>>>(p);
+        constexpr int S = FullStages<V, 1, 24>::value;
+        const size_t smem = (size_t)kWarps * S * V * 32 * 16 + sizeof(float) * 32 * V * VecE<Tin>::value;
+        const void *k = (const void *)fwd_full_kernel<Tin, Tout, V, S>;
+        if (smem > 48 * 1024) {
+            cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (e != cudaSuccess) return e;
+        }
+        const int grid = persistent_grid(k, kThreads, smem, work, 1 << 30);
+        fwd_full_kernel<Tin, Tout, V, S><<<grid, kThreads, smem, s>>>(p);
     } else {
         const size_t smem = sizeof(float) * (round_up(a.r, 4) + kWarps * kMaxSources);
         const void *k = (const void *)fwd_lr_kernel<Tin, Tout, V, U>;
@@ -322,6 +352,7 @@ static cudaError_t launch_fwd_w(const FwdArgs &a, cudaStream_t s) {
     if (vecs <= 32) return launch_fwd_t<Tin, Tout, 1>(a, s);
     if (vecs <= 64) return launch_fwd_t<Tin, Tout, 2>(a, s);
     if (vecs <= 128) return launch_fwd_t<Tin, Tout, 4>(a, s);
+    if (a.variant != kFull) return launch_fwd_t<Tin, Tout, 4>(a, s, (vecs + 127) / 128);  // rows split over warps
     return launch_fwd_t<Tin, Tout, 8>(a, s);
 }
 
@@ -422,6 +453,7 @@ static cudaError_t launch_diag_t(const FwdArgs &a, float *neff, float *mean_alph
     p.eps = a.eps;
     p.inv_r = 1.f / (float)a.r;
     p.sliced = a.variant == kSliced;
+    p.chunks = 1;
     constexpr int esz = sizeof(Tin);
     if (a.variant == kSliced)
         p.key_vec = ((a.r * esz) % 16 == 0) && (((a.d - a.r) * esz) % 16 == 0);

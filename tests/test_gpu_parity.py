@@ -156,12 +156,24 @@ def test_projected_key_widths(r):
     _check(si, H.run_gpu(si, "f32", "f32"), H.run_oracle(si), si.n, "rms")
 
 
-@pytest.mark.parametrize("d", [64, 200, 1016, 2048])
+@pytest.mark.parametrize("d", [64, 200, 1016, 1544, 2048])
 @pytest.mark.parametrize("variant", ["sliced", "full"])
 def test_widths(d, variant):
     """Row widths that do not fill a lane's vectors, and the widest row (V = 8)."""
     si = synth.site("slr", variant=variant, n=6, T=150, d=d, r=min(16, d))
     _check(si, H.run_gpu(si, "f32", "f32"), H.run_oracle(si), si.n, "rms")
+
+
+@pytest.mark.parametrize("d", [1544, 2048])
+@pytest.mark.parametrize("variant", ["sliced", "projected", "full"])
+@pytest.mark.parametrize("accumulate", [False, True])
+def test_wide_rows_bf16(d, variant, accumulate):
+    """Rows past 1024 bf16 elements with bf16 gradients: the low-rank forward
+    splits each row over several warps, full keys keep dq in shared memory."""
+    si = synth.site("slr", variant=variant, n=9, T=130, d=d, r=16 if variant != "full" else None)
+    init = _init(si, dtype=torch.bfloat16) if accumulate else None
+    got = H.run_gpu(si, H_OUT[variant], "bf16", accumulate=accumulate, init=init)
+    _check(si, got, H.run_oracle(si), si.n, "ulp", init=init)
 
 
 @pytest.mark.parametrize("d", [128, 512, 1024])
