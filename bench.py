@@ -390,22 +390,38 @@ def time_site(wl, n: int, accumulate: bool, reps: int):
 
 
 def run_profile_site(args):
-    """Small single-site case for profilers: --profile-site n, --tokens T."""
+    """Small single-site case for profilers: --profile-site n sources, --tokens T,
+    --site-variant / --site-d / --site-r (bf16 storage, accumulating backward)."""
     import torch
 
     from __graft_entry__ import build
-    from paper_2607_09694_gb300 import sites
+    from paper_2607_09694_gb300 import lrar, sites, synth
 
     build()
-    torch.cuda.set_device(0)
-    wl = Workload(torch.device("cuda", 0), T=args.tokens, n_sites=args.profile_site)
-    n = args.profile_site
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    n, T, d, variant = args.profile_site, args.tokens, args.site_d, args.site_variant
+    r = d if variant == "full" else args.site_r
+    vals = synth.values(n, T, d, 1, "bf16", (0.5, 2.0), device=dev)
+    keys = synth.keys(n, T, r, 2, "bf16", device=dev) if variant == "projected" else None
+    q = synth.queries(1, r, 1, device=dev)[0].contiguous()
+    dh = synth.upstream(T, d, 1, "bf16", device=dev)
+    h = torch.empty(T, d, dtype=torch.bfloat16, device=dev)
+    lse = torch.empty(T, device=dev)
+    dv = torch.zeros(n, T, d, dtype=torch.bfloat16, device=dev)
+    dk = torch.zeros(n, T, r, dtype=torch.bfloat16, device=dev) if keys is not None else None
+    dq = torch.empty(r, device=dev)
+    ws = torch.empty(max(1, lrar.workspace_size(variant, n, T, d, r) // 4), device=dev)
+    fwd = lambda: lrar.forward(variant, vals, keys, q, h, lse, r=r)
+    bwd = lambda: lrar.backward(variant, vals, keys, q, dh, dv, dq, ws, dkeys=dk, h=h, lse=lse, r=r, accumulate=True)
     for _ in range(args.warmup):
-        time_site(wl, n, True, 1)
-    f, b = time_site(wl, n, True, args.steps)
-    fb = sites.forward_bytes(sites.SiteShape("sliced", n, args.tokens, D, R))
-    bb = sites.backward_bytes(sites.SiteShape("sliced", n, args.tokens, D, R, accumulate=1))
-    print(json.dumps({"profile_site": n, "T": args.tokens, "fwd_ms": f, "bwd_ms": b,
+        fwd()
+        bwd()
+    f = _median_ms(torch, fwd, args.steps)
+    b = _median_ms(torch, bwd, args.steps)
+    shp = sites.SiteShape(variant, n, T, d, r, out_bytes=2)
+    fb, bb = sites.forward_bytes(shp), sites.backward_bytes(shp)
+    print(json.dumps({"profile_site": n, "variant": variant, "T": T, "d": d, "r": r, "fwd_ms": f, "bwd_ms": b,
                       "fwd_gbs": fb / f / 1e6, "bwd_gbs": bb / b / 1e6}), flush=True)
 
 
@@ -662,6 +678,10 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-site", type=int, default=0, help="time one site with this many sources (profiling)")
     ap.add_argument("--tokens", type=int, default=4096, help="tokens of the --profile-site case")
+    ap.add_argument("--site-variant", choices=["sliced", "projected", "full"], default="sliced",
+                    help="key variant of the --profile-site case")
+    ap.add_argument("--site-d", type=int, default=D, help="width d of the --profile-site case")
+    ap.add_argument("--site-r", type=int, default=R, help="key rank r of the --profile-site case (not full)")
     ap.add_argument("--suite", action="store_true", help="time every workload's headline site (JSON line each)")
     args = ap.parse_args()
     if args.warmup < 3:

@@ -605,7 +605,7 @@ __global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(c
 // alpha_i, g_i = <dh, o_i>, ds_i (Eq. 11-12), and the value gradient
 // alpha_i dh + ds_i rho_i (q - (s_i / d) kbar_i) written in one pass (the key
 // is the value, Eq. 13).  Operands stay packed and are unpacked one vector at
-// a time; q_s is zero past d.  dq accumulates in dqf: V * E registers, or with
+// a time; q_s (laid out by q_slot) is zero past d.  dq accumulates in dqf: V * E registers, or with
 // DQS the warp's d floats in shared memory.
 template <typename Tin, typename Tg, int V, bool DQS = false>
 __device__ __forceinline__ void full_bwd_row(const Frag<Tin, VecE<Tin>::value> *f,
@@ -617,16 +617,16 @@ __device__ __forceinline__ void full_bwd_row(const Frag<Tin, VecE<Tin>::value> *
     constexpr int E = VecE<Tin>::value;
     float g = 0.f, ss = 0.f, qo = 0.f;
 #pragma unroll
-    for (int v = 0; v < V; ++v) {
-        const int e = (lane + 32 * v) * E;
-        float o[E], dv[E];
+    for (int v = 0; v < V; ++v) {  // vectors past d are zero in f, dh and q
+        float o[E], dv[E], qv[E];
         f[v].get(o);
         dhr[v].get(dv);
+        q_get<E>(q_s, v, lane, qv);
 #pragma unroll
         for (int t = 0; t < E; ++t) {
             g = fmaf(dv[t], o[t], g);
             ss = fmaf(o[t], o[t], ss);
-            qo = fmaf(q_s[e + t], o[t], qo);
+            qo = fmaf(qv[t], o[t], qo);
         }
     }
     g = warp_sum(g);
@@ -642,9 +642,10 @@ __device__ __forceinline__ void full_bwd_row(const Frag<Tin, VecE<Tin>::value> *
     for (int v = 0; v < V; ++v) {
         const int e = (lane + 32 * v) * E;
         if (e < d) {
-            float o[E], dv[E], w[E];
+            float o[E], dv[E], w[E], qv[E];
             f[v].get(o);
             dhr[v].get(dv);
+            q_get<E>(q_s, v, lane, qv);
             if (accumulate) old[v].get(w);
             else
 #pragma unroll
@@ -652,7 +653,7 @@ __device__ __forceinline__ void full_bwd_row(const Frag<Tin, VecE<Tin>::value> *
 #pragma unroll
             for (int t = 0; t < E; ++t) {
                 w[t] = fmaf(a, dv[t], w[t]);
-                w[t] = fmaf(c1, q_s[e + t], w[t]);
+                w[t] = fmaf(c1, qv[t], w[t]);
                 w[t] = fmaf(-c2, o[t], w[t]);
                 if (DQS) dqf[e + t] = fmaf(c1, o[t], dqf[e + t]);  // this warp's row in shared memory
                 else dqf[v * E + t] = fmaf(c1, o[t], dqf[v * E + t]);
@@ -735,11 +736,11 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_full_pipe_kernel(const BwdPar
     extern __shared__ __align__(16) unsigned char smem_raw[];
     constexpr bool DQS = V * E > 32;  // dq in shared memory past 32 registers
     const size_t ring_bytes = full_ring_bytes(S * P * V, p.d);
-    float *q_s = reinterpret_cast<float *>(smem_raw + ring_bytes);  // [32 V E], zero past d
+    float *q_s = reinterpret_cast<float *>(smem_raw + ring_bytes);  // [32 V E] (q_slot), zero past d
     // dq partials: per warp rows of 32 V E floats after q_s (DQS), else the drained ring
     float *scratch = DQS ? q_s + 32 * V * E : reinterpret_cast<float *>(smem_raw);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int j = threadIdx.x; j < 32 * V * E; j += kThreads) q_s[j] = (p.query && j < p.d) ? p.query[j] : 0.f;
+    for (int j = threadIdx.x; j < 32 * V * E; j += kThreads) q_s[q_slot<E>(j)] = (p.query && j < p.d) ? p.query[j] : 0.f;
     if (DQS)
         for (int j = threadIdx.x; j < kWarps * 32 * V * E; j += kThreads) scratch[j] = 0.f;
     __syncthreads();
@@ -824,10 +825,10 @@ template <typename Tin, typename Tg, int V, int U>
 __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(const BwdParams p) {
     constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
-    float *q_s = smem;                    // [32 V E], zero past d
+    float *q_s = smem;                    // [32 V E] (q_slot), zero past d
     float *scratch = q_s + 32 * V * E;    // [kWarps][round_up(d, 4)], used once at the end
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int j = threadIdx.x; j < 32 * V * E; j += kThreads) q_s[j] = (p.query && j < p.d) ? p.query[j] : 0.f;
+    for (int j = threadIdx.x; j < 32 * V * E; j += kThreads) q_s[q_slot<E>(j)] = (p.query && j < p.d) ? p.query[j] : 0.f;
     __syncthreads();
 
     const Tin *__restrict__ values = static_cast<const Tin *>(p.values);

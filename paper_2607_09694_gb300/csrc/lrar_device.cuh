@@ -159,4 +159,22 @@ template <int V, int P, int B> struct FullStages {
     static constexpr int value = raw < 2 ? 2 : (raw > 8 ? 8 : raw);
 };
 
+// The query of a full-key row in shared memory, laid out so that a lane reads
+// the E coordinates of its vector v as E / 4 bank-conflict-free 16-byte loads:
+// row element e = (lane + 32 v) E + t sits at float ((v E/4 + t/4) 32 + lane) 4 + t % 4.
+template <int E> __device__ __forceinline__ int q_slot(int e) {
+    const int v = e / (32 * E), lane = (e / E) % 32, t = e % E;
+    return ((v * (E / 4) + t / 4) * 32 + lane) * 4 + (t % 4);
+}
+template <int E> __device__ __forceinline__ void q_get(const float *__restrict__ q_s, int v, int lane, float *qv) {
+#pragma unroll
+    for (int k = 0; k < E / 4; ++k) {
+        const float4 a = *reinterpret_cast<const float4 *>(q_s + ((v * (E / 4) + k) * 32 + lane) * 4);
+        qv[4 * k] = a.x;
+        qv[4 * k + 1] = a.y;
+        qv[4 * k + 2] = a.z;
+        qv[4 * k + 3] = a.w;
+    }
+}
+
 }  // namespace lrar

@@ -210,12 +210,15 @@ __device__ __forceinline__ void full_row_step(const Frag<Tin, VecE<Tin>::value> 
 #pragma unroll
     for (int v = 0; v < V; ++v) f[v].get(o + v * E);
 #pragma unroll
-    for (int v = 0; v < V; ++v)
+    for (int v = 0; v < V; ++v) {
+        float qv[E];
+        q_get<E>(q_s, v, lane, qv);  // q is zero past d
 #pragma unroll
         for (int t = 0; t < E; ++t) {
             ss = fmaf(o[v * E + t], o[v * E + t], ss);
-            qo = fmaf(q_s[(lane + 32 * v) * E + t], o[v * E + t], qo);  // q is zero past d
+            qo = fmaf(qv[t], o[v * E + t], qo);
         }
+    }
     ss = warp_sum(ss);
     qo = warp_sum(qo);
     const float s = rsqrtf(fmaf(ss, inv_d, eps)) * qo;  // Eq. (2) with RMSNorm(o_i) as the key
@@ -241,9 +244,9 @@ template <typename Tin, typename Tout, int V, int S>
 __global__ void __launch_bounds__(kThreads, (V * VecE<Tin>::value <= 32 ? 2 : 1)) fwd_full_kernel(const FwdParams p) {
     constexpr int E = VecE<Tin>::value;
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    float *q_s = reinterpret_cast<float *>(smem_raw + (size_t)kWarps * S * V * 32 * 16);  // [32 V E], zero past d
+    float *q_s = reinterpret_cast<float *>(smem_raw + (size_t)kWarps * S * V * 32 * 16);  // [32 V E] (q_slot), zero past d
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int j = threadIdx.x; j < 32 * V * E; j += kThreads) q_s[j] = (p.query && j < p.d) ? p.query[j] : 0.f;
+    for (int j = threadIdx.x; j < 32 * V * E; j += kThreads) q_s[q_slot<E>(j)] = (p.query && j < p.d) ? p.query[j] : 0.f;
     __syncthreads();
     const uint32_t ring_w = smem_u32(smem_raw) + (uint32_t)(warp * S * V * 32 * 16) + 16u * lane;
     const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
