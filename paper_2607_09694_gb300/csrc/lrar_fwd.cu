@@ -32,17 +32,30 @@ struct FwdParams {
     int chunks;   // warps per token row (low-rank forward): each mixes one 32 x V-vector chunk
 };
 
+// Staged keys in shared memory: key i of a token occupies `per` = r / E
+// 16-byte cells from cell i * per, piece c stored at cell i * per + key_swz(i, c).
+// The routing lane of source i reads the pieces of key i one at a time; the
+// swizzle spreads the eight lanes of a 16-byte access phase over all banks
+// (a power-of-two per; other widths are stored in order).
+__device__ __forceinline__ int key_swz(int i, int c, int per) {
+    if (per & (per - 1)) return c;
+    return per >= 8 ? c ^ (i & 7) : c ^ ((i * per >> 3) & (per - 1));
+}
+
 // sum_j k_j^2 and sum_j q_j k_j of one key of r elements.
+// With sw >= 0, kp points at a key staged in shared memory by stage_keys for
+// source sw, its pieces in key_swz order.
 template <typename Tin>
 __device__ __forceinline__ void key_stats(const Tin *__restrict__ kp, int r, const float *__restrict__ q_s,
-                                          bool vec, float &ss, float &qk) {
+                                          bool vec, float &ss, float &qk, int sw = -1) {
     ss = 0.f;
     qk = 0.f;
     if (vec) {
         constexpr int E = VecE<Tin>::value;
         for (int j = 0; j < r; j += E) {
             Frag<Tin, E> f;
-            f.load_nc(kp + j);
+            if (sw >= 0) f.a = *reinterpret_cast<const uint4 *>(kp + key_swz(sw, j / E, r / E) * E);
+            else f.load_nc(kp + j);
             float k[E];
             f.get(k);
 #pragma unroll
@@ -63,11 +76,13 @@ __device__ __forceinline__ void key_stats(const Tin *__restrict__ kp, int r, con
 // Routing stage for token x (Eq. 8-9): lane owns sources lane + 32k.
 // Leaves alpha_i in a_s[i] (and s_i, rho_i in s_s, rho_s when non-null);
 // returns lse = log sum_i exp(s_i) in every lane.
+// With kb_s, the token's keys are read from that shared buffer [n][r] (filled
+// by stage_keys) instead of global memory.
 template <typename Tin>
 __device__ __forceinline__ float lr_route(const Tin *__restrict__ values, const Tin *__restrict__ keys, int64_t T,
                                           int n, int d, int r, float eps, float inv_r, int sliced, int key_vec,
                                           int64_t x, int lane, const float *__restrict__ q_s, float *a_s, float *s_s,
-                                          float *rho_s) {
+                                          float *rho_s, const Tin *kb_s = nullptr) {
     float s_reg[kSrcRegs];
     float m = -INFINITY;
 #pragma unroll
@@ -75,9 +90,13 @@ __device__ __forceinline__ float lr_route(const Tin *__restrict__ values, const 
         const int i = lane + 32 * k;
         float s = -INFINITY;
         if (i < n) {
-            const Tin *kp = sliced ? values + ((int64_t)i * T + x) * d + (d - r) : keys + ((int64_t)i * T + x) * r;
             float ss, qk;
-            key_stats<Tin>(kp, r, q_s, key_vec != 0, ss, qk);
+            if (kb_s) {
+                key_stats<Tin>(kb_s + i * r, r, q_s, true, ss, qk, i);
+            } else {
+                const Tin *kp = sliced ? values + ((int64_t)i * T + x) * d + (d - r) : keys + ((int64_t)i * T + x) * r;
+                key_stats<Tin>(kp, r, q_s, key_vec != 0, ss, qk);
+            }
             const float rho = rsqrtf(fmaf(ss, inv_r, eps));
             s = rho * qk;
             if (s_s) {
@@ -124,8 +143,33 @@ __device__ __forceinline__ void store_row(Tout *__restrict__ hrow, int d, int la
     }
 }
 
+// Copy the n keys of token x (aligned 16-byte vectors) into the warp's shared
+// buffer kbuf with cp.async, one commit group; consecutive lanes take
+// consecutive pieces, so each instruction covers whole keys.  The caller waits
+// and syncs the warp before the routing lanes read them.
+template <typename Tin>
+__device__ __forceinline__ void stage_keys(const Tin *__restrict__ values, const Tin *__restrict__ keys, int64_t T,
+                                           int n, int d, int r, int sliced, int64_t x, int lane, uint32_t kbuf) {
+    constexpr int E = VecE<Tin>::value;
+    const int per = r / E;
+    const bool pow2 = (per & (per - 1)) == 0;
+    const int sh = 31 - __clz(per);
+    for (int j = lane; j < n * per; j += 32) {
+        const int i = pow2 ? j >> sh : j / per, c = j - i * per;
+        const Tin *src = sliced ? values + ((int64_t)i * T + x) * d + (d - r) + c * E
+                                : keys + ((int64_t)i * T + x) * r + c * E;
+        cp_async16(kbuf + 16u * (uint32_t)(i * per + key_swz(i, c, per)), src);
+    }
+    cp_async_commit();
+}
+
 // ------------------------------------------------- low-rank keys (LR) ----
-template <typename Tin, typename Tout, int V, int U>
+// KS: each warp stages its next token's keys in shared memory with cp.async
+// while it mixes the current token's last rows (kPrefetchRows before the end),
+// so the routing reads no global memory on its critical path.
+constexpr int kPrefetchRows = 8;
+
+template <typename Tin, typename Tout, int V, int U, bool KS>
 __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(const FwdParams p) {
     constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
@@ -133,6 +177,8 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
     float *a_all = smem + round_up(p.r, 4);                    // [kWarps][kMaxSources]
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     float *a_s = a_all + warp * kMaxSources;
+    const int kb_elems = round_up(p.n * p.r, 16 / (int)sizeof(Tin));  // per warp, whole 16-byte cells
+    Tin *kb_s = reinterpret_cast<Tin *>(a_all + kWarps * kMaxSources) + warp * kb_elems;
     for (int j = threadIdx.x; j < p.r; j += kThreads) q_s[j] = p.query ? p.query[j] : 0.f;
     __syncthreads();
 
@@ -144,14 +190,28 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
 
     // item = (token, chunk): rows wider than one warp's V vectors are split
     // across warps, each of which recomputes the (cheap) routing of its token
+    const uint32_t kbuf = smem_u32(kb_s);
+    const int pf_at = p.n > kPrefetchRows ? (p.n - kPrefetchRows) / U * U : 0;
+    if (KS && (int64_t)blockIdx.x * kWarps + warp < items)
+        stage_keys<Tin>(values, keys, p.T, p.n, p.d, p.r, p.sliced, ((int64_t)blockIdx.x * kWarps + warp) / p.chunks,
+                        lane, kbuf);
     for (int64_t it = (int64_t)blockIdx.x * kWarps + warp; it < items; it += nwarps) {
         const int64_t x = it / p.chunks;
         const int e0 = (int)(it - x * p.chunks) * 32 * V * E;  // first element of this chunk
         const int dc = p.d - e0;                               // elements from the chunk start to the row end
+        if (KS) {
+            cp_async_wait_all();
+            __syncwarp();  // every lane's pieces are visible to the warp
+        }
         const float lse = lr_route<Tin>(values, keys, p.T, p.n, p.d, p.r, p.eps, p.inv_r, p.sliced, p.key_vec, x,
-                                        lane, q_s, a_s, nullptr, nullptr);
+                                        lane, q_s, a_s, nullptr, nullptr, KS ? kb_s : nullptr);
         if (lane == 0 && p.lse && e0 == 0) p.lse[x] = lse;
-        __syncwarp();
+        __syncwarp();  // a_s written; kb_s free for the next token
+        bool staged = !KS || it + nwarps >= items;
+        auto stage_next = [&]() {
+            stage_keys<Tin>(values, keys, p.T, p.n, p.d, p.r, p.sliced, (it + nwarps) / p.chunks, lane, kbuf);
+            staged = true;
+        };
 
         // Eq. (10): h = sum_i alpha_i o_i, fp32 accumulation.
         float acc[V * E];
@@ -160,6 +220,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
         const Tin *row0 = values + x * p.d + e0;
         int i = 0;
         for (; i + U <= p.n; i += U) {
+            if (!staged && i == pf_at) stage_next();
             Frag<Tin, E> f[U][V];
 #pragma unroll
             for (int u = 0; u < U; ++u)
@@ -195,9 +256,11 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
                 for (int t = 0; t < E; ++t) acc[v * E + t] = fmaf(a, o[t], acc[v * E + t]);
             }
         }
+        if (!staged) stage_next();
         store_row<Tin, Tout, V>(static_cast<Tout *>(p.h) + x * p.d + e0, dc, lane, acc, 1.f);
         __syncwarp();  // a_s is rewritten for the next token
     }
+    if (KS) cp_async_wait_all();
 }
 
 // ------------------------------------------------------- full keys -------
@@ -302,6 +365,12 @@ __global__ void __launch_bounds__(kThreads, (V * VecE<Tin>::value <= 32 ? 2 : 1)
 }
 
 // ------------------------------------------------------------- launch ----
+#ifndef LRAR_STAGE_KEYS
+#define LRAR_STAGE_KEYS 1
+#endif
+constexpr bool kStageKeys = LRAR_STAGE_KEYS;
+constexpr size_t kStageKeyBytes = 12 * 1024;  // per warp
+
 template <typename Tin, typename Tout, int V>
 static cudaError_t launch_fwd_t(const FwdArgs &a, cudaStream_t s, int chunks = 1) {
     constexpr int U = V >= 8 ? 1 : (V == 4 ? 2 : 4);
@@ -336,14 +405,22 @@ static cudaError_t launch_fwd_t(const FwdArgs &a, cudaStream_t s, int chunks = 1
         const int grid = persistent_grid(k, kThreads, smem, work, 1 << 30);
         fwd_full_kernel<Tin, Tout, V, S><<<grid, kThreads, smem, s>>>(p);
     } else {
-        const size_t smem = sizeof(float) * (round_up(a.r, 4) + kWarps * kMaxSources);
-        const void *k = (const void *)fwd_lr_kernel<Tin, Tout, V, U>;
+        // Keys staged in shared memory when rows are split over warps (each warp
+        // routes its token, so routing weighs twice as much), the keys are whole
+        // aligned vectors and a warp's buffer leaves room for two CTAs per SM.
+        // At one warp per row staging measured neutral to slightly slower.
+        const size_t kb = (size_t)round_up(a.n * a.r, 16 / esz) * esz;
+        const bool ks = kStageKeys && chunks > 1 && p.key_vec && kb <= kStageKeyBytes;
+        const size_t smem = sizeof(float) * (round_up(a.r, 4) + kWarps * kMaxSources) + (ks ? kWarps * kb : 0);
+        const void *k = ks ? (const void *)fwd_lr_kernel<Tin, Tout, V, U, true>
+                           : (const void *)fwd_lr_kernel<Tin, Tout, V, U, false>;
         if (smem > 48 * 1024) {
             cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
             if (e != cudaSuccess) return e;
         }
         const int grid = persistent_grid(k, kThreads, smem, work, 1 << 30);
-        fwd_lr_kernel<Tin, Tout, V, U><<<grid, kThreads, smem, s>>>(p);
+        if (ks) fwd_lr_kernel<Tin, Tout, V, U, true><<<grid, kThreads, smem, s>>>(p);
+        else fwd_lr_kernel<Tin, Tout, V, U, false><<<grid, kThreads, smem, s>>>(p);
     }
     return cudaGetLastError();
 }

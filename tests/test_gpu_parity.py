@@ -176,6 +176,15 @@ def test_wide_rows_bf16(d, variant, accumulate):
     _check(si, got, H.run_oracle(si), si.n, "ulp", init=init)
 
 
+@pytest.mark.parametrize("variant,r,n", [("sliced", 12, 9), ("projected", 100, 9), ("sliced", 64, 100),
+                                          ("projected", 64, 65)])
+def test_wide_rows_key_shapes(variant, r, n):
+    """Split rows (d = 2048 bf16) whose keys are not whole 16-byte vectors, or
+    too many to stage in shared memory (n r > 6144), next to a staged case."""
+    si = synth.site("slr", variant=variant, n=n, T=90, d=2048, r=r)
+    _check(si, H.run_gpu(si, "f32", "f32"), H.run_oracle(si), si.n, "rms")
+
+
 @pytest.mark.parametrize("d", [128, 512, 1024])
 @pytest.mark.parametrize("variant", ["sliced", "projected", "full"])
 def test_fp32_widths(d, variant):
