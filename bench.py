@@ -491,6 +491,23 @@ def run_suite(args):
     fwd_bwd("S-LR d2048 n65 r64 T32768", "sliced", 32768, 2048, 64, 65, 3)
     fwd_bwd("Block S-LR site d2048 n9 r64 T32768", "sliced", 32768, 2048, 64, 9, 3)
 
+    # routing diagnostics (Eq. 16): reads only the keys (the S-LR tails, one 32-byte
+    # sector per row at r = 16), writes N_eff per token and the mean alpha per source
+    for variant, r, seed in (("sliced", 16, 1), ("projected", 32, 2)):
+        T, d, n = 16384, 1024, 49
+        vals = synth.values(n, T, d, seed, "bf16", (0.5, 2.0), device=dev)
+        keys = synth.keys(n, T, r, seed, "bf16", device=dev) if variant == "projected" else None
+        q = synth.queries(1, r, seed, std=1.0, device=dev)[0].contiguous()
+        neff = torch.empty(T, device=dev)
+        mean_alpha = torch.empty(n, device=dev)
+        ws = torch.empty(lrar.diagnostics_workspace_size(n) // 4, device=dev)
+        ms = _median_ms(torch, lambda: lrar.diagnostics(variant, vals, keys, q, neff, mean_alpha, ws, r=r), reps)
+        key_bytes = T * (n * r * 2 + 4)
+        emit({"suite": f"routing diagnostics {variant} d{d} n{n} r{r}", "T": T, "ms": ms, "key_bytes": key_bytes,
+              "key_gbs": key_bytes / ms / 1e6, "tokens_per_s": T / (ms / 1e3)})
+        del vals, keys
+        torch.cuda.empty_cache()
+
     # Block AttnRes forward sweep of the 32-layer decoder (64 outputs, c = 8):
     # every site on its own versus the two-phase path.
     T, d, r, c, M = 32768, 2048, 64, 8, 64
