@@ -57,10 +57,12 @@ def _load():
             lib.oracle_block_num_sources.argtypes = [i, i]
             lib.oracle_full_num_sources.argtypes = [i]
             lib.oracle_set_threads.argtypes = [i]
+            lib.oracle_projection.argtypes = [i, vp, vp, i64, i, i, i64p, i64, dp]
             lib.oracle_set_threads.restype = None
             for f in (lib.oracle_forward, lib.oracle_backward, lib.oracle_diagnostics,
                       lib.oracle_block_sources, lib.oracle_block_fanout,
-                      lib.oracle_block_num_sources, lib.oracle_full_num_sources, lib.oracle_get_threads):
+                      lib.oracle_block_num_sources, lib.oracle_full_num_sources, lib.oracle_get_threads,
+                      lib.oracle_projection):
                 f.restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -209,3 +211,22 @@ def block_fanout(dsources, t: int, c: int):
     if rc != 0:
         raise ValueError("oracle_block_fanout rejected its arguments")
     return out
+
+
+def projection(a, w, d: int, tokens=None):
+    """Eq. (11)-(12): [o; k] = [W_O; W_K] a per token; a [T, m], w [d + r, m].
+    Returns dict(o [n_tok, d], keys [n_tok, r]) in float64."""
+    aa, dt = _as_array(a)
+    wa, wdt = _as_array(w)
+    if wdt != dt:
+        raise TypeError("a and w must have the same element type")
+    T, m = aa.shape
+    nrows = wa.shape[0]
+    if wa.shape[1] != m or not 0 <= d <= nrows:
+        raise ValueError("w must be [d + r, m]")
+    tk, n_tok = _tok(tokens, T)
+    y = np.zeros((n_tok, nrows))
+    rc = _load().oracle_projection(dt, _ptr(aa), _ptr(wa), T, m, nrows, _ptr(tk), n_tok, _ptr(y))
+    if rc != 0:
+        raise ValueError("oracle_projection rejected its arguments")
+    return {"o": y[:, :d], "keys": y[:, d:]}

@@ -13,7 +13,9 @@
  *   Eq. (8)  lr_key_norm        kbar_i = RMSNorm(k_i), parameter-free (§3.2, App. A.5)
  *   Eq. (9)  lr_attnres_weight  alpha_i = softmax_i(q^T kbar_i), no temperature (§3.2)
  *   Eq. (10) lr_attnres_output  h = sum_i alpha_i o_i (§3.2)
- *   Eq. (12) fused_projection   P-LR keys are a separate input tensor (§3.3)
+ *   Eq. (12) fused_projection   P-LR keys are a separate input tensor of the mix
+ *                                (§3.3); oracle_projection evaluates Eq. (11)-(12)
+ *                                itself: [o; k] = [W_O; W_K] a
  *   Eq. (14) sliced_key         S-LR key = last r coordinates of o_i (§3.4)
  *   Eq. (2)  attnres_weight     AttnRes key = o_i itself, r = d (§3.1)
  *   Eq. (5), (6)                Block AttnRes summaries are plain sums (§3.1)
@@ -393,4 +395,32 @@ int oracle_diagnostics(int variant, int dtype, const void *values, const void *k
     free(alpha);
     free(h);
     return rc;
+}
+
+/*
+ * P-LR fused output projection, Eq. (11)-(12) (§3.3), for the listed tokens:
+ *   y[u][j] = sum_c w[j][c] a[x_u][c],   j = 0..nrows-1,
+ * where rows 0..d-1 of w are the ordinary output projection W_O (so y's first
+ * d columns are the sub-layer output o) and rows d..d+r-1 are the key rows
+ * W_K (the P-LR key k).  Eq. (13)'s embedding key is the case d = 0.
+ *   a [T, m], w [nrows, m] (element type dtype), y [n_tok, nrows] float64.
+ */
+int oracle_projection(int dtype, const void *a, const void *w, int64_t T, int m, int nrows,
+                      const int64_t *tokens, int64_t n_tok, double *y) {
+    if (!a || !w || !y || T < 0 || m < 1 || nrows < 1) return -1;
+    if (dtype < OR_F64 || dtype > OR_BF16) return -1;
+    if (!tokens) n_tok = T;
+    if (n_tok < 0) return -1;
+    for (int64_t u = 0; u < n_tok; ++u)
+        if (tokens && (tokens[u] < 0 || tokens[u] >= T)) return -1;
+#pragma omp parallel for schedule(static)
+    for (int64_t u = 0; u < n_tok; ++u) {
+        const int64_t x = tokens ? tokens[u] : u;
+        for (int j = 0; j < nrows; ++j) {
+            double acc = 0.0;
+            for (int c = 0; c < m; ++c) acc += elem(w, dtype, (int64_t)j * m + c) * elem(a, dtype, x * m + c);
+            y[u * nrows + j] = acc;
+        }
+    }
+    return 0;
 }

@@ -29,7 +29,7 @@ from dataclasses import dataclass, field
 
 import torch
 
-_TAGS = {"values": 1, "scale": 2, "keys": 3, "query": 4, "dh": 5, "outputs": 6}
+_TAGS = {"values": 1, "scale": 2, "keys": 3, "query": 4, "dh": 5, "outputs": 6, "proj_a": 7, "proj_w": 8}
 _CHUNK = 1 << 22
 _MASK = (1 << 62) - 1
 

@@ -37,6 +37,9 @@ MUTANTS = [
     ("block slot off by one", "int slot = (i == 0) ? 0 : 1 + (i - 1) / c;", "int slot = (i == 0) ? 0 : 1 + i / c;", 0),
     ("fan-out slot off by one", "int slot = (i == 0) ? 0 : 1 + (i - 1) / c;", "int slot = (i == 0) ? 0 : 1 + i / c;", 1),
     ("N_eff without exp", "neff[u] = exp(H);", "neff[u] = H;", 0),
+    ("projection with a transposed weight", "elem(w, dtype, (int64_t)j * m + c)", "elem(w, dtype, (int64_t)c * nrows + j)", 0),
+    ("projection drops the last input column", "for (int c = 0; c < m; ++c) acc +=", "for (int c = 0; c < m - 1; ++c) acc +=", 0),
+    ("projection reads token 0", "elem(a, dtype, x * m + c)", "elem(a, dtype, c)", 0),
 ]
 
 

@@ -305,3 +305,46 @@ def test_block_fanout_is_the_adjoint(t, c):
     dout = oracle.block_fanout(dsrc, t, c)
     assert abs(np.sum(dsrc * src) - np.sum(dout * outs)) < 1e-12
     assert src.shape[0] == oracle.block_num_sources(t, c)
+
+
+# ------------------------------------------------ P-LR fused projection ----
+def test_projection_matches_a_library_matmul():
+    """Eq. (11)-(12): [o; k] = [W_O; W_K] a equals numpy's float64 matmul of the
+    same operands (an independent routine), split after the first d rows."""
+    g = _rng(31)
+    T, m, d, r = 9, 24, 10, 6
+    a = g.standard_normal((T, m))
+    w = g.standard_normal((d + r, m))
+    out = oracle.projection(a, w, d)
+    y = a @ w.T
+    assert np.allclose(out["o"], y[:, :d], rtol=1e-13, atol=1e-13)
+    assert np.allclose(out["keys"], y[:, d:], rtol=1e-13, atol=1e-13)
+
+
+def test_projection_selects_rows():
+    """W_O = I gives o = a exactly; each W_K row a unit vector e_j picks a's
+    coordinate j (pins the split and catches a transposed operand)."""
+    g = _rng(32)
+    T, m, r = 4, 6, 3
+    a = g.standard_normal((T, m))
+    pick = [5, 0, 2]
+    w = np.concatenate([np.eye(m), np.eye(m)[pick]], axis=0)
+    out = oracle.projection(a, w, m)
+    assert np.array_equal(out["o"], a)
+    assert np.array_equal(out["keys"], a[:, pick])
+
+
+def test_projection_embedding_key_and_tokens():
+    """d = 0 is Eq. (13)'s embedding key k_0 = W_0^K o_0; evaluating listed
+    tokens equals the rows of the full run; bf16 words decode exactly."""
+    import torch
+
+    g = _rng(33)
+    T, m, r = 7, 16, 4
+    a = torch.from_numpy(g.standard_normal((T, m))).to(torch.bfloat16)
+    w = torch.from_numpy(g.standard_normal((r, m))).to(torch.bfloat16)
+    full = oracle.projection(a, w, 0)
+    assert full["o"].shape == (T, 0)
+    assert np.allclose(full["keys"], a.double().numpy() @ w.double().numpy().T, rtol=1e-13, atol=1e-13)
+    part = oracle.projection(a, w, 0, tokens=[6, 1])
+    assert np.array_equal(part["keys"], full["keys"][[6, 1]])
