@@ -225,6 +225,29 @@ int lrar_diagnostics(int variant, int in_dtype, const void *values, const void *
                      int n_src, int64_t T, int d, int r, float eps, float *neff, float *mean_alpha, void *workspace,
                      size_t workspace_bytes, void *stream);
 
+/*
+ * P-LR fused output projection (§3.3, Eq. 11-12) on the tensor cores:
+ *   [o ; k] = [W_O ; W_K] a    for every token, i.e.  Y = A W^T,  Y [T, d + r]
+ * Columns 0..d-1 of Y go to o, columns d..d+r-1 to keys, so a sub-layer's
+ * output projection writes its value slot and its key slot in one pass (the
+ * keys are never re-read to build the key stack).  With d = 0 it is Eq. 13's
+ * embedding key k_0 = W_0^K o_0.  bfloat16 operands, float32 accumulation,
+ * bfloat16 outputs rounded to nearest even.
+ *   a       [T, m] row-major activations entering the output projection
+ *           (m = d for attention, the SwiGLU hidden width for the FFN)
+ *   w       [d + r, m] row-major: the d rows of W_O, then the r rows of W_K
+ *   o       [T, d] (may be NULL when d == 0);  keys [T, r] (NULL when r == 0)
+ *   status  optional device int: set to 1 if a pipeline wait inside the kernel
+ *           gave up (about 2 s; then the outputs are not valid).  Never written
+ *           otherwise, so the caller zeroes it beforehand.
+ * in_dtype must be LRAR_BF16 (LRAR_ERR_UNSUPPORTED otherwise); m, d and r must
+ * be multiples of 8 and a, w, o, keys 16-byte aligned (LRAR_ERR_ALIGNMENT).
+ * T == 0 is a no-op.  No counterpart of the depth mix's other rules: the call
+ * reads a and w, writes o and keys, and is ordered on `stream` like every call.
+ */
+int lrar_project(int in_dtype, const void *a, const void *w, int64_t T, int m, int d, int r, void *o, void *keys,
+                 int *status, void *stream);
+
 /* Static text for a status code. */
 const char *lrar_strerror(int code);
 

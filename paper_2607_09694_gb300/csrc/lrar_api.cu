@@ -342,6 +342,25 @@ LRAR_API int lrar_block_phase2(int variant, int in_dtype, int pre_dtype, int out
     return LRAR_OK;
 }
 
+LRAR_API int lrar_project(int in_dtype, const void *a, const void *w, int64_t T, int m, int d, int r, void *o,
+                          void *keys, int *status, void *stream) {
+    if (!dtype_ok(in_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown input dtype %d", in_dtype);
+    if (in_dtype != LRAR_BF16) return fail(LRAR_ERR_UNSUPPORTED, "lrar_project takes bfloat16 operands");
+    if (T < 0 || m < 1 || d < 0 || r < 0 || d + r < 1)
+        return fail(LRAR_ERR_INVALID_ARG, "need T >= 0, m >= 1, d >= 0, r >= 0, d + r >= 1 (got T=%lld m=%d d=%d r=%d)",
+                    (long long)T, m, d, r);
+    if ((int64_t)d + r > 65535 * 176LL || T > (int64_t)0x7fffffff)
+        return fail(LRAR_ERR_UNSUPPORTED, "projection too large (T < 2^31, d + r <= 65535 * 176)");
+    if (m % 8 || d % 8 || r % 8) return fail(LRAR_ERR_ALIGNMENT, "m, d and r must be multiples of 8");
+    if (!a || !w) return fail(LRAR_ERR_INVALID_ARG, "a and w are required");
+    if ((d > 0 && !o) || (r > 0 && !keys)) return fail(LRAR_ERR_INVALID_ARG, "o (d > 0) and keys (r > 0) are required");
+    if (!aligned16(a) || !aligned16(w) || (o && !aligned16(o)) || (keys && !aligned16(keys)))
+        return fail(LRAR_ERR_ALIGNMENT, "a, w, o and keys must be 16-byte aligned");
+    if (status && !aligned4(status)) return fail(LRAR_ERR_ALIGNMENT, "status must be 4-byte aligned");
+    if (T == 0) return LRAR_OK;
+    return lrar::launch_project(a, w, T, m, d, r, o, keys, status, static_cast<cudaStream_t>(stream));
+}
+
 LRAR_API int lrar_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *src, int64_t count,
                                    float alpha, float beta, void *stream) {
     if (!dtype_ok(dst_dtype) || !dtype_ok(src_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown dtype");

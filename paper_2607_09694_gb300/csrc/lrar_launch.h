@@ -75,6 +75,11 @@ cudaError_t launch_block_phase2(const BlockPh2Args &a, cudaStream_t s);
 // Sets the calling thread's lrar_last_error() message; returns `code`.
 int record_error(int code, const char *message);
 
+// P-LR fused output projection on the tensor cores (lrar_proj.cu); returns an
+// LRAR status (argument checks done by the caller).
+int launch_project(const void *a, const void *w, int64_t T, int m, int d, int r, void *o, void *keys, int *status,
+                   cudaStream_t s);
+
 // Largest d one warp covers (the kernels keep a whole token row per warp).
 int max_width(int in_dtype);
 

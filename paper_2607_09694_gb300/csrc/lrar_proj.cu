@@ -1,0 +1,229 @@
+// lrar_proj.cu -- the P-LR fused output projection (§3.3, Eq. 11-12) on the
+// fifth-generation tensor cores:
+//
+//   [o ; k] = [W_O ; W_K] a      per token, i.e.  Y[T, d + r] = A[T, m] W[d + r, m]^T
+//
+// with the first d columns of Y written to the value slot o [T, d] and the last
+// r to the key slot k [T, r], so the keys land in the key stack of the mix
+// without a second pass.  (Eq. 13's embedding key, k_0 = W_0^K o_0, is the
+// same call with d = 0.)
+//
+// One CTA computes one 128 x kPN tile of Y:
+//   warp 4  one lane streams K-blocks of A and W (64 columns each) into a
+//           kPStages-deep shared-memory ring with TMA (128-byte swizzle);
+//   warp 5  allocates the fp32 accumulator in TMEM, and one lane issues
+//           tcgen05.mma (M = 128, N = kPN, K = 16) per 16 columns of a block,
+//           committing each block's MMAs to the barrier that frees its stage;
+//   warps 0-3  read the accumulator back with tcgen05.ld (warp w owns TMEM
+//           lanes 32w..32w+31, i.e. rows of the tile) and store bf16 rows.
+// Every wait on a barrier is bounded; a wait that runs out sets *status and
+// the kernel drains its copies and frees TMEM before it returns.
+#include <mutex>
+
+#include "lrar.h"
+#include "lrar_device.cuh"
+#include "lrar_launch.h"
+#include "lrar_sm100.cuh"
+
+namespace lrar {
+namespace {
+
+using namespace sm100;
+
+constexpr int kPM = 128;                        // tile rows (tokens), one TMEM lane each
+constexpr int kPN = 176;                        // tile columns of Y (1056 = 6 x 176)
+constexpr int kPK = 64;                         // K-block: 64 bf16 = one 128-byte swizzle row
+constexpr int kPStages = 4;                     // ring depth
+constexpr int kPThreads = 192;                  // 6 warps
+constexpr uint32_t kTmemCols = 256;             // power of two >= kPN
+constexpr int kABytes = kPM * kPK * 2;          // 16 KB
+constexpr int kBBytes = kPN * kPK * 2;          // 22 KB
+constexpr int kStageBytes = kABytes + kBBytes;  // multiple of 1024: every tile stays 1024-aligned
+constexpr size_t kProjSmem = (size_t)kPStages * kStageBytes + 1024 /* alignment slack */ + 256 /* barriers */;
+constexpr long long kWaitLimit = 4LL << 30;     // SM cycles (about 2 s) before a wait gives up
+
+static_assert(kStageBytes % 1024 == 0, "stage tiles must keep 1024-byte alignment");
+static_assert(kPN % 16 == 0 && kPN <= 256, "M = 128 MMA needs N a multiple of 16, at most 256");
+
+struct ProjParams {
+    bf16 *o;     // [T, d]
+    bf16 *keys;  // [T, r]
+    int64_t T;
+    int m, d, r;
+    int *status;  // set to 1 when a wait ran out (may be null)
+};
+
+__device__ __forceinline__ void report_timeout(int *status) {
+    if (status) atomicExch(status, 1);
+}
+
+__global__ void __launch_bounds__(kPThreads, 1)
+    proj_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_w,
+                const ProjParams p) {
+    extern __shared__ unsigned char smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;  // 128-byte swizzled tiles need 1024-byte alignment
+    const uint32_t bars = base + kPStages * kStageBytes;
+    auto full = [&](int s) { return bars + 8u * s; };               // TMA bytes of stage s landed
+    auto empty = [&](int s) { return bars + 8u * (kPStages + s); };  // MMAs reading stage s are done
+    const uint32_t acc_bar = bars + 16u * kPStages;                  // accumulator complete
+    const uint32_t tmem_slot = acc_bar + 8u;
+    auto stage_a = [&](int s) { return base + (uint32_t)(s * kStageBytes); };
+    auto stage_b = [&](int s) { return base + (uint32_t)(s * kStageBytes + kABytes); };
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t m0 = (int64_t)blockIdx.x * kPM;
+    const int n0 = blockIdx.y * kPN;
+    const int N = p.d + p.r;
+    const int nkb = (p.m + kPK - 1) / kPK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kPStages; ++s) {
+            mbar_init(full(s), 1);
+            mbar_init(empty(s), 1);
+        }
+        mbar_init(acc_bar, 1);
+        mbar_fence_init();
+    }
+    if (warp == 4 && lane == 0) {
+        tma_prefetch_map(&map_a);
+        tma_prefetch_map(&map_w);
+    }
+    if (warp == 5) {
+        tmem_alloc(tmem_slot, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(smem_raw + (tmem_slot - raw));
+
+    int issued = 0;  // K-blocks whose loads were issued (producer lane)
+    if (warp == 4 && lane == 0) {
+        for (int kb = 0; kb < nkb; ++kb) {
+            const int s = kb % kPStages;
+            const uint32_t round = (uint32_t)(kb / kPStages);
+            if (round > 0 && !mbar_wait(empty(s), (round - 1) & 1u, kWaitLimit)) {
+                report_timeout(p.status);
+                break;
+            }
+            mbar_arrive_expect_tx(full(s), (uint32_t)kStageBytes);
+            tma_load_2d(stage_a(s), &map_a, full(s), kb * kPK, (int)m0);
+            tma_load_2d(stage_b(s), &map_w, full(s), kb * kPK, n0);
+            issued = kb + 1;
+        }
+    } else if (warp == 5 && lane == 0) {
+        constexpr uint32_t idesc = idesc_bf16_f32(kPM, kPN);
+        for (int kb = 0; kb < nkb; ++kb) {
+            const int s = kb % kPStages;
+            if (!mbar_wait(full(s), (uint32_t)(kb / kPStages) & 1u, kWaitLimit)) {
+                report_timeout(p.status);
+                break;
+            }
+            tc_fence_after();
+            const uint64_t ad = sw128_kmajor_desc(stage_a(s)), bd = sw128_kmajor_desc(stage_b(s));
+#pragma unroll
+            for (int k = 0; k < kPK / 16; ++k)  // +32 bytes along K per step: +2 in the address field
+                tc_mma_f16(tmem, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
+            tc_commit(empty(s));
+        }
+        tc_commit(acc_bar);  // arrives once every MMA issued above has completed
+    } else if (warp < 4) {
+        const bool ok = mbar_wait(acc_bar, 0, kWaitLimit);
+        if (!ok && lane == 0) report_timeout(p.status);
+        tc_fence_after();
+        const int64_t row = m0 + warp * 32 + lane;
+        const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+#pragma unroll 1
+        for (int c0 = 0; c0 < kPN; c0 += 16) {
+            if (n0 + c0 >= N) break;  // warp-uniform
+            uint32_t v[16];
+            tc_ld16(trow + (uint32_t)c0, v);
+            tc_wait_ld();
+            if (!ok || row >= p.T) continue;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int col = n0 + c0 + 8 * h;  // 8 columns = one 16-byte store
+                if (col >= N) break;
+                float f[8];
+#pragma unroll
+                for (int t = 0; t < 8; ++t) f[t] = __uint_as_float(v[8 * h + t]);
+                Frag<bf16, 8> out;
+                out.set(f);
+                if (col < p.d) out.store(p.o + row * p.d + col);
+                else out.store(p.keys + row * p.r + (col - p.d));
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 4 && lane == 0) {
+        // Normally every load was consumed; after a timeout, wait (bounded) for
+        // the copies still in flight before the CTA's shared memory goes away.
+        for (int kb = issued - kPStages > 0 ? issued - kPStages : 0; kb < issued; ++kb)
+            if (!mbar_wait(full(kb % kPStages), (uint32_t)(kb / kPStages) & 1u, kWaitLimit)) report_timeout(p.status);
+    }
+    if (warp == 5) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(f);
+    });
+    return fn;
+}
+
+// Row-major bf16 matrix [rows, cols] read in boxes of box_rows x 64 columns,
+// 128-byte swizzle; reads past either edge return zeros.
+bool make_map(CUtensorMap *map, const void *ptr, int64_t rows, int cols, int box_rows) {
+    EncodeTiledFn fn = encode_tiled();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)kPK, (cuuint32_t)box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+int launch_project(const void *a, const void *w, int64_t T, int m, int d, int r, void *o, void *keys, int *status,
+                   cudaStream_t s) {
+    CUtensorMap map_a, map_w;
+    if (!make_map(&map_a, a, T, m, kPM) || !make_map(&map_w, w, d + r, m, kPN))
+        return record_error(LRAR_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point or arguments)");
+    cudaError_t e = cudaFuncSetAttribute(proj_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kProjSmem);
+    if (e != cudaSuccess) return record_error(LRAR_ERR_CUDA, cudaGetErrorString(e));
+    ProjParams p;
+    p.o = static_cast<bf16 *>(o);
+    p.keys = static_cast<bf16 *>(keys);
+    p.T = T;
+    p.m = m;
+    p.d = d;
+    p.r = r;
+    p.status = status;
+    const dim3 grid((unsigned)((T + kPM - 1) / kPM), (unsigned)((d + r + kPN - 1) / kPN));
+    proj_kernel<<<grid, kPThreads, kProjSmem, s>>>(map_a, map_w, p);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return record_error(LRAR_ERR_CUDA, cudaGetErrorString(e));
+    return LRAR_OK;
+}
+
+}  // namespace lrar

@@ -26,7 +26,7 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "liblrar.so")
 EXPORTS = ("lrar_forward", "lrar_backward", "lrar_backward_workspace_size", "lrar_block_accumulate",
            "lrar_strerror", "lrar_last_error", "lrar_version", "lrar_backward_noalloc", "lrar_diagnostics",
-           "lrar_diagnostics_workspace_size", "lrar_block_phase1", "lrar_block_phase2")
+           "lrar_diagnostics_workspace_size", "lrar_block_phase1", "lrar_block_phase2", "lrar_project")
 MAX_BLOCK_SITES = 64
 
 _lock = threading.Lock()
@@ -66,6 +66,8 @@ def load(path: str | None = None):
         lib.lrar_diagnostics_workspace_size.restype = sz
         lib.lrar_backward_workspace_size.argtypes = [i, i, i64, i, i]
         lib.lrar_backward_workspace_size.restype = sz
+        lib.lrar_project.argtypes = [i, vp, vp, i64, i, i, i, vp, vp, vp, vp]
+        lib.lrar_project.restype = i
         lib.lrar_block_accumulate.argtypes = [i, vp, i, vp, i64, f32, f32, vp]
         lib.lrar_block_accumulate.restype = i
         lib.lrar_strerror.argtypes = [i]
@@ -220,6 +222,20 @@ def block_accumulate(dst: torch.Tensor, src: torch.Tensor, alpha: float = 1.0, b
         raise ValueError("dst and src sizes differ")
     _check(load().lrar_block_accumulate(dtype_code(dst), _ptr(dst), dtype_code(src), _ptr(src), dst.numel(),
                                         float(alpha), float(beta), _stream(stream)))
+
+
+def project(a: torch.Tensor, w: torch.Tensor, o: torch.Tensor | None, keys: torch.Tensor | None,
+            status: torch.Tensor | None = None, stream=None) -> None:
+    """lrar_project: [o ; keys] = [W_O ; W_K] a per token (§3.3, Eq. 11-12).
+    a [T, m], w [d + r, m], o [T, d] (None when d = 0), keys [T, r] (None when r = 0),
+    all bfloat16; status: optional int32 device scalar set to 1 if the kernel gave up."""
+    T, m = a.shape
+    d = 0 if o is None else o.shape[-1]
+    r = 0 if keys is None else keys.shape[-1]
+    if w.shape[0] != d + r or w.shape[-1] != m:
+        raise ValueError(f"w must be [{d + r}, {m}], got {tuple(w.shape)}")
+    _check(load().lrar_project(dtype_code(a), _ptr(a), _ptr(w), T, m, d, r, _ptr(o), _ptr(keys), _ptr(status),
+                               _stream(stream)))
 
 
 def version() -> int:

@@ -172,3 +172,17 @@ def test_binding_raises_typed_error(lib):
 def test_missing_library_fails_loudly(tmp_path):
     with pytest.raises(RuntimeError, match="missing"):
         lrar.load(str(tmp_path / "nope.so"))
+
+
+def test_project_rejects(lib):
+    f = lib.lrar_project
+    assert f(0, FAKE, FAKE, 8, 64, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_UNSUPPORTED   # float32 operands
+    assert f(5, FAKE, FAKE, 8, 64, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_INVALID_ARG   # unknown dtype
+    assert f(1, FAKE, FAKE, 8, 64, 0, 0, None, None, None, None) == lrar.ERR_INVALID_ARG    # d + r == 0
+    assert f(1, FAKE, FAKE, 8, 0, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_INVALID_ARG   # m == 0
+    assert f(1, FAKE, FAKE, 8, 60, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_ALIGNMENT    # m % 8
+    assert f(1, FAKE, FAKE, 8, 64, 64, 12, FAKE, FAKE, None, None) == lrar.ERR_ALIGNMENT    # r % 8
+    assert f(1, None, FAKE, 8, 64, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_INVALID_ARG
+    assert f(1, FAKE, FAKE, 8, 64, 64, 16, None, FAKE, None, None) == lrar.ERR_INVALID_ARG  # o needed when d > 0
+    assert f(1, FAKE + 8, FAKE, 8, 64, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_ALIGNMENT
+    assert f(1, FAKE, FAKE, 0, 64, 64, 16, FAKE, FAKE, None, None) == lrar.OK                # T == 0: no-op
