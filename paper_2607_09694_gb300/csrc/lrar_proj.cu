@@ -8,16 +8,20 @@
 // without a second pass.  (Eq. 13's embedding key, k_0 = W_0^K o_0, is the
 // same call with d = 0.)
 //
-// One CTA computes one 128 x kPN tile of Y:
+// Persistent kernel, one CTA per SM walking the 128 x kPN tiles of Y:
 //   warp 4  one lane streams K-blocks of A and W (64 columns each) into a
-//           kPStages-deep shared-memory ring with TMA (128-byte swizzle);
-//   warp 5  allocates the fp32 accumulator in TMEM, and one lane issues
+//           kPStages-deep shared-memory ring with TMA (128-byte swizzle); the
+//           ring runs on across tiles;
+//   warp 5  allocates two fp32 accumulators in TMEM, and one lane issues
 //           tcgen05.mma (M = 128, N = kPN, K = 16) per 16 columns of a block,
-//           committing each block's MMAs to the barrier that frees its stage;
-//   warps 0-3  read the accumulator back with tcgen05.ld (warp w owns TMEM
-//           lanes 32w..32w+31, i.e. rows of the tile) and store bf16 rows.
-// Every wait on a barrier is bounded; a wait that runs out sets *status and
-// the kernel drains its copies and frees TMEM before it returns.
+//           committing each block's MMAs to the barrier that frees its stage
+//           and each finished tile to its accumulator's barrier;
+//   warps 0-3  read a finished accumulator back with tcgen05.ld (warp w owns
+//           TMEM lanes 32w..32w+31, i.e. rows of the tile) and store bf16 rows
+//           while the MMAs of the next tile fill the other accumulator.
+// Every wait on a barrier is bounded; a wait that runs out sets *status and a
+// shared abort flag that ends the other roles' waits, and the kernel drains
+// its copies and MMAs and frees TMEM before it returns.
 #include <mutex>
 
 #include "lrar.h"
@@ -33,9 +37,10 @@ using namespace sm100;
 constexpr int kPM = 128;                        // tile rows (tokens), one TMEM lane each
 constexpr int kPN = 176;                        // tile columns of Y (1056 = 6 x 176)
 constexpr int kPK = 64;                         // K-block: 64 bf16 = one 128-byte swizzle row
-constexpr int kPStages = 4;                     // ring depth
+constexpr int kPStages = 5;                     // ring depth
 constexpr int kPThreads = 192;                  // 6 warps
-constexpr uint32_t kTmemCols = 256;             // power of two >= kPN
+constexpr uint32_t kAccCols = 256;              // TMEM columns per accumulator (>= kPN)
+constexpr uint32_t kTmemCols = 2 * kAccCols;    // two accumulators: the whole TMEM of the SM
 constexpr int kABytes = kPM * kPK * 2;          // 16 KB
 constexpr int kBBytes = kPN * kPK * 2;          // 22 KB
 constexpr int kStageBytes = kABytes + kBBytes;  // multiple of 1024: every tile stays 1024-aligned
@@ -43,7 +48,7 @@ constexpr size_t kProjSmem = (size_t)kPStages * kStageBytes + 1024 /* alignment 
 constexpr long long kWaitLimit = 4LL << 30;     // SM cycles (about 2 s) before a wait gives up
 
 static_assert(kStageBytes % 1024 == 0, "stage tiles must keep 1024-byte alignment");
-static_assert(kPN % 16 == 0 && kPN <= 256, "M = 128 MMA needs N a multiple of 16, at most 256");
+static_assert(kPN % 16 == 0 && kPN <= (int)kAccCols, "M = 128 MMA needs N a multiple of 16 within an accumulator");
 
 struct ProjParams {
     bf16 *o;     // [T, d]
@@ -53,7 +58,8 @@ struct ProjParams {
     int *status;  // set to 1 when a wait ran out (may be null)
 };
 
-__device__ __forceinline__ void report_timeout(int *status) {
+__device__ __forceinline__ void give_up(int *status, volatile int *abort) {
+    *abort = 1;
     if (status) atomicExch(status, 1);
 }
 
@@ -64,25 +70,33 @@ __global__ void __launch_bounds__(kPThreads, 1)
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;  // 128-byte swizzled tiles need 1024-byte alignment
     const uint32_t bars = base + kPStages * kStageBytes;
-    auto full = [&](int s) { return bars + 8u * s; };               // TMA bytes of stage s landed
-    auto empty = [&](int s) { return bars + 8u * (kPStages + s); };  // MMAs reading stage s are done
-    const uint32_t acc_bar = bars + 16u * kPStages;                  // accumulator complete
-    const uint32_t tmem_slot = acc_bar + 8u;
+    auto full = [&](int s) { return bars + 8u * s; };                      // TMA bytes of stage s landed
+    auto empty = [&](int s) { return bars + 8u * (kPStages + s); };         // MMAs reading stage s are done
+    auto acc_full = [&](int b) { return bars + 8u * (2 * kPStages + b); };  // accumulator b holds a tile
+    auto acc_empty = [&](int b) { return bars + 8u * (2 * kPStages + 2 + b); };  // accumulator b was read
+    const uint32_t done_bar = bars + 8u * (2 * kPStages + 4);              // every MMA issued has completed
+    const uint32_t tmem_slot = done_bar + 8u;
+    volatile int *abort = reinterpret_cast<volatile int *>(smem_raw + (tmem_slot + 4u - raw));
     auto stage_a = [&](int s) { return base + (uint32_t)(s * kStageBytes); };
     auto stage_b = [&](int s) { return base + (uint32_t)(s * kStageBytes + kABytes); };
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t m0 = (int64_t)blockIdx.x * kPM;
-    const int n0 = blockIdx.y * kPN;
     const int N = p.d + p.r;
     const int nkb = (p.m + kPK - 1) / kPK;
+    const int n_nt = (N + kPN - 1) / kPN;
+    const int64_t n_tiles = (p.T + kPM - 1) / kPM * n_nt;  // tile t: rows (t / n_nt) * kPM, columns (t % n_nt) * kPN
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kPStages; ++s) {
             mbar_init(full(s), 1);
             mbar_init(empty(s), 1);
         }
-        mbar_init(acc_bar, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(acc_full(b), 1);
+            mbar_init(acc_empty(b), 4);  // one arrival per epilogue warp
+        }
+        mbar_init(done_bar, 1);
+        *abort = 0;
         mbar_fence_init();
     }
     if (warp == 4 && lane == 0) {
@@ -98,71 +112,105 @@ __global__ void __launch_bounds__(kPThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(smem_raw + (tmem_slot - raw));
 
-    int issued = 0;  // K-blocks whose loads were issued (producer lane)
+    int64_t issued = 0;  // K-blocks whose loads were issued (producer lane)
     if (warp == 4 && lane == 0) {
-        for (int kb = 0; kb < nkb; ++kb) {
-            const int s = kb % kPStages;
-            const uint32_t round = (uint32_t)(kb / kPStages);
-            if (round > 0 && !mbar_wait(empty(s), (round - 1) & 1u, kWaitLimit)) {
-                report_timeout(p.status);
-                break;
+        int64_t g = 0;
+        for (int64_t t = blockIdx.x; t < n_tiles && !*abort; t += gridDim.x) {
+            const int m0 = (int)(t / n_nt) * kPM, n0 = (int)(t % n_nt) * kPN;
+            for (int kb = 0; kb < nkb; ++kb, ++g) {
+                const int s = (int)(g % kPStages);
+                const uint32_t round = (uint32_t)(g / kPStages);
+                if (round > 0 && !mbar_wait(empty(s), (round - 1) & 1u, kWaitLimit, abort)) {
+                    give_up(p.status, abort);
+                    break;
+                }
+                mbar_arrive_expect_tx(full(s), (uint32_t)kStageBytes);
+                tma_load_2d(stage_a(s), &map_a, full(s), kb * kPK, m0);
+                tma_load_2d(stage_b(s), &map_w, full(s), kb * kPK, n0);
+                issued = g + 1;
             }
-            mbar_arrive_expect_tx(full(s), (uint32_t)kStageBytes);
-            tma_load_2d(stage_a(s), &map_a, full(s), kb * kPK, (int)m0);
-            tma_load_2d(stage_b(s), &map_w, full(s), kb * kPK, n0);
-            issued = kb + 1;
         }
     } else if (warp == 5 && lane == 0) {
         constexpr uint32_t idesc = idesc_bf16_f32(kPM, kPN);
-        for (int kb = 0; kb < nkb; ++kb) {
-            const int s = kb % kPStages;
-            if (!mbar_wait(full(s), (uint32_t)(kb / kPStages) & 1u, kWaitLimit)) {
-                report_timeout(p.status);
+        int64_t g = 0;
+        int it = 0;
+        for (int64_t t = blockIdx.x; t < n_tiles && !*abort; t += gridDim.x, ++it) {
+            const int b = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1);
+            if (use > 0 && !mbar_wait(acc_empty(b), (use - 1) & 1u, kWaitLimit, abort)) {
+                give_up(p.status, abort);
                 break;
             }
             tc_fence_after();
-            const uint64_t ad = sw128_kmajor_desc(stage_a(s)), bd = sw128_kmajor_desc(stage_b(s));
+            const uint32_t acc = tmem + b * kAccCols;
+            bool ok = true;
+            for (int kb = 0; kb < nkb; ++kb, ++g) {
+                const int s = (int)(g % kPStages);
+                if (!mbar_wait(full(s), (uint32_t)(g / kPStages) & 1u, kWaitLimit, abort)) {
+                    give_up(p.status, abort);
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint64_t ad = sw128_kmajor_desc(stage_a(s)), bd = sw128_kmajor_desc(stage_b(s));
 #pragma unroll
-            for (int k = 0; k < kPK / 16; ++k)  // +32 bytes along K per step: +2 in the address field
-                tc_mma_f16(tmem, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
-            tc_commit(empty(s));
-        }
-        tc_commit(acc_bar);  // arrives once every MMA issued above has completed
-    } else if (warp < 4) {
-        const bool ok = mbar_wait(acc_bar, 0, kWaitLimit);
-        if (!ok && lane == 0) report_timeout(p.status);
-        tc_fence_after();
-        const int64_t row = m0 + warp * 32 + lane;
-        const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-#pragma unroll 1
-        for (int c0 = 0; c0 < kPN; c0 += 16) {
-            if (n0 + c0 >= N) break;  // warp-uniform
-            uint32_t v[16];
-            tc_ld16(trow + (uint32_t)c0, v);
-            tc_wait_ld();
-            if (!ok || row >= p.T) continue;
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int col = n0 + c0 + 8 * h;  // 8 columns = one 16-byte store
-                if (col >= N) break;
-                float f[8];
-#pragma unroll
-                for (int t = 0; t < 8; ++t) f[t] = __uint_as_float(v[8 * h + t]);
-                Frag<bf16, 8> out;
-                out.set(f);
-                if (col < p.d) out.store(p.o + row * p.d + col);
-                else out.store(p.keys + row * p.r + (col - p.d));
+                for (int k = 0; k < kPK / 16; ++k)  // +32 bytes along K per step: +2 in the address field
+                    tc_mma_f16(acc, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
+                tc_commit(empty(s));
             }
+            if (!ok) break;
+            tc_commit(acc_full(b));
+        }
+        tc_commit(done_bar);  // arrives once every MMA issued above has completed
+        if (!mbar_wait(done_bar, 0, kWaitLimit)) give_up(p.status, abort);
+    } else if (warp < 4) {
+        int it = 0;
+        for (int64_t t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
+            const int b = it & 1;
+            // warp-uniform decision: tcgen05.ld below needs all 32 lanes
+            if (!__all_sync(0xffffffffu, mbar_wait(acc_full(b), (uint32_t)(it >> 1) & 1u, kWaitLimit, abort))) {
+                if (lane == 0) give_up(p.status, abort);
+                break;
+            }
+            tc_fence_after();
+            const int64_t row = (t / n_nt) * kPM + warp * 32 + lane;
+            const int n0 = (int)(t % n_nt) * kPN;
+            const uint32_t trow = tmem + b * kAccCols + ((uint32_t)(warp * 32) << 16);
+#pragma unroll 1
+            for (int c0 = 0; c0 < kPN; c0 += 16) {
+                if (n0 + c0 >= N) break;  // warp-uniform
+                uint32_t v[16];
+                tc_ld16(trow + (uint32_t)c0, v);
+                tc_wait_ld();
+                if (row >= p.T) continue;
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int col = n0 + c0 + 8 * h;  // 8 columns = one 16-byte store
+                    if (col >= N) break;
+                    float f[8];
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) f[q] = __uint_as_float(v[8 * h + q]);
+                    Frag<bf16, 8> out;
+                    out.set(f);
+                    if (col < p.d) out.store(p.o + row * p.d + col);
+                    else out.store(p.keys + row * p.r + (col - p.d));
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(acc_empty(b));  // this warp's rows of accumulator b are read
         }
     }
 
     tc_fence_before();
     __syncthreads();
     if (warp == 4 && lane == 0) {
-        // Normally every load was consumed; after a timeout, wait (bounded) for
+        // Normally every load was consumed; after giving up, wait (bounded) for
         // the copies still in flight before the CTA's shared memory goes away.
-        for (int kb = issued - kPStages > 0 ? issued - kPStages : 0; kb < issued; ++kb)
-            if (!mbar_wait(full(kb % kPStages), (uint32_t)(kb / kPStages) & 1u, kWaitLimit)) report_timeout(p.status);
+        for (int64_t g = issued - kPStages > 0 ? issued - kPStages : 0; g < issued; ++g)
+            if (!mbar_wait(full((int)(g % kPStages)), (uint32_t)(g / kPStages) & 1u, kWaitLimit)) {
+                if (p.status) atomicExch(p.status, 1);
+            }
     }
     if (warp == 5) {
         tc_fence_after();
@@ -219,7 +267,9 @@ int launch_project(const void *a, const void *w, int64_t T, int m, int d, int r,
     p.d = d;
     p.r = r;
     p.status = status;
-    const dim3 grid((unsigned)((T + kPM - 1) / kPM), (unsigned)((d + r + kPN - 1) / kPN));
+    const int64_t tiles = (T + kPM - 1) / kPM * ((d + r + kPN - 1) / kPN);
+    const int grid = persistent_grid((const void *)proj_kernel, kPThreads, kProjSmem, tiles, 1 << 30);
+    if (grid < 1) return record_error(LRAR_ERR_CUDA, "no SM can hold the projection kernel");
     proj_kernel<<<grid, kPThreads, kProjSmem, s>>>(map_a, map_w, p);
     e = cudaGetLastError();
     if (e != cudaSuccess) return record_error(LRAR_ERR_CUDA, cudaGetErrorString(e));

@@ -44,6 +44,20 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, long lo
     return true;
 }
 
+// The same, also giving up as soon as *abort (shared memory, set by another
+// role of the CTA that gave up) is non-zero.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, long long limit, volatile int *abort) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const long long t0 = clock64();
+    while (!mbar_try_wait(bar, parity))
+        if (*abort || clock64() - t0 > limit) return false;
+    return true;
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
 // ------------------------------------------------------------------ TMA ----
 // 2-D tile load into shared memory; completion is counted in bytes on bar.
 // x is the innermost coordinate (elements), y the row.
