@@ -22,6 +22,7 @@
 // Every wait on a barrier is bounded; a wait that runs out sets *status and a
 // shared abort flag that ends the other roles' waits, and the kernel drains
 // its copies and MMAs and frees TMEM before it returns.
+#include <cmath>
 #include <mutex>
 
 #include "lrar.h"
@@ -35,20 +36,23 @@ namespace {
 using namespace sm100;
 
 constexpr int kPM = 128;                        // tile rows (tokens), one TMEM lane each
-constexpr int kPN = 176;                        // tile columns of Y (1056 = 6 x 176)
 constexpr int kPK = 64;                         // K-block: 64 bf16 = one 128-byte swizzle row
 constexpr int kPStages = 5;                     // ring depth
 constexpr int kPThreads = 192;                  // 6 warps
-constexpr uint32_t kAccCols = 256;              // TMEM columns per accumulator (>= kPN)
+constexpr uint32_t kAccCols = 256;              // TMEM columns per accumulator (>= the tile width)
 constexpr uint32_t kTmemCols = 2 * kAccCols;    // two accumulators: the whole TMEM of the SM
 constexpr int kABytes = kPM * kPK * 2;          // 16 KB
-constexpr int kBBytes = kPN * kPK * 2;          // 22 KB
-constexpr int kStageBytes = kABytes + kBBytes;  // multiple of 1024: every tile stays 1024-aligned
-constexpr size_t kProjSmem = (size_t)kPStages * kStageBytes + 1024 /* alignment slack */ + 256 /* barriers */;
 constexpr long long kWaitLimit = 4LL << 30;     // SM cycles (about 2 s) before a wait gives up
 
-static_assert(kStageBytes % 1024 == 0, "stage tiles must keep 1024-byte alignment");
-static_assert(kPN % 16 == 0 && kPN <= (int)kAccCols, "M = 128 MMA needs N a multiple of 16 within an accumulator");
+// Tile width BN (columns of Y): 176 covers d + r = 1056 in 6 tiles, 160 in 7
+// with a better balanced last wave; the host picks per call.
+template <int BN> struct ProjTile {
+    static constexpr int kBBytes = BN * kPK * 2;
+    static constexpr int kStageBytes = kABytes + kBBytes;  // multiple of 1024: tiles stay 1024-aligned
+    static constexpr size_t kSmem = (size_t)kPStages * kStageBytes + 1024 /* alignment slack */ + 256 /* barriers */;
+    static_assert(kStageBytes % 1024 == 0, "stage tiles must keep 1024-byte alignment");
+    static_assert(BN % 16 == 0 && BN <= (int)kAccCols, "M = 128 MMA needs N a multiple of 16 within an accumulator");
+};
 
 struct ProjParams {
     bf16 *o;     // [T, d]
@@ -63,9 +67,11 @@ __device__ __forceinline__ void give_up(int *status, volatile int *abort) {
     if (status) atomicExch(status, 1);
 }
 
+template <int kPN>
 __global__ void __launch_bounds__(kPThreads, 1)
     proj_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_w,
                 const ProjParams p) {
+    constexpr int kStageBytes = ProjTile<kPN>::kStageBytes;
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;  // 128-byte swizzled tiles need 1024-byte alignment
@@ -250,14 +256,14 @@ bool make_map(CUtensorMap *map, const void *ptr, int64_t rows, int cols, int box
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-}  // namespace
-
-int launch_project(const void *a, const void *w, int64_t T, int m, int d, int r, void *o, void *keys, int *status,
-                   cudaStream_t s) {
-    CUtensorMap map_a, map_w;
-    if (!make_map(&map_a, a, T, m, kPM) || !make_map(&map_w, w, d + r, m, kPN))
+template <int BN>
+int launch_project_t(const CUtensorMap &map_a, const void *w, int64_t T, int m, int d, int r, void *o, void *keys,
+                     int *status, cudaStream_t s) {
+    CUtensorMap map_w;
+    if (!make_map(&map_w, w, d + r, m, BN))
         return record_error(LRAR_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point or arguments)");
-    cudaError_t e = cudaFuncSetAttribute(proj_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kProjSmem);
+    constexpr size_t smem = ProjTile<BN>::kSmem;
+    cudaError_t e = cudaFuncSetAttribute(proj_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return record_error(LRAR_ERR_CUDA, cudaGetErrorString(e));
     ProjParams p;
     p.o = static_cast<bf16 *>(o);
@@ -267,13 +273,37 @@ int launch_project(const void *a, const void *w, int64_t T, int m, int d, int r,
     p.d = d;
     p.r = r;
     p.status = status;
-    const int64_t tiles = (T + kPM - 1) / kPM * ((d + r + kPN - 1) / kPN);
-    const int grid = persistent_grid((const void *)proj_kernel, kPThreads, kProjSmem, tiles, 1 << 30);
+    const int64_t tiles = (T + kPM - 1) / kPM * ((d + r + BN - 1) / BN);
+    const int grid = persistent_grid((const void *)proj_kernel<BN>, kPThreads, smem, tiles, 1 << 30);
     if (grid < 1) return record_error(LRAR_ERR_CUDA, "no SM can hold the projection kernel");
-    proj_kernel<<<grid, kPThreads, kProjSmem, s>>>(map_a, map_w, p);
+    proj_kernel<BN><<<grid, kPThreads, smem, s>>>(map_a, map_w, p);
     e = cudaGetLastError();
     if (e != cudaSuccess) return record_error(LRAR_ERR_CUDA, cudaGetErrorString(e));
     return LRAR_OK;
+}
+
+// Estimated useful fraction of the SMs' tile time for width BN: tiles over
+// whole waves of one tile per SM, times the share of computed columns kept.
+double tile_efficiency(int64_t T, int N, int BN, int sms) {
+    const int64_t nt = (N + BN - 1) / BN, tiles = (T + kPM - 1) / kPM * nt;
+    const double waves = (double)tiles / sms;
+    return waves / std::ceil(waves) * (double)N / (double)(nt * BN);
+}
+
+}  // namespace
+
+int launch_project(const void *a, const void *w, int64_t T, int m, int d, int r, void *o, void *keys, int *status,
+                   cudaStream_t s) {
+    CUtensorMap map_a;
+    if (!make_map(&map_a, a, T, m, kPM))
+        return record_error(LRAR_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point or arguments)");
+    int dev = 0, sms = 1;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    // 176 wins ties: its tile reads fewer bytes per multiply-add
+    if (tile_efficiency(T, d + r, 160, sms) > 1.02 * tile_efficiency(T, d + r, 176, sms))
+        return launch_project_t<160>(map_a, w, T, m, d, r, o, keys, status, s);
+    return launch_project_t<176>(map_a, w, T, m, d, r, o, keys, status, s);
 }
 
 }  // namespace lrar

@@ -90,6 +90,14 @@ def test_full_size_sampled_tokens():
     _compare(16384, 1024, 1024, 32, seed=9, tokens=tokens)
 
 
+def test_large_decoder_sampled_tokens():
+    """The d = 2048 decoder (m = d = 2048, r = 64, T = 32768): d + r = 2112 is
+    twelve 176-wide tiles, the other tile width of the kernel."""
+    g = np.random.default_rng(10)
+    tokens = np.sort(np.concatenate([g.choice(32768, 24, replace=False), [0, 32767]]))
+    _compare(32768, 2048, 2048, 64, seed=10, tokens=tokens)
+
+
 def test_keys_land_in_the_key_stack_of_the_mix():
     """Projected keys written straight into slot i of a [n, T, r] key stack are
     the keys the mix reads: the forward over that stack equals the oracle's
