@@ -226,6 +226,30 @@ int lrar_diagnostics(int variant, int in_dtype, const void *values, const void *
                      size_t workspace_bytes, void *stream);
 
 /*
+ * Sources as separate tensors (a pointer table instead of one stacked buffer):
+ * every argument and rule is that of lrar_forward / lrar_backward, except
+ *   values   HOST array of n_src device pointers; values[i] is source i's
+ *            row-major [T, d] matrix (16-byte aligned)
+ *   keys     HOST array of n_src pointers to [T, r] P-LR key matrices
+ *            (LRAR_PROJECTED only, else ignored)
+ *   dvalues, dkeys  HOST arrays of n_src pointers to the matching gradient
+ *            matrices (each [T, d] / [T, r] of grad_dtype)
+ * The arrays are read during the call and copied into the launch, so they
+ * may be reused as soon as the call returns (a captured CUDA graph keeps the
+ * pointers it saw).  A NULL array, a NULL entry or an unaligned entry is
+ * rejected (LRAR_ERR_INVALID_ARG / LRAR_ERR_ALIGNMENT) before anything runs.
+ * Gradient matrices of different sources must not overlap.
+ */
+int lrar_forward_ptrs(int variant, int in_dtype, int out_dtype, const void *const *values, const void *const *keys,
+                      const float *query, int n_src, int64_t T, int d, int r, float eps, void *h, float *lse,
+                      void *stream);
+int lrar_backward_ptrs(int variant, int in_dtype, int grad_dtype, const void *const *values,
+                       const void *const *keys, const float *query, int n_src, int64_t T, int d, int r, float eps,
+                       const void *dh, const void *h, int h_dtype, const float *lse, void *const *dvalues,
+                       void *const *dkeys, float *dq, int accumulate, void *workspace, size_t workspace_bytes,
+                       void *stream);
+
+/*
  * P-LR fused output projection (§3.3, Eq. 11-12) on the tensor cores:
  *   [o ; k] = [W_O ; W_K] a    for every token, i.e.  Y = A W^T,  Y [T, d + r]
  * Columns 0..d-1 of Y go to o, columns d..d+r-1 to keys, so a sub-layer's

@@ -121,18 +121,31 @@ LRAR_API const char *lrar_strerror(int code) {
     }
 }
 
-LRAR_API int lrar_forward(int variant, int in_dtype, int out_dtype, const void *values, const void *keys,
-                          const float *query, int n_src, int64_t T, int d, int r, float eps, void *h, float *lse,
-                          void *stream) {
-    int rc = check_shape(variant, in_dtype, n_src, T, d, r, eps);
-    if (rc) return rc;
-    if (!dtype_ok(out_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown output dtype %d", out_dtype);
-    if (T == 0) return LRAR_OK;
-    if (!values || !h) return fail(LRAR_ERR_INVALID_ARG, "values and h are required");
-    if (variant == LRAR_PROJECTED && !keys) return fail(LRAR_ERR_INVALID_ARG, "projected keys are required");
+namespace {
+
+// Source tables of a stacked [n, T, width] buffer: entry i = base + i * T * width.
+void stack_table(const void *base, int n, int64_t T, int width, int esz, const void **tab) {
+    for (int i = 0; i < n; ++i)
+        tab[i] = base ? static_cast<const char *>(base) + (size_t)i * (size_t)T * (size_t)width * (size_t)esz
+                      : nullptr;
+}
+
+// Every entry of a caller's source table present and 16-byte aligned.
+int check_table(const void *const *tab, int n, const char *what) {
+    if (!tab) return fail(LRAR_ERR_INVALID_ARG, "%s table is required", what);
+    for (int i = 0; i < n; ++i) {
+        if (!tab[i]) return fail(LRAR_ERR_INVALID_ARG, "%s[%d] is NULL", what, i);
+        if (!aligned16(tab[i])) return fail(LRAR_ERR_ALIGNMENT, "%s[%d] must be 16-byte aligned", what, i);
+    }
+    return LRAR_OK;
+}
+
+int forward_impl(int variant, int in_dtype, int out_dtype, const void *const *values, const void *const *keys,
+                 const float *query, int n_src, int64_t T, int d, int r, float eps, void *h, float *lse,
+                 void *stream) {
+    if (!h) return fail(LRAR_ERR_INVALID_ARG, "h is required");
     if (!query && n_src > 1) return fail(LRAR_ERR_INVALID_ARG, "query is required when n_src > 1");
-    if (!aligned16(values) || !aligned16(h) || (variant == LRAR_PROJECTED && !aligned16(keys)) ||
-        (query && !aligned4(query)) || (lse && !aligned4(lse)))
+    if (!aligned16(h) || (query && !aligned4(query)) || (lse && !aligned4(lse)))
         return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (query and lse 4-byte)");
     lrar::FwdArgs a;
     a.variant = variant;
@@ -153,42 +166,38 @@ LRAR_API int lrar_forward(int variant, int in_dtype, int out_dtype, const void *
     return LRAR_OK;
 }
 
-LRAR_API size_t lrar_backward_workspace_size(int variant, int n_src, int64_t T, int d, int r) {
-    (void)n_src;
-    (void)T;
-    const int rq = variant == LRAR_FULL ? d : r;
-    if (rq < 1) return 0;
-    return sizeof(float) * (size_t)lrar::kMaxPartials * (size_t)rq;
-}
-
-LRAR_API int lrar_backward(int variant, int in_dtype, int grad_dtype, const void *values, const void *keys,
-                           const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh,
-                           const void *h, int h_dtype, const float *lse, void *dvalues, void *dkeys, float *dq,
-                           int accumulate, void *workspace, size_t workspace_bytes, void *stream) {
+// Checks of the backward that do not depend on how the sources are passed;
+// returns 1 (with *early set to the status) when nothing is left to launch.
+int backward_common(int variant, int in_dtype, int grad_dtype, int n_src, int64_t T, int d, int r, float eps,
+                    int h_dtype, float *dq, int accumulate, void *stream, bool *done) {
+    *done = false;
     int rc = check_shape(variant, in_dtype, n_src, T, d, r, eps);
     if (rc) return rc;
     if (!dtype_ok(grad_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown gradient dtype %d", grad_dtype);
     if (accumulate != 0 && accumulate != 1) return fail(LRAR_ERR_INVALID_ARG, "accumulate must be 0 or 1");
     if (variant == LRAR_FULL && !dtype_ok(h_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown h dtype %d", h_dtype);
     if (!dq) return fail(LRAR_ERR_INVALID_ARG, "dq is required");
-    const int rq = variant == LRAR_FULL ? d : r;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (T == 0) {  // dq is a sum over no tokens
+        *done = true;
         if (!accumulate) {
-            cudaError_t e = cudaMemsetAsync(dq, 0, sizeof(float) * (size_t)rq, s);
+            const int rq = variant == LRAR_FULL ? d : r;
+            cudaError_t e = cudaMemsetAsync(dq, 0, sizeof(float) * (size_t)rq, static_cast<cudaStream_t>(stream));
             if (e != cudaSuccess) return cuda_fail(e, "lrar_backward");
         }
-        return LRAR_OK;
     }
-    if (!values || !dh || !dvalues) return fail(LRAR_ERR_INVALID_ARG, "values, dh and dvalues are required");
-    if (variant == LRAR_PROJECTED && (!keys || !dkeys))
-        return fail(LRAR_ERR_INVALID_ARG, "projected keys and dkeys are required");
+    return LRAR_OK;
+}
+
+int backward_impl(int variant, int in_dtype, int grad_dtype, const void *const *values, const void *const *keys,
+                  const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh, const void *h,
+                  int h_dtype, const float *lse, void *const *dvalues, void *const *dkeys, float *dq,
+                  int accumulate, void *workspace, size_t workspace_bytes, void *stream) {
+    if (!dh) return fail(LRAR_ERR_INVALID_ARG, "dh is required");
     if (variant == LRAR_FULL && (!h || !lse))
         return fail(LRAR_ERR_INVALID_ARG, "full AttnRes backward needs the forward's h and lse");
     if (!query && n_src > 1) return fail(LRAR_ERR_INVALID_ARG, "query is required when n_src > 1");
-    if (!aligned16(values) || !aligned16(dh) || !aligned16(dvalues) || !aligned4(dq) ||
-        (variant == LRAR_PROJECTED && (!aligned16(keys) || !aligned16(dkeys))) ||
-        (variant == LRAR_FULL && (!aligned16(h) || !aligned4(lse))) || (query && !aligned4(query)))
+    if (!aligned16(dh) || !aligned4(dq) || (variant == LRAR_FULL && (!aligned16(h) || !aligned4(lse))) ||
+        (query && !aligned4(query)))
         return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (query, lse and dq 4-byte)");
     if (!workspace || workspace_bytes < lrar_backward_workspace_size(variant, n_src, T, d, r))
         return fail(LRAR_ERR_WORKSPACE, "workspace needs %zu bytes (got %zu)",
@@ -215,9 +224,93 @@ LRAR_API int lrar_backward(int variant, int in_dtype, int grad_dtype, const void
     a.dq = dq;
     a.accumulate = accumulate;
     a.partials = static_cast<float *>(workspace);
-    cudaError_t e = lrar::launch_backward(a, s);
+    cudaError_t e = lrar::launch_backward(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "lrar_backward");
     return LRAR_OK;
+}
+
+}  // namespace
+
+LRAR_API int lrar_forward(int variant, int in_dtype, int out_dtype, const void *values, const void *keys,
+                          const float *query, int n_src, int64_t T, int d, int r, float eps, void *h, float *lse,
+                          void *stream) {
+    int rc = check_shape(variant, in_dtype, n_src, T, d, r, eps);
+    if (rc) return rc;
+    if (!dtype_ok(out_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown output dtype %d", out_dtype);
+    if (T == 0) return LRAR_OK;
+    if (!values || !h) return fail(LRAR_ERR_INVALID_ARG, "values and h are required");
+    if (variant == LRAR_PROJECTED && !keys) return fail(LRAR_ERR_INVALID_ARG, "projected keys are required");
+    if (!aligned16(values) || (variant == LRAR_PROJECTED && !aligned16(keys)))
+        return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (query and lse 4-byte)");
+    const void *vt[LRAR_MAX_SOURCES], *kt[LRAR_MAX_SOURCES];
+    stack_table(values, n_src, T, d, esize(in_dtype), vt);
+    stack_table(variant == LRAR_PROJECTED ? keys : nullptr, n_src, T, r, esize(in_dtype), kt);
+    return forward_impl(variant, in_dtype, out_dtype, vt, kt, query, n_src, T, d, r, eps, h, lse, stream);
+}
+
+LRAR_API int lrar_forward_ptrs(int variant, int in_dtype, int out_dtype, const void *const *values,
+                               const void *const *keys, const float *query, int n_src, int64_t T, int d, int r,
+                               float eps, void *h, float *lse, void *stream) {
+    int rc = check_shape(variant, in_dtype, n_src, T, d, r, eps);
+    if (rc) return rc;
+    if (!dtype_ok(out_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown output dtype %d", out_dtype);
+    if (T == 0) return LRAR_OK;
+    if ((rc = check_table(values, n_src, "values"))) return rc;
+    if (variant == LRAR_PROJECTED && (rc = check_table(keys, n_src, "keys"))) return rc;
+    return forward_impl(variant, in_dtype, out_dtype, values, keys, query, n_src, T, d, r, eps, h, lse, stream);
+}
+
+LRAR_API size_t lrar_backward_workspace_size(int variant, int n_src, int64_t T, int d, int r) {
+    (void)n_src;
+    (void)T;
+    const int rq = variant == LRAR_FULL ? d : r;
+    if (rq < 1) return 0;
+    return sizeof(float) * (size_t)lrar::kMaxPartials * (size_t)rq;
+}
+
+LRAR_API int lrar_backward(int variant, int in_dtype, int grad_dtype, const void *values, const void *keys,
+                           const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh,
+                           const void *h, int h_dtype, const float *lse, void *dvalues, void *dkeys, float *dq,
+                           int accumulate, void *workspace, size_t workspace_bytes, void *stream) {
+    bool done;
+    int rc = backward_common(variant, in_dtype, grad_dtype, n_src, T, d, r, eps, h_dtype, dq, accumulate, stream,
+                             &done);
+    if (rc || done) return rc;
+    if (!values || !dvalues) return fail(LRAR_ERR_INVALID_ARG, "values, dh and dvalues are required");
+    if (variant == LRAR_PROJECTED && (!keys || !dkeys))
+        return fail(LRAR_ERR_INVALID_ARG, "projected keys and dkeys are required");
+    if (!aligned16(values) || !aligned16(dvalues) ||
+        (variant == LRAR_PROJECTED && (!aligned16(keys) || !aligned16(dkeys))))
+        return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (query, lse and dq 4-byte)");
+    const int esz = esize(in_dtype), gsz = esize(grad_dtype);
+    const void *vt[LRAR_MAX_SOURCES], *kt[LRAR_MAX_SOURCES], *dvt[LRAR_MAX_SOURCES], *dkt[LRAR_MAX_SOURCES];
+    const bool pl = variant == LRAR_PROJECTED;
+    stack_table(values, n_src, T, d, esz, vt);
+    stack_table(pl ? keys : nullptr, n_src, T, r, esz, kt);
+    stack_table(dvalues, n_src, T, d, gsz, dvt);
+    stack_table(pl ? dkeys : nullptr, n_src, T, r, gsz, dkt);
+    return backward_impl(variant, in_dtype, grad_dtype, vt, kt, query, n_src, T, d, r, eps, dh, h, h_dtype, lse,
+                         const_cast<void *const *>(dvt), const_cast<void *const *>(dkt), dq, accumulate, workspace,
+                         workspace_bytes, stream);
+}
+
+LRAR_API int lrar_backward_ptrs(int variant, int in_dtype, int grad_dtype, const void *const *values,
+                                const void *const *keys, const float *query, int n_src, int64_t T, int d, int r,
+                                float eps, const void *dh, const void *h, int h_dtype, const float *lse,
+                                void *const *dvalues, void *const *dkeys, float *dq, int accumulate, void *workspace,
+                                size_t workspace_bytes, void *stream) {
+    bool done;
+    int rc = backward_common(variant, in_dtype, grad_dtype, n_src, T, d, r, eps, h_dtype, dq, accumulate, stream,
+                             &done);
+    if (rc || done) return rc;
+    if ((rc = check_table(values, n_src, "values"))) return rc;
+    if ((rc = check_table(const_cast<const void *const *>(dvalues), n_src, "dvalues"))) return rc;
+    if (variant == LRAR_PROJECTED) {
+        if ((rc = check_table(keys, n_src, "keys"))) return rc;
+        if ((rc = check_table(const_cast<const void *const *>(dkeys), n_src, "dkeys"))) return rc;
+    }
+    return backward_impl(variant, in_dtype, grad_dtype, values, keys, query, n_src, T, d, r, eps, dh, h, h_dtype, lse,
+                         dvalues, dkeys, dq, accumulate, workspace, workspace_bytes, stream);
 }
 
 LRAR_API size_t lrar_diagnostics_workspace_size(int n_src) {
@@ -248,12 +341,15 @@ LRAR_API int lrar_diagnostics(int variant, int in_dtype, const void *values, con
                     lrar_diagnostics_workspace_size(n_src));
     if (mean_alpha && !aligned16(workspace)) return fail(LRAR_ERR_ALIGNMENT, "workspace must be 16-byte aligned");
     if (!neff && !mean_alpha) return LRAR_OK;
+    const void *vt[LRAR_MAX_SOURCES], *kt[LRAR_MAX_SOURCES];
+    stack_table(values, n_src, T, d, esize(in_dtype), vt);
+    stack_table(variant == LRAR_PROJECTED ? keys : nullptr, n_src, T, r, esize(in_dtype), kt);
     lrar::FwdArgs a;
     a.variant = variant;
     a.in_dtype = in_dtype;
     a.out_dtype = in_dtype;
-    a.values = values;
-    a.keys = variant == LRAR_PROJECTED ? keys : nullptr;
+    a.values = vt;
+    a.keys = variant == LRAR_PROJECTED ? kt : nullptr;
     a.query = query;
     a.n = n_src;
     a.T = T;

@@ -32,9 +32,9 @@
 namespace lrar {
 
 struct BwdParams {
-    const void *values, *keys, *dh, *h;
+    SrcTab vt, kt, dvt, dkt;  // values, P-LR keys and their gradients, one matrix per source
+    const void *dh, *h;
     const float *query, *lse;
-    void *dvalues, *dkeys;
     float *partials;
     int64_t T;
     int n, d, r;
@@ -71,9 +71,8 @@ __device__ __forceinline__ void key_stats_b(const Tin *__restrict__ kp, int r, c
 }
 
 template <typename Tin>
-__device__ __forceinline__ void lr_route_b(const BwdParams &p, const Tin *__restrict__ values,
-                                           const Tin *__restrict__ keys, int64_t x, int lane,
-                                           const float *__restrict__ q_s, float *a_s, float *s_s, float *rho_s) {
+__device__ __forceinline__ void lr_route_b(const BwdParams &p, int64_t x, int lane, const float *__restrict__ q_s,
+                                           float *a_s, float *s_s, float *rho_s) {
     float s_reg[kSrcRegs];
     float m = -INFINITY;
 #pragma unroll
@@ -81,8 +80,7 @@ __device__ __forceinline__ void lr_route_b(const BwdParams &p, const Tin *__rest
         const int i = lane + 32 * k;
         float s = -INFINITY;
         if (i < p.n) {
-            const Tin *kp = p.sliced ? values + ((int64_t)i * p.T + x) * p.d + (p.d - p.r)
-                                     : keys + ((int64_t)i * p.T + x) * p.r;
+            const Tin *kp = p.sliced ? src_row<Tin>(p.vt, i, x, p.d) + (p.d - p.r) : src_row<Tin>(p.kt, i, x, p.r);
             float ss, qk;
             key_stats_b<Tin>(kp, p.r, q_s, p.key_vec != 0, ss, qk);
             const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
@@ -154,7 +152,7 @@ __device__ __forceinline__ float lr_bwd_row(const Frag<Tin, VecE<Tin>::value> *f
 }
 
 template <typename Tin, typename Tg, int V, int U, bool ACC>
-__global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(const BwdParams p) {
+__global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(const __grid_constant__ BwdParams p) {
     constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
     const int rp = round_up(p.r, 4);
@@ -171,19 +169,14 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
     for (int j = threadIdx.x; j < kWarps * rp; j += kThreads) dq_all[j] = 0.f;
     __syncthreads();
 
-    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
-    const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
     const Tin *__restrict__ dh = static_cast<const Tin *>(p.dh);
-    Tg *__restrict__ dvalues = static_cast<Tg *>(p.dvalues);
-    Tg *__restrict__ dkeys = static_cast<Tg *>(p.dkeys);
-    const int64_t src_stride = p.T * (int64_t)p.d;
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     const int tail0 = p.sliced ? p.d - p.r : p.d;  // first key coordinate inside the value row
     const int skip0 = round_up(tail0, E);          // vectors starting here lie wholly in the key slice
 
     for (int64_t x = (int64_t)blockIdx.x * kWarps + warp; x < p.T; x += nwarps) {
         // (1) routing: s_i, rho_i, alpha_i
-        lr_route_b<Tin>(p, values, keys, x, lane, q_s, a_s, s_s, rho_s);
+        lr_route_b<Tin>(p, x, lane, q_s, a_s, s_s, rho_s);
         __syncwarp();
 
         // (2) value pass; dh stays packed in registers and widens per use
@@ -205,17 +198,15 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
 #pragma unroll
                 for (int v = 0; v < V; ++v) {
                     const int e = (lane + 32 * v) * E;
-                    const int64_t off = (int64_t)(i + u) * src_stride + row_off + e;
-                    if (e < p.d) f[u][v].load_nc(values + off);
+                    if (e < p.d) f[u][v].load_nc(src_row<Tin>(p.vt, i + u, x, p.d) + e);
                     else f[u][v].zero();
-                    if (ACC && e < skip0) old[u][v].load(dvalues + off);
+                    if (ACC && e < skip0) old[u][v].load(dst_row<Tg>(p.dvt, i + u, x, p.d) + e);
                     else old[u][v].zero();
                 }
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 const float gp = lr_bwd_row<Tin, Tg, V, ACC>(f[u], old[u], dhr, a_s[i + u],
-                                                             dvalues + (int64_t)(i + u) * src_stride + row_off, tail0,
-                                                             wend, lane);
+                                                             dst_row<Tg>(p.dvt, i + u, x, p.d), tail0, wend, lane);
                 const float g = warp_sum(gp);
                 if (lane == 0) g_s[i + u] = g;
             }
@@ -226,15 +217,13 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
 #pragma unroll
             for (int v = 0; v < V; ++v) {
                 const int e = (lane + 32 * v) * E;
-                const int64_t off = (int64_t)i * src_stride + row_off + e;
-                if (e < p.d) f[v].load_nc(values + off);
+                if (e < p.d) f[v].load_nc(src_row<Tin>(p.vt, i, x, p.d) + e);
                 else f[v].zero();
-                if (ACC && e < skip0) old[v].load(dvalues + off);
+                if (ACC && e < skip0) old[v].load(dst_row<Tg>(p.dvt, i, x, p.d) + e);
                 else old[v].zero();
             }
-            const float gp = lr_bwd_row<Tin, Tg, V, ACC>(f, old, dhr, a_s[i],
-                                                         dvalues + (int64_t)i * src_stride + row_off, tail0, wend,
-                                                         lane);
+            const float gp = lr_bwd_row<Tin, Tg, V, ACC>(f, old, dhr, a_s[i], dst_row<Tg>(p.dvt, i, x, p.d), tail0,
+                                                         wend, lane);
             const float g = warp_sum(gp);
             if (lane == 0) g_s[i] = g;
         }
@@ -256,18 +245,18 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(cons
             for (int k = 0; k < p.n; ++k) {
                 const float rho = rho_s[k], s = s_s[k], ds = g_s[k];
                 float kij;
-                if (p.sliced) kij = to_f(__ldg(values + (int64_t)k * src_stride + row_off + c));
-                else kij = to_f(__ldg(keys + ((int64_t)k * p.T + x) * p.r + j));
+                if (p.sliced) kij = to_f(__ldg(src_row<Tin>(p.vt, k, x, p.d) + c));
+                else kij = to_f(__ldg(src_row<Tin>(p.kt, k, x, p.r) + j));
                 const float kbar = rho * kij;
                 const float dk = ds * rho * (qj - s * p.inv_r * kbar);
                 dqj = fmaf(ds, kbar, dqj);
                 if (p.sliced) {
                     // c < skip0: the value pass stored the old value (or 0) here
-                    Tg *dp = dvalues + (int64_t)k * src_stride + row_off + c;
+                    Tg *dp = dst_row<Tg>(p.dvt, k, x, p.d) + c;
                     const float base = (c < skip0 || p.accumulate) ? to_f(*dp) : 0.f;
                     *dp = from_f<Tg>(base + fmaf(a_s[k], dh_c, dk));
                 } else {
-                    Tg *dp = dkeys + ((int64_t)k * p.T + x) * p.r + j;
+                    Tg *dp = dst_row<Tg>(p.dkt, k, x, p.r) + j;
                     *dp = from_f<Tg>(p.accumulate ? to_f(*dp) + dk : dk);
                 }
             }
@@ -316,9 +305,7 @@ template <int V, bool ACC> struct BwdStages {
 // a fixed butterfly.  S-LR slices are vector-aligned here, so no element of
 // the slice was touched by the value pass.
 template <typename T, bool ACC>
-__device__ __forceinline__ void key_pass_vec(const BwdParams &p, const T *__restrict__ values,
-                                             const T *__restrict__ keys, const T *__restrict__ dh,
-                                             T *__restrict__ dvalues, T *__restrict__ dkeys, int64_t x, int lane,
+__device__ __forceinline__ void key_pass_vec(const BwdParams &p, const T *__restrict__ dh, int64_t x, int lane,
                                              int tail0, const float *__restrict__ q_s, const float *a_s,
                                              const float *s_s, const float *rho_s, const float *ds_s, float *dq_s) {
     constexpr int E = VecE<T>::value;
@@ -326,7 +313,6 @@ __device__ __forceinline__ void key_pass_vec(const BwdParams &p, const T *__rest
     const int NV = p.r / E;
     const int jv = lane % NV, kst = 32 / NV;
     const int j0 = jv * E;
-    const int64_t src_stride = p.T * (int64_t)p.d;
     const int64_t row_off = x * p.d;
     float dqv[E];
 #pragma unroll
@@ -338,14 +324,12 @@ __device__ __forceinline__ void key_pass_vec(const BwdParams &p, const T *__rest
             const int k = kb + m * kst;
             if (k < p.n) {
                 if (p.sliced) {
-                    const int64_t off = (int64_t)k * src_stride + row_off + tail0 + j0;
-                    kf[m].load_nc(values + off);
-                    if (ACC) of[m].load(dvalues + off);
+                    kf[m].load_nc(src_row<T>(p.vt, k, x, p.d) + tail0 + j0);
+                    if (ACC) of[m].load(dst_row<T>(p.dvt, k, x, p.d) + tail0 + j0);
                     else of[m].zero();
                 } else {
-                    const int64_t off = ((int64_t)k * p.T + x) * p.r + j0;
-                    kf[m].load_nc(keys + off);
-                    if (ACC) of[m].load(dkeys + off);
+                    kf[m].load_nc(src_row<T>(p.kt, k, x, p.r) + j0);
+                    if (ACC) of[m].load(dst_row<T>(p.dkt, k, x, p.r) + j0);
                     else of[m].zero();
                 }
             }
@@ -373,8 +357,8 @@ __device__ __forceinline__ void key_pass_vec(const BwdParams &p, const T *__rest
                 }
                 Frag<T, E> out;
                 out.set(w);
-                if (p.sliced) out.store(dvalues + (int64_t)k * src_stride + row_off + tail0 + j0);
-                else out.store(dkeys + ((int64_t)k * p.T + x) * p.r + j0);
+                if (p.sliced) out.store(dst_row<T>(p.dvt, k, x, p.d) + tail0 + j0);
+                else out.store(dst_row<T>(p.dkt, k, x, p.r) + j0);
             }
         }
     }
@@ -393,12 +377,9 @@ __device__ __forceinline__ void key_pass_vec(const BwdParams &p, const T *__rest
 // gradient) loads in flight; lanes that share a coordinate combine their dq
 // parts with a fixed butterfly.  Other widths take one coordinate per lane.
 template <typename T, bool ACC>
-__device__ __forceinline__ void key_pass(const BwdParams &p, const T *__restrict__ values,
-                                         const T *__restrict__ keys, const T *__restrict__ dh,
-                                         T *__restrict__ dvalues, T *__restrict__ dkeys, int64_t x, int lane,
-                                         int tail0, int skip0, const float *__restrict__ q_s, const float *a_s,
+__device__ __forceinline__ void key_pass(const BwdParams &p, const T *__restrict__ dh, int64_t x, int lane, int tail0,
+                                         int skip0, const float *__restrict__ q_s, const float *a_s,
                                          const float *s_s, const float *rho_s, const float *ds_s, float *dq_s) {
-    const int64_t src_stride = p.T * (int64_t)p.d;
     const int64_t row_off = x * p.d;
     const bool shared_j = (32 % p.r) == 0;  // 32/r lanes per coordinate
     const bool multi_j = (p.r % 32) == 0;   // r/32 coordinates per lane
@@ -420,11 +401,11 @@ __device__ __forceinline__ void key_pass(const BwdParams &p, const T *__restrict
                     kv[m] = ov[m] = 0.f;
                     if (k < p.n) {
                         if (p.sliced) {
-                            kv[m] = to_f(__ldg(values + (int64_t)k * src_stride + row_off + c));
-                            if (rd_old) ov[m] = to_f(dvalues[(int64_t)k * src_stride + row_off + c]);
+                            kv[m] = to_f(__ldg(src_row<T>(p.vt, k, x, p.d) + c));
+                            if (rd_old) ov[m] = to_f(dst_row<T>(p.dvt, k, x, p.d)[c]);
                         } else {
-                            kv[m] = to_f(__ldg(keys + ((int64_t)k * p.T + x) * p.r + j));
-                            if (rd_old) ov[m] = to_f(dkeys[((int64_t)k * p.T + x) * p.r + j]);
+                            kv[m] = to_f(__ldg(src_row<T>(p.kt, k, x, p.r) + j));
+                            if (rd_old) ov[m] = to_f(dst_row<T>(p.dkt, k, x, p.r)[j]);
                         }
                     }
                 }
@@ -437,9 +418,9 @@ __device__ __forceinline__ void key_pass(const BwdParams &p, const T *__restrict
                         const float dk = ds * rho * (qj - s * p.inv_r * kbar);
                         dqj = fmaf(ds, kbar, dqj);
                         if (p.sliced)
-                            dvalues[(int64_t)k * src_stride + row_off + c] = from_f<T>(ov[m] + fmaf(a_s[k], dh_c, dk));
+                            dst_row<T>(p.dvt, k, x, p.d)[c] = from_f<T>(ov[m] + fmaf(a_s[k], dh_c, dk));
                         else
-                            dkeys[((int64_t)k * p.T + x) * p.r + j] = from_f<T>(ov[m] + dk);
+                            dst_row<T>(p.dkt, k, x, p.r)[j] = from_f<T>(ov[m] + dk);
                     }
                 }
             }
@@ -460,17 +441,17 @@ __device__ __forceinline__ void key_pass(const BwdParams &p, const T *__restrict
             for (int k = 0; k < p.n; ++k) {
                 const float rho = rho_s[k], s = s_s[k], ds = ds_s[k];
                 float kij;
-                if (p.sliced) kij = to_f(__ldg(values + (int64_t)k * src_stride + row_off + c));
-                else kij = to_f(__ldg(keys + ((int64_t)k * p.T + x) * p.r + j));
+                if (p.sliced) kij = to_f(__ldg(src_row<T>(p.vt, k, x, p.d) + c));
+                else kij = to_f(__ldg(src_row<T>(p.kt, k, x, p.r) + j));
                 const float kbar = rho * kij;
                 const float dk = ds * rho * (qj - s * p.inv_r * kbar);
                 dqj = fmaf(ds, kbar, dqj);
                 if (p.sliced) {
-                    T *dp = dvalues + (int64_t)k * src_stride + row_off + c;
+                    T *dp = dst_row<T>(p.dvt, k, x, p.d) + c;
                     const float base = (c < skip0 || ACC) ? to_f(*dp) : 0.f;
                     *dp = from_f<T>(base + fmaf(a_s[k], dh_c, dk));
                 } else {
-                    T *dp = dkeys + ((int64_t)k * p.T + x) * p.r + j;
+                    T *dp = dst_row<T>(p.dkt, k, x, p.r) + j;
                     *dp = from_f<T>(ACC ? to_f(*dp) + dk : dk);
                 }
             }
@@ -480,7 +461,7 @@ __device__ __forceinline__ void key_pass(const BwdParams &p, const T *__restrict
 }
 
 template <typename T, int V, int S, bool ACC, bool VK>
-__global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(const BwdParams p) {
+__global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(const __grid_constant__ BwdParams p) {
     constexpr int E = VecE<T>::value;
     constexpr int P = ACC ? 2 : 1;  // planes per stage: o, old gradient
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -500,12 +481,7 @@ __global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(c
     for (int j = threadIdx.x; j < kWarps * rp; j += kThreads) dq_all[j] = 0.f;
     __syncthreads();
 
-    const T *__restrict__ values = static_cast<const T *>(p.values);
-    const T *__restrict__ keys = static_cast<const T *>(p.keys);
     const T *__restrict__ dh = static_cast<const T *>(p.dh);
-    T *__restrict__ dvalues = static_cast<T *>(p.dvalues);
-    T *__restrict__ dkeys = static_cast<T *>(p.dkeys);
-    const int64_t src_stride = p.T * (int64_t)p.d;
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     const int tail0 = p.sliced ? p.d - p.r : p.d;
     const int skip0 = round_up(tail0, E);
@@ -519,12 +495,13 @@ __global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(c
     };
     auto issue = [&](int st) {
         if (ix < p.T) {
-            const int64_t off = ((int64_t)ii * p.T + ix) * p.d;
+            const T *row = src_row<T>(p.vt, ii, ix, p.d);
+            const T *old = ACC ? dst_row<T>(p.dvt, ii, ix, p.d) : nullptr;
 #pragma unroll
             for (int v = 0; v < V; ++v) {
                 const int e = (lane + 32 * v) * E;
-                if (e < p.d) cp_async16(cell(st, 0, v), values + off + e);
-                if (ACC && e < wend) cp_async16(cell(st, P - 1, v), dvalues + off + e);
+                if (e < p.d) cp_async16(cell(st, 0, v), row + e);
+                if (ACC && e < wend) cp_async16(cell(st, P - 1, v), old + e);
             }
             if (++ii == p.n) {
                 ii = 0;
@@ -548,10 +525,9 @@ __global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(c
     int st_c = 0, st_i = S - 1;
 
     for (int64_t x = x0; x < p.T; x += nwarps) {
-        lr_route_b<T>(p, values, keys, x, lane, q_s, a_s, s_s, rho_s);
+        lr_route_b<T>(p, x, lane, q_s, a_s, s_s, rho_s);
         __syncwarp();
 
-        const int64_t row_off = x * p.d;
         for (int i = 0; i < p.n; ++i) {
             issue(st_i);
             cp_async_wait<S - 1>();  // this lane's copies of row i have landed
@@ -565,7 +541,7 @@ __global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(c
                 if (ACC && e < wend) old[v].a = ld_shared16(cell(st_c, P - 1, v));
                 else old[v].zero();
             }
-            const float gp = lr_bwd_row<T, T, V, ACC>(f, old, dhr, a_s[i], dvalues + (int64_t)i * src_stride + row_off,
+            const float gp = lr_bwd_row<T, T, V, ACC>(f, old, dhr, a_s[i], dst_row<T>(p.dvt, i, x, p.d),
                                                       tail0, wend, lane);
             const float g = warp_sum(gp);
             if (lane == 0) g_s[i] = g;
@@ -583,11 +559,9 @@ __global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(c
         for (int k = lane; k < p.n; k += 32) g_s[k] = a_s[k] * (g_s[k] - gbar);
         __syncwarp();
         if (VK)  // chosen on the host (vector_key_pass): only one pass is compiled in
-            key_pass_vec<T, ACC>(p, values, keys, dh, dvalues, dkeys, x, lane, tail0, q_s, a_s, s_s, rho_s, g_s,
-                                 dq_s);
+            key_pass_vec<T, ACC>(p, dh, x, lane, tail0, q_s, a_s, s_s, rho_s, g_s, dq_s);
         else
-            key_pass<T, ACC>(p, values, keys, dh, dvalues, dkeys, x, lane, tail0, skip0, q_s, a_s, s_s, rho_s, g_s,
-                             dq_s);
+            key_pass<T, ACC>(p, dh, x, lane, tail0, skip0, q_s, a_s, s_s, rho_s, g_s, dq_s);
         __syncwarp();
     }
     cp_async_wait_all();
@@ -730,7 +704,7 @@ __host__ __device__ inline size_t full_ring_bytes(int cells, int d) {
 // per SM: dq, dh and a row stay in registers, and the deep ring keeps enough
 // bytes in flight for eight warps.
 template <typename T, int V, int S, bool ACC>
-__global__ void __launch_bounds__(kThreads, 1) bwd_full_pipe_kernel(const BwdParams p) {
+__global__ void __launch_bounds__(kThreads, 1) bwd_full_pipe_kernel(const __grid_constant__ BwdParams p) {
     constexpr int E = VecE<T>::value;
     constexpr int P = ACC ? 2 : 1;
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -746,10 +720,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_full_pipe_kernel(const BwdPar
     __syncthreads();
     const uint32_t ring_w = smem_u32(smem_raw) + (uint32_t)(warp * S * P * V * 32 * 16) + 16u * lane;
 
-    const T *__restrict__ values = static_cast<const T *>(p.values);
     const T *__restrict__ dh = static_cast<const T *>(p.dh);
-    T *__restrict__ dvalues = static_cast<T *>(p.dvalues);
-    const int64_t src_stride = p.T * (int64_t)p.d;
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     const float inv_d = 1.f / (float)p.d;
     const int64_t x0 = (int64_t)blockIdx.x * kWarps + warp;
@@ -761,13 +732,14 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_full_pipe_kernel(const BwdPar
     };
     auto issue = [&](int st) {
         if (ix < p.T) {
-            const int64_t off = ((int64_t)ii * p.T + ix) * p.d;
+            const T *row = src_row<T>(p.vt, ii, ix, p.d);
+            const T *old = ACC ? dst_row<T>(p.dvt, ii, ix, p.d) : nullptr;
 #pragma unroll
             for (int v = 0; v < V; ++v) {
                 const int e = (lane + 32 * v) * E;
                 if (e < p.d) {
-                    cp_async16(cell(st, 0, v), values + off + e);
-                    if (ACC) cp_async16(cell(st, P - 1, v), dvalues + off + e);
+                    cp_async16(cell(st, 0, v), row + e);
+                    if (ACC) cp_async16(cell(st, P - 1, v), old + e);
                 }
             }
             if (++ii == p.n) {
@@ -809,7 +781,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_full_pipe_kernel(const BwdPar
                 else old[v].zero();
             }
             full_bwd_row<T, T, V, DQS>(f, old, dhr, q_s, dqf, gbar, lse, inv_d, p.eps,
-                                       dvalues + (int64_t)i * src_stride + row_off, p.d, lane, ACC);
+                                       dst_row<T>(p.dvt, i, x, p.d), p.d, lane, ACC);
             st_c = (st_c + 1 == S) ? 0 : st_c + 1;
             st_i = (st_i + 1 == S) ? 0 : st_i + 1;
         }
@@ -822,7 +794,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_full_pipe_kernel(const BwdPar
 // Full keys with gradients in another dtype than the inputs: rows loaded into
 // registers, U at a time.
 template <typename Tin, typename Tg, int V, int U>
-__global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(const BwdParams p) {
+__global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(const __grid_constant__ BwdParams p) {
     constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
     float *q_s = smem;                    // [32 V E] (q_slot), zero past d
@@ -831,10 +803,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(co
     for (int j = threadIdx.x; j < 32 * V * E; j += kThreads) q_s[q_slot<E>(j)] = (p.query && j < p.d) ? p.query[j] : 0.f;
     __syncthreads();
 
-    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
     const Tin *__restrict__ dh = static_cast<const Tin *>(p.dh);
-    Tg *__restrict__ dvalues = static_cast<Tg *>(p.dvalues);
-    const int64_t src_stride = p.T * (int64_t)p.d;
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     const float inv_d = 1.f / (float)p.d;
     float dqf[V * E];
@@ -861,16 +830,15 @@ __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(co
 #pragma unroll
                 for (int v = 0; v < V; ++v) {
                     const int e = (lane + 32 * v) * E;
-                    const int64_t off = (int64_t)(i + u) * src_stride + row_off + e;
-                    if (e < p.d) f[u][v].load_nc(values + off);
+                    if (e < p.d) f[u][v].load_nc(src_row<Tin>(p.vt, i + u, x, p.d) + e);
                     else f[u][v].zero();
-                    if (p.accumulate && e < p.d) old[u][v].load(dvalues + off);
+                    if (p.accumulate && e < p.d) old[u][v].load(dst_row<Tg>(p.dvt, i + u, x, p.d) + e);
                     else old[u][v].zero();
                 }
 #pragma unroll
             for (int u = 0; u < U; ++u)
                 full_bwd_row<Tin, Tg, V>(f[u], old[u], dhr, q_s, dqf, gbar, lse, inv_d, p.eps,
-                                         dvalues + (int64_t)(i + u) * src_stride + row_off, p.d, lane, p.accumulate);
+                                         dst_row<Tg>(p.dvt, i + u, x, p.d), p.d, lane, p.accumulate);
         }
         for (; i < p.n; ++i) {
             Frag<Tin, E> f[V];
@@ -878,14 +846,13 @@ __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(co
 #pragma unroll
             for (int v = 0; v < V; ++v) {
                 const int e = (lane + 32 * v) * E;
-                const int64_t off = (int64_t)i * src_stride + row_off + e;
-                if (e < p.d) f[v].load_nc(values + off);
+                if (e < p.d) f[v].load_nc(src_row<Tin>(p.vt, i, x, p.d) + e);
                 else f[v].zero();
-                if (p.accumulate && e < p.d) old[v].load(dvalues + off);
+                if (p.accumulate && e < p.d) old[v].load(dst_row<Tg>(p.dvt, i, x, p.d) + e);
                 else old[v].zero();
             }
             full_bwd_row<Tin, Tg, V>(f, old, dhr, q_s, dqf, gbar, lse, inv_d, p.eps,
-                                     dvalues + (int64_t)i * src_stride + row_off, p.d, lane, p.accumulate);
+                                     dst_row<Tg>(p.dvt, i, x, p.d), p.d, lane, p.accumulate);
         }
     }
     full_dq_partial<Tin, V>(p, dqf, scratch, lane, warp);
@@ -930,14 +897,17 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     // wider gradients than inputs double the old-gradient registers per row
     constexpr int UA = sizeof(Tg) > sizeof(Tin) ? (BwdRows<V, true>::value + 1) / 2 : BwdRows<V, true>::value;
     BwdParams p;
-    p.values = a.values;
-    p.keys = a.keys;
+    for (int i = 0; i < kMaxTab; ++i) {
+        const bool in = i < a.n;
+        p.vt.p[i] = in ? a.values[i] : nullptr;
+        p.kt.p[i] = (in && a.keys) ? a.keys[i] : nullptr;
+        p.dvt.p[i] = in ? a.dvalues[i] : nullptr;
+        p.dkt.p[i] = (in && a.dkeys) ? a.dkeys[i] : nullptr;
+    }
     p.dh = a.dh;
     p.h = a.h;
     p.query = a.query;
     p.lse = a.lse;
-    p.dvalues = a.dvalues;
-    p.dkeys = a.dkeys;
     p.partials = a.partials;
     p.T = a.T;
     p.n = a.n;
@@ -952,7 +922,7 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     if (a.variant == kSliced)
         p.key_vec = ((a.r * esz) % 16 == 0) && (((a.d - a.r) * esz) % 16 == 0);
     else
-        p.key_vec = ((a.r * esz) % 16 == 0) && ((reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
+        p.key_vec = (a.r * esz) % 16 == 0;  // every key matrix is 16-byte aligned (checked by the API)
     // Vector key pass (key_pass_vec) when the keys are whole aligned vectors whose
     // row divides a warp, except for accumulating keys of fewer than four vectors,
     // where the scalar batches measured slightly faster.

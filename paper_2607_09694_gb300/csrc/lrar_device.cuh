@@ -6,11 +6,14 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "lrar_launch.h"
+
 namespace lrar {
 
 constexpr int kWarps = 8;                 // warps per CTA
 constexpr int kThreads = kWarps * 32;
 constexpr int kMaxSources = 128;          // LRAR_MAX_SOURCES
+static_assert(kMaxSources == kMaxTab, "source tables hold every source");
 constexpr int kSrcRegs = kMaxSources / 32;
 constexpr int kMaxPartials = 1024;        // CTAs whose dq partials the workspace holds
 
@@ -175,6 +178,16 @@ template <int E> __device__ __forceinline__ void q_get(const float *__restrict__
         qv[4 * k + 2] = a.z;
         qv[4 * k + 3] = a.w;
     }
+}
+
+// Row x of source i (width elements per row) in a source table.
+template <typename T>
+__device__ __forceinline__ const T *src_row(const SrcTab &t, int i, int64_t x, int width) {
+    return static_cast<const T *>(t.p[i]) + x * width;
+}
+template <typename T>
+__device__ __forceinline__ T *dst_row(const SrcTab &t, int i, int64_t x, int width) {
+    return static_cast<T *>(const_cast<void *>(t.p[i])) + x * width;
 }
 
 }  // namespace lrar

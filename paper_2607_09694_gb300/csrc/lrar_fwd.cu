@@ -20,7 +20,7 @@
 namespace lrar {
 
 struct FwdParams {
-    const void *values, *keys;
+    SrcTab vt, kt;  // value and P-LR key tables
     const float *query;
     void *h;
     float *lse;
@@ -79,8 +79,8 @@ __device__ __forceinline__ void key_stats(const Tin *__restrict__ kp, int r, con
 // With kb_s, the token's keys are read from that shared buffer [n][r] (filled
 // by stage_keys) instead of global memory.
 template <typename Tin>
-__device__ __forceinline__ float lr_route(const Tin *__restrict__ values, const Tin *__restrict__ keys, int64_t T,
-                                          int n, int d, int r, float eps, float inv_r, int sliced, int key_vec,
+__device__ __forceinline__ float lr_route(const SrcTab &vt, const SrcTab &kt, int n, int d, int r, float eps,
+                                          float inv_r, int sliced, int key_vec,
                                           int64_t x, int lane, const float *__restrict__ q_s, float *a_s, float *s_s,
                                           float *rho_s, const Tin *kb_s = nullptr) {
     float s_reg[kSrcRegs];
@@ -94,7 +94,7 @@ __device__ __forceinline__ float lr_route(const Tin *__restrict__ values, const 
             if (kb_s) {
                 key_stats<Tin>(kb_s + i * r, r, q_s, true, ss, qk, i);
             } else {
-                const Tin *kp = sliced ? values + ((int64_t)i * T + x) * d + (d - r) : keys + ((int64_t)i * T + x) * r;
+                const Tin *kp = sliced ? src_row<Tin>(vt, i, x, d) + (d - r) : src_row<Tin>(kt, i, x, r);
                 key_stats<Tin>(kp, r, q_s, key_vec != 0, ss, qk);
             }
             const float rho = rsqrtf(fmaf(ss, inv_r, eps));
@@ -148,16 +148,15 @@ __device__ __forceinline__ void store_row(Tout *__restrict__ hrow, int d, int la
 // consecutive pieces, so each instruction covers whole keys.  The caller waits
 // and syncs the warp before the routing lanes read them.
 template <typename Tin>
-__device__ __forceinline__ void stage_keys(const Tin *__restrict__ values, const Tin *__restrict__ keys, int64_t T,
-                                           int n, int d, int r, int sliced, int64_t x, int lane, uint32_t kbuf) {
+__device__ __forceinline__ void stage_keys(const SrcTab &vt, const SrcTab &kt, int n, int d, int r, int sliced,
+                                           int64_t x, int lane, uint32_t kbuf) {
     constexpr int E = VecE<Tin>::value;
     const int per = r / E;
     const bool pow2 = (per & (per - 1)) == 0;
     const int sh = 31 - __clz(per);
     for (int j = lane; j < n * per; j += 32) {
         const int i = pow2 ? j >> sh : j / per, c = j - i * per;
-        const Tin *src = sliced ? values + ((int64_t)i * T + x) * d + (d - r) + c * E
-                                : keys + ((int64_t)i * T + x) * r + c * E;
+        const Tin *src = (sliced ? src_row<Tin>(vt, i, x, d) + (d - r) : src_row<Tin>(kt, i, x, r)) + c * E;
         cp_async16(kbuf + 16u * (uint32_t)(i * per + key_swz(i, c, per)), src);
     }
     cp_async_commit();
@@ -170,7 +169,7 @@ __device__ __forceinline__ void stage_keys(const Tin *__restrict__ values, const
 constexpr int kPrefetchRows = 8;
 
 template <typename Tin, typename Tout, int V, int U, bool KS>
-__global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(const FwdParams p) {
+__global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(const __grid_constant__ FwdParams p) {
     constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
     float *q_s = smem;                                         // [r]
@@ -182,9 +181,6 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
     for (int j = threadIdx.x; j < p.r; j += kThreads) q_s[j] = p.query ? p.query[j] : 0.f;
     __syncthreads();
 
-    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
-    const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
-    const int64_t src_stride = p.T * (int64_t)p.d;
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     const int64_t items = p.T * p.chunks;
 
@@ -193,7 +189,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
     const uint32_t kbuf = smem_u32(kb_s);
     const int pf_at = p.n > kPrefetchRows ? (p.n - kPrefetchRows) / U * U : 0;
     if (KS && (int64_t)blockIdx.x * kWarps + warp < items)
-        stage_keys<Tin>(values, keys, p.T, p.n, p.d, p.r, p.sliced, ((int64_t)blockIdx.x * kWarps + warp) / p.chunks,
+        stage_keys<Tin>(p.vt, p.kt, p.n, p.d, p.r, p.sliced, ((int64_t)blockIdx.x * kWarps + warp) / p.chunks,
                         lane, kbuf);
     for (int64_t it = (int64_t)blockIdx.x * kWarps + warp; it < items; it += nwarps) {
         const int64_t x = it / p.chunks;
@@ -203,13 +199,13 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
             cp_async_wait_all();
             __syncwarp();  // every lane's pieces are visible to the warp
         }
-        const float lse = lr_route<Tin>(values, keys, p.T, p.n, p.d, p.r, p.eps, p.inv_r, p.sliced, p.key_vec, x,
+        const float lse = lr_route<Tin>(p.vt, p.kt, p.n, p.d, p.r, p.eps, p.inv_r, p.sliced, p.key_vec, x,
                                         lane, q_s, a_s, nullptr, nullptr, KS ? kb_s : nullptr);
         if (lane == 0 && p.lse && e0 == 0) p.lse[x] = lse;
         __syncwarp();  // a_s written; kb_s free for the next token
         bool staged = !KS || it + nwarps >= items;
         auto stage_next = [&]() {
-            stage_keys<Tin>(values, keys, p.T, p.n, p.d, p.r, p.sliced, (it + nwarps) / p.chunks, lane, kbuf);
+            stage_keys<Tin>(p.vt, p.kt, p.n, p.d, p.r, p.sliced, (it + nwarps) / p.chunks, lane, kbuf);
             staged = true;
         };
 
@@ -217,7 +213,6 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
         float acc[V * E];
 #pragma unroll
         for (int t = 0; t < V * E; ++t) acc[t] = 0.f;
-        const Tin *row0 = values + x * p.d + e0;
         int i = 0;
         for (; i + U <= p.n; i += U) {
             if (!staged && i == pf_at) stage_next();
@@ -227,7 +222,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
 #pragma unroll
                 for (int v = 0; v < V; ++v) {
                     const int e = (lane + 32 * v) * E;
-                    if (e < dc) f[u][v].load_nc(row0 + (int64_t)(i + u) * src_stride + e);
+                    if (e < dc) f[u][v].load_nc(src_row<Tin>(p.vt, i + u, x, p.d) + e0 + e);
                     else f[u][v].zero();
                 }
 #pragma unroll
@@ -248,7 +243,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
             for (int v = 0; v < V; ++v) {
                 const int e = (lane + 32 * v) * E;
                 Frag<Tin, E> f;
-                if (e < dc) f.load_nc(row0 + (int64_t)i * src_stride + e);
+                if (e < dc) f.load_nc(src_row<Tin>(p.vt, i, x, p.d) + e0 + e);
                 else f.zero();
                 float o[E];
                 f.get(o);
@@ -304,7 +299,8 @@ __device__ __forceinline__ void full_row_step(const Frag<Tin, VecE<Tin>::value> 
 // The ring runs across tokens: the next token's first rows travel while this
 // one finishes.  Scores and the mix use the online softmax of full_row_step.
 template <typename Tin, typename Tout, int V, int S>
-__global__ void __launch_bounds__(kThreads, (V * VecE<Tin>::value <= 32 ? 2 : 1)) fwd_full_kernel(const FwdParams p) {
+__global__ void __launch_bounds__(kThreads, (V * VecE<Tin>::value <= 32 ? 2 : 1))
+    fwd_full_kernel(const __grid_constant__ FwdParams p) {
     constexpr int E = VecE<Tin>::value;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     float *q_s = reinterpret_cast<float *>(smem_raw + (size_t)kWarps * S * V * 32 * 16);  // [32 V E] (q_slot), zero past d
@@ -312,7 +308,6 @@ __global__ void __launch_bounds__(kThreads, (V * VecE<Tin>::value <= 32 ? 2 : 1)
     for (int j = threadIdx.x; j < 32 * V * E; j += kThreads) q_s[q_slot<E>(j)] = (p.query && j < p.d) ? p.query[j] : 0.f;
     __syncthreads();
     const uint32_t ring_w = smem_u32(smem_raw) + (uint32_t)(warp * S * V * 32 * 16) + 16u * lane;
-    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     const float inv_d = 1.f / (float)p.d;
     const int64_t x0 = (int64_t)blockIdx.x * kWarps + warp;
@@ -322,11 +317,11 @@ __global__ void __launch_bounds__(kThreads, (V * VecE<Tin>::value <= 32 ? 2 : 1)
     auto cell = [&](int st, int v) -> uint32_t { return ring_w + (uint32_t)((st * V + v) * 32 * 16); };
     auto issue = [&](int st) {
         if (ix < p.T) {
-            const int64_t off = ((int64_t)ii * p.T + ix) * p.d;
+            const Tin *row = src_row<Tin>(p.vt, ii, ix, p.d);
 #pragma unroll
             for (int v = 0; v < V; ++v) {
                 const int e = (lane + 32 * v) * E;
-                if (e < p.d) cp_async16(cell(st, v), values + off + e);
+                if (e < p.d) cp_async16(cell(st, v), row + e);
             }
             if (++ii == p.n) {
                 ii = 0;
@@ -365,6 +360,13 @@ __global__ void __launch_bounds__(kThreads, (V * VecE<Tin>::value <= 32 ? 2 : 1)
 }
 
 // ------------------------------------------------------------- launch ----
+static void fill_tables(FwdParams &p, const FwdArgs &a) {
+    for (int i = 0; i < kMaxTab; ++i) {
+        p.vt.p[i] = i < a.n ? a.values[i] : nullptr;
+        p.kt.p[i] = (i < a.n && a.keys) ? a.keys[i] : nullptr;
+    }
+}
+
 #ifndef LRAR_STAGE_KEYS
 #define LRAR_STAGE_KEYS 1
 #endif
@@ -375,8 +377,7 @@ template <typename Tin, typename Tout, int V>
 static cudaError_t launch_fwd_t(const FwdArgs &a, cudaStream_t s, int chunks = 1) {
     constexpr int U = V >= 8 ? 1 : (V == 4 ? 2 : 4);
     FwdParams p;
-    p.values = a.values;
-    p.keys = a.keys;
+    fill_tables(p, a);
     p.query = a.query;
     p.h = a.h;
     p.lse = a.lse;
@@ -392,7 +393,7 @@ static cudaError_t launch_fwd_t(const FwdArgs &a, cudaStream_t s, int chunks = 1
     if (a.variant == kSliced)
         p.key_vec = ((a.r * esz) % 16 == 0) && (((a.d - a.r) * esz) % 16 == 0);
     else
-        p.key_vec = ((a.r * esz) % 16 == 0) && ((reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
+        p.key_vec = (a.r * esz) % 16 == 0;  // every key matrix is 16-byte aligned (checked by the API)
     const int64_t work = (a.T * chunks + kWarps - 1) / kWarps;
     if (a.variant == kFull) {
         constexpr int S = FullStages<V, 1, 24>::value;
@@ -443,7 +444,8 @@ static cudaError_t launch_fwd_w(const FwdArgs &a, cudaStream_t s) {
 // read once for its score).  Each CTA writes one row of mean partials (already
 // divided by T) for a fixed-order sum.
 template <typename Tin, int V>
-__global__ void __launch_bounds__(kThreads) diag_kernel(const FwdParams p, float *neff, float *partials, int full) {
+__global__ void __launch_bounds__(kThreads)
+    diag_kernel(const __grid_constant__ FwdParams p, float *neff, float *partials, int full) {
     constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
     float *q_s = smem;                                    // [r]
@@ -456,17 +458,15 @@ __global__ void __launch_bounds__(kThreads) diag_kernel(const FwdParams p, float
     for (int j = threadIdx.x; j < kWarps * kMaxSources; j += kThreads) m_all[j] = 0.f;
     __syncthreads();
 
-    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
-    const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     const float inv_T = 1.f / (float)p.T;
     for (int64_t x = (int64_t)blockIdx.x * kWarps + warp; x < p.T; x += nwarps) {
         if (!full) {
-            lr_route<Tin>(values, keys, p.T, p.n, p.d, p.r, p.eps, p.inv_r, p.sliced, p.key_vec, x, lane, q_s, a_s,
+            lr_route<Tin>(p.vt, p.kt, p.n, p.d, p.r, p.eps, p.inv_r, p.sliced, p.key_vec, x, lane, q_s, a_s,
                           nullptr, nullptr);
         } else {
             for (int i = 0; i < p.n; ++i) {  // score of source i from its whole row (r = d)
-                const Tin *row = values + ((int64_t)i * p.T + x) * p.d;
+                const Tin *row = src_row<Tin>(p.vt, i, x, p.d);
                 float ss = 0.f, qo = 0.f;
 #pragma unroll
                 for (int v = 0; v < V; ++v) {
@@ -521,8 +521,7 @@ __global__ void __launch_bounds__(kThreads) diag_kernel(const FwdParams p, float
 template <typename Tin, int V>
 static cudaError_t launch_diag_t(const FwdArgs &a, float *neff, float *mean_alpha, float *partials, cudaStream_t s) {
     FwdParams p;
-    p.values = a.values;
-    p.keys = a.keys;
+    fill_tables(p, a);
     p.query = a.query;
     p.h = nullptr;
     p.lse = nullptr;
@@ -538,7 +537,7 @@ static cudaError_t launch_diag_t(const FwdArgs &a, float *neff, float *mean_alph
     if (a.variant == kSliced)
         p.key_vec = ((a.r * esz) % 16 == 0) && (((a.d - a.r) * esz) % 16 == 0);
     else
-        p.key_vec = ((a.r * esz) % 16 == 0) && ((reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
+        p.key_vec = (a.r * esz) % 16 == 0;  // every key matrix is 16-byte aligned (checked by the API)
     const size_t smem = sizeof(float) * (round_up(a.r, 4) + 2 * kWarps * kMaxSources);
     const void *k = (const void *)diag_kernel<Tin, V>;
     if (smem > 48 * 1024) {

@@ -10,10 +10,18 @@ namespace lrar {
 enum { kFull = 0, kSliced = 1, kProjected = 2 };
 enum { kF32 = 0, kBF16 = 1 };
 
+// Source tables: entry i is the base of source i's row-major [T, width]
+// matrix, so row x of source i starts at p[i] + x * width elements.  A stacked
+// [n, T, width] buffer is the table base + i * T * width.
+constexpr int kMaxTab = 128;
+struct SrcTab {
+    const void *p[kMaxTab];
+};
+
 struct FwdArgs {
     int variant, in_dtype, out_dtype;
-    const void *values;
-    const void *keys;
+    const void *const *values;  // host array of n source pointers
+    const void *const *keys;    // host array of n P-LR key pointers (P-LR only)
     const float *query;  // may be null when n == 1
     int n;
     int64_t T;
@@ -25,8 +33,8 @@ struct FwdArgs {
 
 struct BwdArgs {
     int variant, in_dtype, grad_dtype, h_dtype;
-    const void *values;
-    const void *keys;
+    const void *const *values;  // host arrays of n pointers, as in FwdArgs
+    const void *const *keys;
     const float *query;
     int n;
     int64_t T;
@@ -35,8 +43,8 @@ struct BwdArgs {
     const void *dh;
     const void *h;
     const float *lse;
-    void *dvalues;
-    void *dkeys;
+    void *const *dvalues;  // host arrays of n gradient pointers (dkeys: P-LR only)
+    void *const *dkeys;
     float *dq;
     int accumulate;
     float *partials;  // workspace: [kMaxPartials][rq] floats

@@ -26,7 +26,8 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "liblrar.so")
 EXPORTS = ("lrar_forward", "lrar_backward", "lrar_backward_workspace_size", "lrar_block_accumulate",
            "lrar_strerror", "lrar_last_error", "lrar_version", "lrar_backward_noalloc", "lrar_diagnostics",
-           "lrar_diagnostics_workspace_size", "lrar_block_phase1", "lrar_block_phase2", "lrar_project")
+           "lrar_diagnostics_workspace_size", "lrar_block_phase1", "lrar_block_phase2", "lrar_project",
+           "lrar_forward_ptrs", "lrar_backward_ptrs")
 MAX_BLOCK_SITES = 64
 
 _lock = threading.Lock()
@@ -66,6 +67,11 @@ def load(path: str | None = None):
         lib.lrar_diagnostics_workspace_size.restype = sz
         lib.lrar_backward_workspace_size.argtypes = [i, i, i64, i, i]
         lib.lrar_backward_workspace_size.restype = sz
+        lib.lrar_forward_ptrs.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, vp]
+        lib.lrar_forward_ptrs.restype = i
+        lib.lrar_backward_ptrs.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, i, vp, vp, vp, vp, i, vp,
+                                           sz, vp]
+        lib.lrar_backward_ptrs.restype = i
         lib.lrar_project.argtypes = [i, vp, vp, i64, i, i, i, vp, vp, vp, vp]
         lib.lrar_project.restype = i
         lib.lrar_block_accumulate.argtypes = [i, vp, i, vp, i64, f32, f32, vp]
@@ -151,6 +157,43 @@ def backward(variant, values: torch.Tensor, keys: torch.Tensor | None, query: to
                                 _ptr(query), n, T, d, r, eps, _ptr(dh), _ptr(h), dtype_code(h), _ptr(lse),
                                 _ptr(dvalues), _ptr(dkeys), _ptr(dq), int(bool(accumulate)), _ptr(workspace),
                                 ws_bytes, _stream(stream)))
+
+
+def _table(ts):
+    """Host array of device pointers for a list of source tensors (None -> NULL)."""
+    if ts is None:
+        return None
+    return (ctypes.c_void_p * len(ts))(*[t.data_ptr() for t in ts])
+
+
+def forward_ptrs(variant, values, keys, query: torch.Tensor | None, h: torch.Tensor, lse: torch.Tensor | None = None,
+                 r: int | None = None, eps: float = DEFAULT_EPS, stream=None) -> None:
+    """lrar_forward_ptrs: like forward, with the sources given as a list of
+    separate [T, d] tensors (and P-LR keys as a list of [T, r] tensors)."""
+    variant = _variant(variant)
+    n = len(values)
+    T, d = values[0].shape
+    if r is None:
+        r = d if variant == FULL else (keys[0].shape[-1] if variant == PROJECTED else query.numel())
+    _check(load().lrar_forward_ptrs(variant, dtype_code(values[0]), dtype_code(h), _table(values), _table(keys),
+                                    _ptr(query), n, T, d, r, eps, _ptr(h), _ptr(lse), _stream(stream)))
+
+
+def backward_ptrs(variant, values, keys, query: torch.Tensor | None, dh: torch.Tensor, dvalues, dq: torch.Tensor,
+                  workspace: torch.Tensor, dkeys=None, h: torch.Tensor | None = None, lse: torch.Tensor | None = None,
+                  r: int | None = None, accumulate: bool = False, eps: float = DEFAULT_EPS, stream=None) -> None:
+    """lrar_backward_ptrs: like backward, with sources and their gradients as
+    lists of separate tensors (gradient i goes to dvalues[i], dkeys[i])."""
+    variant = _variant(variant)
+    n = len(values)
+    T, d = values[0].shape
+    if r is None:
+        r = d if variant == FULL else (keys[0].shape[-1] if variant == PROJECTED else query.numel())
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check(load().lrar_backward_ptrs(variant, dtype_code(values[0]), dtype_code(dvalues[0]), _table(values),
+                                     _table(keys), _ptr(query), n, T, d, r, eps, _ptr(dh), _ptr(h), dtype_code(h),
+                                     _ptr(lse), _table(dvalues), _table(dkeys), _ptr(dq), int(bool(accumulate)),
+                                     _ptr(workspace), ws_bytes, _stream(stream)))
 
 
 def backward_noalloc(variant, values: torch.Tensor, keys: torch.Tensor | None, query: torch.Tensor | None,

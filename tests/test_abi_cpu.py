@@ -186,3 +186,27 @@ def test_project_rejects(lib):
     assert f(1, FAKE, FAKE, 8, 64, 64, 16, None, FAKE, None, None) == lrar.ERR_INVALID_ARG  # o needed when d > 0
     assert f(1, FAKE + 8, FAKE, 8, 64, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_ALIGNMENT
     assert f(1, FAKE, FAKE, 0, 64, 64, 16, FAKE, FAKE, None, None) == lrar.OK                # T == 0: no-op
+
+
+def test_pointer_tables_rejected_before_launch(lib):
+    import ctypes as C
+
+    T, d, r, n = 8, 64, 4, 3
+    good = (C.c_void_p * n)(FAKE, FAKE + 4096, FAKE + 8192)
+    null_entry = (C.c_void_p * n)(FAKE, None, FAKE)
+    odd_entry = (C.c_void_p * n)(FAKE, FAKE + 8, FAKE)
+    f = lib.lrar_forward_ptrs
+    assert f(1, 1, 1, None, None, FAKE, n, T, d, r, EPS, FAKE, None, None) == lrar.ERR_INVALID_ARG
+    assert f(1, 1, 1, null_entry, None, FAKE, n, T, d, r, EPS, FAKE, None, None) == lrar.ERR_INVALID_ARG
+    assert f(1, 1, 1, odd_entry, None, FAKE, n, T, d, r, EPS, FAKE, None, None) == lrar.ERR_ALIGNMENT
+    assert f(2, 1, 1, good, None, FAKE, n, T, d, r, EPS, FAKE, None, None) == lrar.ERR_INVALID_ARG  # P-LR keys
+    assert f(1, 1, 1, good, None, FAKE, 0, T, d, r, EPS, FAKE, None, None) == lrar.ERR_INVALID_ARG  # n_src
+    assert f(1, 1, 1, None, None, FAKE, n, 0, d, r, EPS, None, None, None) == lrar.OK  # T == 0
+    b = lib.lrar_backward_ptrs
+    ws = lib.lrar_backward_workspace_size(1, n, T, d, r)
+    assert b(1, 1, 1, good, None, FAKE, n, T, d, r, EPS, FAKE, None, 1, None, None, None, FAKE, 0, FAKE, ws,
+             None) == lrar.ERR_INVALID_ARG  # dvalues table
+    assert b(1, 1, 1, good, None, FAKE, n, T, d, r, EPS, FAKE, None, 1, None, odd_entry, None, FAKE, 0, FAKE, ws,
+             None) == lrar.ERR_ALIGNMENT
+    assert b(1, 1, 1, good, None, FAKE, n, T, d, r, EPS, FAKE, None, 1, None, good, None, FAKE, 0, FAKE, 16,
+             None) == lrar.ERR_WORKSPACE
