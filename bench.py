@@ -326,6 +326,10 @@ def run_ours(args):
                 "bwd_gbs": hbb / hb / 1e6, "fwd_bwd_gbs": (hfb + hbb) / (hf + hb) / 1e6,
                 "frac": (hfb + hbb) / (hf + hb) / 1e6 / peak, "tokens_per_s": T_TOK / ((hf + hb) / 1e3)}
 
+    # the same step as separate source tensors through the whole-decoder
+    # driver, captured once into a CUDA graph and replayed (one launch per step)
+    graph = run_graph(wl, step_bytes)
+
     # end to end through the public API with host buffers
     e2e = run_e2e(wl, args, dist, dev, step_bytes, world)
 
@@ -357,6 +361,7 @@ def run_ours(args):
                      "peak_source": f"{peak_kind} hbm_gbs (copy bandwidth)",
                      "fwd_gbs": fwd_gbs, "bwd_gbs": bwd_gbs},
         "e2e": e2e,
+        "graph_step": graph,
         "gpu_launches": Workload.launches_per_step() * args.steps,
         "clocks": clk,
     }
@@ -547,6 +552,23 @@ def run_suite(args):
               "per_site_ms": tn, "two_phase_ms": tt, "speedup": tn / tt, "per_site_bytes": naive_bytes,
               "two_phase_bytes": tp_bytes, "per_site_gbs": naive_bytes / tn / 1e6,
               "two_phase_gbs": tp_bytes / tt / 1e6})
+
+
+def run_graph(wl, step_bytes, reps: int = 10):
+    """Median ms of one whole step replayed from a CUDA graph of the
+    whole-decoder driver (sources as separate tensors: views of the stack)."""
+    import torch
+
+    from paper_2607_09694_gb300.sweep import DepthSweep
+
+    ns = wl.values.shape[0]
+    sw = DepthSweep("sliced", [wl.values[i] for i in range(ns)], wl.queries, [wl.dh[i] for i in range(ns)], wl.h,
+                    wl.lse, [wl.dvalues[i] for i in range(ns)], wl.dq, r=R, eps=EPS)
+    sw.capture()
+    ms = _median_ms(torch, sw.replay, reps)
+    return {"ms_per_step": ms, "gbs": step_bytes / ms / 1e6, "launches_per_replay": 3 * ns + 1,
+            "what": "DepthSweep over per-source tensor views, one CUDA graph replay per step (49 forward, "
+                    "49 backward, 49 dq sums, one dq zeroing)"}
 
 
 def run_e2e(wl, args, dist, dev, step_bytes, world):
