@@ -13,8 +13,11 @@
 //            h = exp(lse_j - lse) h_pre_j + exp(s_P - lse) b_P.
 //
 // The result is the site's mix over [completed sources, b_P] (Eq. 8-10).
-// Phase 1 tiles a token's row over warps: warp (g, ch) of a CTA owns the
-// 32 x 16-byte chunk ch of token g's rows and keeps c accumulators per element.
+// Phase 1 tiles a token's row over the warps of a group: warp (g, ch) of a CTA
+// owns the 32 x 16-byte chunk ch of token g's rows and keeps c accumulators per
+// element.  The chunk warps split the c queries for scoring and share the
+// weights through shared memory (double-buffered, one named barrier per pass),
+// and each pass scores the next token while the current token's rows load.
 #include "lrar_device.cuh"
 #include "lrar_launch.h"
 
@@ -33,77 +36,125 @@ struct Ph1Params {
     int sliced, key_vec;
 };
 
-template <typename Tin, typename Tout>
-__global__ void __launch_bounds__(kThreads) block_phase1_kernel(const Ph1Params p) {
+__device__ __forceinline__ void group_sync(int id, int threads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+
+// Scores of token x for the queries j = ch, ch + chunks, ... (Eq. 8-9): lane i
+// takes source i; then the softmax of each of those queries over the n sources.
+// Weights go to aw[j * n + i], lse_j to the output.
+template <typename Tin>
+__device__ __forceinline__ float ph1_dot(const Tin *__restrict__ kp, const float *__restrict__ qj, int r, bool vec,
+                                         float *ss) {
     constexpr int E = VecE<Tin>::value;
-    constexpr int U = 4;  // rows in flight per lane
+    float qk = 0.f, s2 = 0.f;
+    if (vec) {
+#pragma unroll 4
+        for (int jj = 0; jj < r; jj += E) {
+            Frag<Tin, E> f;
+            f.load_nc(kp + jj);
+            float k[E];
+            f.get(k);
+#pragma unroll
+            for (int t = 0; t < E; ++t) {
+                s2 = fmaf(k[t], k[t], s2);
+                qk = fmaf(qj[jj + t], k[t], qk);
+            }
+        }
+    } else {
+        for (int jj = 0; jj < r; ++jj) {
+            const float k = to_f(__ldg(kp + jj));
+            s2 = fmaf(k, k, s2);
+            qk = fmaf(qj[jj], k, qk);
+        }
+    }
+    if (ss) *ss = s2;
+    return qk;
+}
+
+// Scores of token x for the queries j = ch, ch + chunks, ... (Eq. 8-9): lane i
+// takes source i; then the softmax of each of those queries over the n sources.
+// Weights go to aw[j * n + i], lse_j to the output.
+template <typename Tin>
+__device__ __forceinline__ void ph1_score(const Ph1Params &p, const float *__restrict__ q_s, int rp, int64_t x,
+                                          int ch, int lane, float *aw) {
+    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
+    const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
+    if (ch < p.c)
+        for (int i = lane; i < p.n; i += 32) {
+            const Tin *kp = p.sliced ? values + ((int64_t)i * p.T + x) * p.d + (p.d - p.r)
+                                     : keys + ((int64_t)i * p.T + x) * p.r;
+            float ss;
+            const float qk0 = ph1_dot<Tin>(kp, q_s + ch * rp, p.r, p.key_vec != 0, &ss);
+            const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
+            aw[ch * p.n + i] = rho * qk0;
+            for (int j = ch + p.chunks; j < p.c; j += p.chunks)  // further queries of this warp (small d)
+                aw[j * p.n + i] = rho * ph1_dot<Tin>(kp, q_s + j * rp, p.r, p.key_vec != 0, nullptr);
+        }
+    __syncwarp();
+    for (int j = ch; j < p.c; j += p.chunks) {
+        float m = -INFINITY;
+        for (int i = lane; i < p.n; i += 32) m = fmaxf(m, aw[j * p.n + i]);
+        m = warp_max(m);
+        float z = 0.f;
+        for (int i = lane; i < p.n; i += 32) z += expf(aw[j * p.n + i] - m);
+        z = warp_sum(z);
+        __syncwarp();
+        for (int i = lane; i < p.n; i += 32) aw[j * p.n + i] = expf(aw[j * p.n + i] - m) / z;
+        if (lane == 0) p.lse_pre[(int64_t)j * p.T + x] = m + logf(z);
+        __syncwarp();
+    }
+}
+
+template <typename Tin, typename Tout, int U>
+__global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_constant__ Ph1Params p) {
+    constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
     const int rp = round_up(p.r, 4);
-    float *q_s = smem;                             // [c][r]
-    float *a_s = q_s + kPh1MaxSites * rp;          // [kWarps][c][n]: scores, then weights
-    float *lse_s = a_s + kWarps * kPh1MaxSites * p.n;  // [kWarps][c]
+    float *q_s = smem;                     // [c][r]
+    float *a_all = q_s + kPh1MaxSites * rp;  // [G][2][kPh1MaxSites][n]: weights, double-buffered by pass
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int G = kWarps / p.chunks;  // tokens per CTA pass
     const int g = warp / p.chunks, ch = warp % p.chunks;
+    const int nthr = p.chunks * 32;   // threads of a token group (named barrier 1 + g)
     for (int j = threadIdx.x; j < p.c * p.r; j += kThreads) q_s[(j / p.r) * rp + j % p.r] = p.queries[j];
     __syncthreads();
 
     const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
-    const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
     Tout *__restrict__ h_pre = static_cast<Tout *>(p.h_pre);
     const int e = (ch * 32 + lane) * E;  // this lane's first element of the row
-    float *ag = a_s + g * kPh1MaxSites * p.n;
+    float *aw0 = a_all + (size_t)g * 2 * kPh1MaxSites * p.n;
+    const int64_t stride = (int64_t)gridDim.x * G;
 
-    for (int64_t base = (int64_t)blockIdx.x * G; base < p.T; base += (int64_t)gridDim.x * G) {
-        const int64_t x = base + g;
-        if (ch == 0 && x < p.T) {
-            // Eq. (8)-(9) for all c queries: lane i scores source i
-            for (int i = lane; i < p.n; i += 32) {
-                const Tin *kp = p.sliced ? values + ((int64_t)i * p.T + x) * p.d + (p.d - p.r)
-                                         : keys + ((int64_t)i * p.T + x) * p.r;
-                float ss = 0.f, qk[kPh1MaxSites];
+    int64_t x = (int64_t)blockIdx.x * G + g;
+    if (x < p.T) ph1_score<Tin>(p, q_s, rp, x, ch, lane, aw0);
+    group_sync(1 + g, nthr);
+    for (int pass = 0; (int64_t)blockIdx.x * G + pass * stride < p.T; ++pass, x += stride) {
+        const float *aw = aw0 + (pass & 1) * kPh1MaxSites * p.n;
+        float *aw_next = aw0 + ((pass + 1) & 1) * kPh1MaxSites * p.n;
+        const bool live = x < p.T && e < p.d;
+        const Tin *row0 = values + x * p.d + e;
+        Frag<Tin, E> f[U];
+        // the first rows of this token travel while the next token is scored
 #pragma unroll
-                for (int j = 0; j < kPh1MaxSites; ++j) qk[j] = 0.f;
-                for (int jj = 0; jj < p.r; ++jj) {
-                    const float k = to_f(__ldg(kp + jj));
-                    ss = fmaf(k, k, ss);
-#pragma unroll
-                    for (int j = 0; j < kPh1MaxSites; ++j)
-                        if (j < p.c) qk[j] = fmaf(q_s[j * rp + jj], k, qk[j]);
-                }
-                const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
-#pragma unroll
-                for (int j = 0; j < kPh1MaxSites; ++j)
-                    if (j < p.c) ag[j * p.n + i] = rho * qk[j];
-            }
-            __syncwarp();
-            for (int j = 0; j < p.c; ++j) {
-                float m = -INFINITY;
-                for (int i = lane; i < p.n; i += 32) m = fmaxf(m, ag[j * p.n + i]);
-                m = warp_max(m);
-                float z = 0.f;
-                for (int i = lane; i < p.n; i += 32) z += expf(ag[j * p.n + i] - m);
-                z = warp_sum(z);
-                __syncwarp();
-                for (int i = lane; i < p.n; i += 32) ag[j * p.n + i] = expf(ag[j * p.n + i] - m) / z;
-                if (lane == 0) lse_s[g * kPh1MaxSites + j] = m + logf(z);
-                __syncwarp();
-            }
+        for (int u = 0; u < U; ++u) {
+            if (live && u < p.n) f[u].load_nc(row0 + (int64_t)u * p.T * p.d);
+            else f[u].zero();
         }
-        __syncthreads();
+        if (x + stride < p.T) ph1_score<Tin>(p, q_s, rp, x + stride, ch, lane, aw_next);
         if (x < p.T) {
             float acc[kPh1MaxSites][E];
 #pragma unroll
             for (int j = 0; j < kPh1MaxSites; ++j)
 #pragma unroll
                 for (int t = 0; t < E; ++t) acc[j][t] = 0.f;
-            const Tin *row0 = values + x * p.d + e;
             for (int i0 = 0; i0 < p.n; i0 += U) {
-                Frag<Tin, E> f[U];
+                if (i0 > 0) {
 #pragma unroll
-                for (int u = 0; u < U; ++u) {
-                    if (i0 + u < p.n && e < p.d) f[u].load_nc(row0 + (int64_t)(i0 + u) * p.T * p.d);
-                    else f[u].zero();
+                    for (int u = 0; u < U; ++u) {
+                        if (live && i0 + u < p.n) f[u].load_nc(row0 + (int64_t)(i0 + u) * p.T * p.d);
+                        else f[u].zero();
+                    }
                 }
 #pragma unroll
                 for (int u = 0; u < U; ++u) {
@@ -113,7 +164,7 @@ __global__ void __launch_bounds__(kThreads) block_phase1_kernel(const Ph1Params 
 #pragma unroll
                         for (int j = 0; j < kPh1MaxSites; ++j) {
                             if (j < p.c) {
-                                const float w = ag[j * p.n + i0 + u];
+                                const float w = aw[j * p.n + i0 + u];
 #pragma unroll
                                 for (int t = 0; t < E; ++t) acc[j][t] = fmaf(w, o[t], acc[j][t]);
                             }
@@ -121,7 +172,7 @@ __global__ void __launch_bounds__(kThreads) block_phase1_kernel(const Ph1Params 
                     }
                 }
             }
-            if (e < p.d) {
+            if (live) {
 #pragma unroll
                 for (int j = 0; j < kPh1MaxSites; ++j) {
                     if (j < p.c) {
@@ -131,9 +182,8 @@ __global__ void __launch_bounds__(kThreads) block_phase1_kernel(const Ph1Params 
                     }
                 }
             }
-            if (ch == 0 && lane < p.c) p.lse_pre[(int64_t)lane * p.T + x] = lse_s[g * kPh1MaxSites + lane];
         }
-        __syncthreads();
+        group_sync(1 + g, nthr);  // next weights complete; this pass's weights free for reuse
     }
 }
 
@@ -215,22 +265,25 @@ static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
     p.eps = a.eps;
     p.inv_r = 1.f / (float)a.r;
     p.sliced = a.variant == kSliced;
-    p.key_vec = 0;
+    constexpr int esz = sizeof(Tin);
+    p.key_vec = (a.r * esz) % 16 == 0 &&
+                (a.variant == kSliced ? ((a.d - a.r) * esz) % 16 == 0
+                                      : (reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
+    const int G = kWarps / chunks;
     const size_t smem = sizeof(float) * ((size_t)kPh1MaxSites * round_up(a.r, 4) +
-                                         (size_t)kWarps * kPh1MaxSites * a.n + (size_t)kWarps * kPh1MaxSites);
-    const void *k = (const void *)block_phase1_kernel<Tin, Tout>;
+                                         (size_t)G * 2 * kPh1MaxSites * a.n);
+    const void *k = (const void *)block_phase1_kernel<Tin, Tout, 8>;
     if (smem > 48 * 1024) {
         cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
     }
-    const int G = kWarps / chunks;
     const int grid = persistent_grid(k, kThreads, smem, (a.T + G - 1) / G, 1 << 30);
     for (int j0 = 0; j0 < a.c; j0 += kPh1MaxSites) {  // groups of at most 8 queries
         p.c = a.c - j0 < kPh1MaxSites ? a.c - j0 : kPh1MaxSites;
         p.queries = a.queries + (size_t)j0 * a.r;
         p.h_pre = static_cast<char *>(a.h_pre) + (size_t)j0 * p.site_stride * sizeof(Tout);
         p.lse_pre = a.lse_pre + (size_t)j0 * a.T;
-        block_phase1_kernel<Tin, Tout><<<grid, kThreads, smem, s>>>(p);
+        block_phase1_kernel<Tin, Tout, 8><<<grid, kThreads, smem, s>>>(p);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
