@@ -49,6 +49,15 @@ def _peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def _bf16_peak():
+    """Measured dense bf16 tensor throughput (burst), TFLOP/s; else the fallback."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
+
+
 def _kernel_source_hash() -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2607_09694_gb300", "csrc")
@@ -495,6 +504,34 @@ def run_suite(args):
     fwd_bwd("full AttnRes keys d1024 n49 (bf16 h)", "full", 16384, 1024, 1024, 49, 1, (0.5, 2.0))
     fwd_bwd("S-LR d2048 n65 r64 T32768", "sliced", 32768, 2048, 64, 65, 3)
     fwd_bwd("Block S-LR site d2048 n9 r64 T32768", "sliced", 32768, 2048, 64, 9, 3)
+
+    # P-LR fused output projection (Eq. 11-12) on the tensor cores, against
+    # cuBLAS (torch.matmul) alone and cuBLAS followed by the split of its output
+    # into the value and key slots that the fused epilogue writes directly
+    tpeak, tsrc = _bf16_peak()
+    for T, m, d, r in ((16384, 1024, 1024, 32), (16384, 2816, 1024, 32), (32768, 2048, 2048, 64),
+                       (16384, 1024, 0, 32)):
+        a = synth.randn((T, m), 1, "proj_a", device=dev).to(torch.bfloat16)
+        w = (synth.randn((d + r, m), 1, "proj_w", device=dev) / m ** 0.5).to(torch.bfloat16)
+        o = torch.empty(T, d, dtype=torch.bfloat16, device=dev) if d else None
+        k = torch.empty(T, r, dtype=torch.bfloat16, device=dev)
+        ours = _median_ms(torch, lambda: lrar.project(a, w, o, k), reps)
+        wt = w.t()
+        cub = _median_ms(torch, lambda: torch.matmul(a, wt), reps)
+
+        def cub_split():
+            y = torch.matmul(a, wt)
+            if o is not None:
+                o.copy_(y[:, :d])
+            k.copy_(y[:, d:])
+
+        cubs = _median_ms(torch, cub_split, reps)
+        flops = 2.0 * T * m * (d + r)
+        emit({"suite": f"P-LR fused projection T{T} m{m} d{d} r{r}", "ms": ours, "tflops": flops / ours / 1e9,
+              "tflops_frac": flops / ours / 1e9 / tpeak, "peak_tflops": tpeak, "peak_source": tsrc,
+              "cublas_ms": cub, "cublas_tflops": flops / cub / 1e9, "cublas_then_split_ms": cubs})
+        del a, w, o, k
+        torch.cuda.empty_cache()
 
     # routing diagnostics (Eq. 16): reads only the keys (the S-LR tails, one 32-byte
     # sector per row at r = 16), writes N_eff per token and the mean alpha per source
