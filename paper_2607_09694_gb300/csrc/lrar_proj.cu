@@ -10,7 +10,7 @@
 //
 // Persistent kernel, one CTA per SM walking the 128 x kPN tiles of Y:
 //   warp 4  one lane streams K-blocks of A and W (64 columns each) into a
-//           kPStages-deep shared-memory ring with TMA (128-byte swizzle); the
+//           shared-memory ring (as deep as fits) with TMA (128-byte swizzle); the
 //           ring runs on across tiles;
 //   warp 5  allocates two fp32 accumulators in TMEM, and one lane issues
 //           tcgen05.mma (M = 128, N = kPN, K = 16) per 16 columns of a block,
@@ -23,6 +23,7 @@
 // shared abort flag that ends the other roles' waits, and the kernel drains
 // its copies and MMAs and frees TMEM before it returns.
 #include <cmath>
+#include <cstdlib>
 #include <mutex>
 
 #include "lrar.h"
@@ -37,19 +38,20 @@ using namespace sm100;
 
 constexpr int kPM = 128;                        // tile rows (tokens), one TMEM lane each
 constexpr int kPK = 64;                         // K-block: 64 bf16 = one 128-byte swizzle row
-constexpr int kPStages = 5;                     // ring depth
 constexpr int kPThreads = 192;                  // 6 warps
 constexpr uint32_t kAccCols = 256;              // TMEM columns per accumulator (>= the tile width)
 constexpr uint32_t kTmemCols = 2 * kAccCols;    // two accumulators: the whole TMEM of the SM
 constexpr int kABytes = kPM * kPK * 2;          // 16 KB
 constexpr long long kWaitLimit = 4LL << 30;     // SM cycles (about 2 s) before a wait gives up
 
-// Tile width BN (columns of Y): 176 covers d + r = 1056 in 6 tiles, 160 in 7
-// with a better balanced last wave; the host picks per call.
+// Tile width BN (columns of Y), picked per call by the host (tile_efficiency).
 template <int BN> struct ProjTile {
     static constexpr int kBBytes = BN * kPK * 2;
     static constexpr int kStageBytes = kABytes + kBBytes;  // multiple of 1024: tiles stay 1024-aligned
-    static constexpr size_t kSmem = (size_t)kPStages * kStageBytes + 1024 /* alignment slack */ + 256 /* barriers */;
+    // as many ring stages as fit in a CTA's 227 KB of shared memory: the feed is
+    // bytes in flight, so the ring is as deep as the tile allows (6 at 160, 5 at 176)
+    static constexpr int kStages = (227 * 1024 - 1024 - 256) / kStageBytes;
+    static constexpr size_t kSmem = (size_t)kStages * kStageBytes + 1024 /* alignment slack */ + 256 /* barriers */;
     static_assert(kStageBytes % 1024 == 0, "stage tiles must keep 1024-byte alignment");
     static_assert(BN % 16 == 0 && BN <= (int)kAccCols, "M = 128 MMA needs N a multiple of 16 within an accumulator");
 };
@@ -72,6 +74,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
     proj_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_w,
                 const ProjParams p) {
     constexpr int kStageBytes = ProjTile<kPN>::kStageBytes;
+    constexpr int kPStages = ProjTile<kPN>::kStages;
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;  // 128-byte swizzled tiles need 1024-byte alignment
@@ -282,13 +285,17 @@ int launch_project_t(const CUtensorMap &map_a, const void *w, int64_t T, int m, 
     return LRAR_OK;
 }
 
-// Estimated useful fraction of the SMs' tile time for width BN: tiles over
-// whole waves of one tile per SM, times the share of computed columns kept.
+// Relative rate of useful work with tile width BN: the share of SM time in
+// whole waves of one tile per SM, times the share of computed columns kept,
+// times the multiply-adds per operand byte of a 128 x BN tile (the shared-memory
+// feed per SM bounds the tensor pipe: measured rates follow BN / (128 + BN)).
 double tile_efficiency(int64_t T, int N, int BN, int sms) {
     const int64_t nt = (N + BN - 1) / BN, tiles = (T + kPM - 1) / kPM * nt;
     const double waves = (double)tiles / sms;
-    return waves / std::ceil(waves) * (double)N / (double)(nt * BN);
+    return waves / std::ceil(waves) * (double)N / (double)(nt * BN) * (double)BN / (double)(kPM + BN);
 }
+
+constexpr int kTileWidths[] = {160, 176, 192, 224, 240, 256};
 
 }  // namespace
 
@@ -300,10 +307,25 @@ int launch_project(const void *a, const void *w, int64_t T, int m, int d, int r,
     int dev = 0, sms = 1;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    // 176 wins ties: its tile reads fewer bytes per multiply-add
-    if (tile_efficiency(T, d + r, 160, sms) > 1.02 * tile_efficiency(T, d + r, 176, sms))
-        return launch_project_t<160>(map_a, w, T, m, d, r, o, keys, status, s);
-    return launch_project_t<176>(map_a, w, T, m, d, r, o, keys, status, s);
+    int bn = 0;
+    double best = -1.0;
+    for (int c : kTileWidths) {  // the wider tile wins ties (fewer bytes per multiply-add)
+        const double e = tile_efficiency(T, d + r, c, sms);
+        if (e >= best * 1.001) {
+            best = e;
+            bn = c;
+        }
+    }
+    if (const char *force = getenv("LRAR_PROJ_TILE")) bn = atoi(force);  // tuning override
+    switch (bn) {
+        case 160: return launch_project_t<160>(map_a, w, T, m, d, r, o, keys, status, s);
+        case 176: return launch_project_t<176>(map_a, w, T, m, d, r, o, keys, status, s);
+        case 192: return launch_project_t<192>(map_a, w, T, m, d, r, o, keys, status, s);
+        case 224: return launch_project_t<224>(map_a, w, T, m, d, r, o, keys, status, s);
+        case 240: return launch_project_t<240>(map_a, w, T, m, d, r, o, keys, status, s);
+        case 256: return launch_project_t<256>(map_a, w, T, m, d, r, o, keys, status, s);
+        default: return record_error(LRAR_ERR_INVALID_ARG, "LRAR_PROJ_TILE must be 160, 176, 192, 224, 240 or 256");
+    }
 }
 
 }  // namespace lrar

@@ -67,6 +67,14 @@ def test_ragged_edges():
     _compare(300, 1000, 1024, 16, seed=4)
 
 
+@pytest.mark.parametrize("width", [160, 176, 192, 224, 240, 256])
+def test_every_tile_width(width, monkeypatch):
+    """Each compiled tile width (forced through LRAR_PROJ_TILE) on ragged T, m and
+    N, the value/key split falling inside a tile."""
+    monkeypatch.setenv("LRAR_PROJ_TILE", str(width))
+    _compare(300, 1000, 1024, 16, seed=4)
+
+
 def test_swiglu_output_projection():
     """The FFN's output projection: m = 2816 (the SwiGLU width of the 0.5B decoder)."""
     _compare(256, 2816, 1024, 32, seed=5)
