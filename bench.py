@@ -439,6 +439,29 @@ def run_profile_site(args):
                       "fwd_gbs": fb / f / 1e6, "bwd_gbs": bb / b / 1e6}), flush=True)
 
 
+def run_profile_proj(args):
+    """Small case of the fused projection for profilers: --profile-proj m, with
+    --tokens T, --site-d d, --site-r r (bf16 operands)."""
+    import torch
+
+    from __graft_entry__ import build
+    from paper_2607_09694_gb300 import lrar, synth
+
+    build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    T, m, d, r = args.tokens, args.profile_proj, args.site_d, args.site_r
+    a = synth.randn((T, m), 1, "proj_a", device=dev).to(torch.bfloat16)
+    w = (synth.randn((d + r, m), 1, "proj_w", device=dev) / m ** 0.5).to(torch.bfloat16)
+    o = torch.empty(T, d, dtype=torch.bfloat16, device=dev) if d else None
+    k = torch.empty(T, r, dtype=torch.bfloat16, device=dev)
+    for _ in range(args.warmup):
+        lrar.project(a, w, o, k)
+    ms = _median_ms(torch, lambda: lrar.project(a, w, o, k), args.steps)
+    flops = 2.0 * T * m * (d + r)
+    print(json.dumps({"profile_proj": m, "T": T, "d": d, "r": r, "ms": ms, "tflops": flops / ms / 1e9}), flush=True)
+
+
 def _median_ms(torch, fn, reps):
     """Median CUDA-event time of fn() over reps back-to-back repetitions (after one warm-up)."""
     fn()
@@ -759,6 +782,8 @@ def main():
     ap.add_argument("--site-d", type=int, default=D, help="width d of the --profile-site case")
     ap.add_argument("--site-r", type=int, default=R, help="key rank r of the --profile-site case (not full)")
     ap.add_argument("--suite", action="store_true", help="time every workload's headline site (JSON line each)")
+    ap.add_argument("--profile-proj", type=int, default=0,
+                    help="time the fused projection with this input width m (profiling; --tokens, --site-d, --site-r)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -766,6 +791,8 @@ def main():
         run_suite(args)
     elif args.profile_site:
         run_profile_site(args)
+    elif args.profile_proj:
+        run_profile_proj(args)
     elif args.impl == "reference":
         run_reference(args)
     else:
