@@ -24,6 +24,7 @@
 namespace lrar {
 
 constexpr int kPh1MaxSites = 8;  // queries per phase-1 launch (more are split by the host)
+constexpr int kPh1Stages = 12;   // ring depth of phase 1 (rows in flight per lane + 1)
 
 struct Ph1Params {
     const void *values, *keys;
@@ -106,12 +107,15 @@ __device__ __forceinline__ void ph1_score(const Ph1Params &p, const float *__res
     }
 }
 
-template <typename Tin, typename Tout, int U>
+// Rows stream through a per-lane cp.async ring (each lane copies and reads
+// back its own 16-byte vector of every row), S - 1 rows ahead and across
+// tokens, so the loads of the next token's rows overlap this token's mix.
+template <typename Tin, typename Tout, int S>
 __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_constant__ Ph1Params p) {
     constexpr int E = VecE<Tin>::value;
-    extern __shared__ float smem[];
+    extern __shared__ __align__(16) unsigned char smem_raw[];
     const int rp = round_up(p.r, 4);
-    float *q_s = smem;                     // [c][r]
+    float *q_s = reinterpret_cast<float *>(smem_raw + (size_t)kWarps * S * 32 * 16);  // [c][r] after the rings
     float *a_all = q_s + kPh1MaxSites * rp;  // [G][2][kPh1MaxSites][n]: weights, double-buffered by pass
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int G = kWarps / p.chunks;  // tokens per CTA pass
@@ -125,22 +129,30 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
     const int e = (ch * 32 + lane) * E;  // this lane's first element of the row
     float *aw0 = a_all + (size_t)g * 2 * kPh1MaxSites * p.n;
     const int64_t stride = (int64_t)gridDim.x * G;
+    const uint32_t ring_w = smem_u32(smem_raw) + (uint32_t)(warp * S * 32 * 16) + 16u * lane;
 
     int64_t x = (int64_t)blockIdx.x * G + g;
+    int64_t ix = x;  // next row to copy: source ii of token ix
+    int ii = 0;
+    auto issue = [&](int st) {
+        if (ix < p.T) {
+            if (e < p.d) cp_async16(ring_w + 16u * 32u * st, values + ((int64_t)ii * p.T + ix) * p.d + e);
+            if (++ii == p.n) {
+                ii = 0;
+                ix += stride;
+            }
+        }
+        cp_async_commit();
+    };
+#pragma unroll
+    for (int st = 0; st < S - 1; ++st) issue(st);
+    int st_c = 0, st_i = S - 1;
+
     if (x < p.T) ph1_score<Tin>(p, q_s, rp, x, ch, lane, aw0);
     group_sync(1 + g, nthr);
     for (int pass = 0; (int64_t)blockIdx.x * G + pass * stride < p.T; ++pass, x += stride) {
         const float *aw = aw0 + (pass & 1) * kPh1MaxSites * p.n;
         float *aw_next = aw0 + ((pass + 1) & 1) * kPh1MaxSites * p.n;
-        const bool live = x < p.T && e < p.d;
-        const Tin *row0 = values + x * p.d + e;
-        Frag<Tin, E> f[U];
-        // the first rows of this token travel while the next token is scored
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            if (live && u < p.n) f[u].load_nc(row0 + (int64_t)u * p.T * p.d);
-            else f[u].zero();
-        }
         if (x + stride < p.T) ph1_score<Tin>(p, q_s, rp, x + stride, ch, lane, aw_next);
         if (x < p.T) {
             float acc[kPh1MaxSites][E];
@@ -148,31 +160,26 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
             for (int j = 0; j < kPh1MaxSites; ++j)
 #pragma unroll
                 for (int t = 0; t < E; ++t) acc[j][t] = 0.f;
-            for (int i0 = 0; i0 < p.n; i0 += U) {
-                if (i0 > 0) {
+            for (int i = 0; i < p.n; ++i) {
+                issue(st_i);
+                cp_async_wait<S - 1>();  // this lane's copy of row i has landed
+                Frag<Tin, E> f;
+                if (e < p.d) f.a = ld_shared16(ring_w + 16u * 32u * st_c);
+                else f.zero();
+                st_c = (st_c + 1 == S) ? 0 : st_c + 1;
+                st_i = (st_i + 1 == S) ? 0 : st_i + 1;
+                float o[E];
+                f.get(o);
 #pragma unroll
-                    for (int u = 0; u < U; ++u) {
-                        if (live && i0 + u < p.n) f[u].load_nc(row0 + (int64_t)(i0 + u) * p.T * p.d);
-                        else f[u].zero();
-                    }
-                }
+                for (int j = 0; j < kPh1MaxSites; ++j) {
+                    if (j < p.c) {
+                        const float w = aw[j * p.n + i];
 #pragma unroll
-                for (int u = 0; u < U; ++u) {
-                    if (i0 + u < p.n) {
-                        float o[E];
-                        f[u].get(o);
-#pragma unroll
-                        for (int j = 0; j < kPh1MaxSites; ++j) {
-                            if (j < p.c) {
-                                const float w = aw[j * p.n + i0 + u];
-#pragma unroll
-                                for (int t = 0; t < E; ++t) acc[j][t] = fmaf(w, o[t], acc[j][t]);
-                            }
-                        }
+                        for (int t = 0; t < E; ++t) acc[j][t] = fmaf(w, o[t], acc[j][t]);
                     }
                 }
             }
-            if (live) {
+            if (e < p.d) {
 #pragma unroll
                 for (int j = 0; j < kPh1MaxSites; ++j) {
                     if (j < p.c) {
@@ -185,6 +192,7 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
         }
         group_sync(1 + g, nthr);  // next weights complete; this pass's weights free for reuse
     }
+    cp_async_wait_all();
 }
 
 struct Ph2Params {
@@ -270,9 +278,10 @@ static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
                 (a.variant == kSliced ? ((a.d - a.r) * esz) % 16 == 0
                                       : (reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
     const int G = kWarps / chunks;
-    const size_t smem = sizeof(float) * ((size_t)kPh1MaxSites * round_up(a.r, 4) +
-                                         (size_t)G * 2 * kPh1MaxSites * a.n);
-    const void *k = (const void *)block_phase1_kernel<Tin, Tout, 8>;
+    constexpr int S = kPh1Stages;
+    const size_t smem = (size_t)kWarps * S * 32 * 16 +
+                        sizeof(float) * ((size_t)kPh1MaxSites * round_up(a.r, 4) + (size_t)G * 2 * kPh1MaxSites * a.n);
+    const void *k = (const void *)block_phase1_kernel<Tin, Tout, S>;
     if (smem > 48 * 1024) {
         cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
@@ -283,7 +292,7 @@ static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
         p.queries = a.queries + (size_t)j0 * a.r;
         p.h_pre = static_cast<char *>(a.h_pre) + (size_t)j0 * p.site_stride * sizeof(Tout);
         p.lse_pre = a.lse_pre + (size_t)j0 * a.T;
-        block_phase1_kernel<Tin, Tout, 8><<<grid, kThreads, smem, s>>>(p);
+        block_phase1_kernel<Tin, Tout, S><<<grid, kThreads, smem, s>>>(p);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
