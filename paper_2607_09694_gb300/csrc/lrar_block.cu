@@ -20,6 +20,7 @@
 // and each pass scores the next token while the current token's rows load.
 #include "lrar_device.cuh"
 #include "lrar_launch.h"
+#include "lrar_sm100.cuh"
 
 namespace lrar {
 
@@ -73,35 +74,87 @@ __device__ __forceinline__ float ph1_dot(const Tin *__restrict__ kp, const float
     return qk;
 }
 
+// The same over a key staged in shared memory (whole 16-byte vectors).
+template <typename Tin>
+__device__ __forceinline__ float ph1_dot_s(const Tin *kp, const float *__restrict__ qj, int r, float *ss) {
+    constexpr int E = VecE<Tin>::value;
+    float qk = 0.f, s2 = 0.f;
+#pragma unroll 4
+    for (int jj = 0; jj < r; jj += E) {
+        Frag<Tin, E> f;
+        f.a = *reinterpret_cast<const uint4 *>(kp + jj);
+        float k[E];
+        f.get(k);
+#pragma unroll
+        for (int t = 0; t < E; ++t) {
+            s2 = fmaf(k[t], k[t], s2);
+            qk = fmaf(qj[jj + t], k[t], qk);
+        }
+    }
+    if (ss) *ss = s2;
+    return qk;
+}
+
+// Staged keys of one token: key i at byte i * kstride of a group's buffer
+// (r * sizeof(Tin) bytes, then 16 bytes of padding against bank conflicts).
+template <typename Tin>
+__device__ __forceinline__ int ph1_kstride(int r) {
+    return r * (int)sizeof(Tin) + 16;
+}
+
+// Copy token x's n keys into a group buffer with bulk copies counted on bar
+// (one warp: lane 0 announces the bytes, lane i copies key i).
+template <typename Tin>
+__device__ __forceinline__ void ph1_stage(const Ph1Params &p, int64_t x, int lane, uint32_t kbuf, uint32_t bar) {
+    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
+    const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
+    const uint32_t kbytes = (uint32_t)(p.r * (int)sizeof(Tin));
+    if (lane == 0) sm100::mbar_arrive_expect_tx(bar, kbytes * (uint32_t)p.n);
+    __syncwarp();
+    for (int i = lane; i < p.n; i += 32) {
+        const Tin *kp = p.sliced ? values + ((int64_t)i * p.T + x) * p.d + (p.d - p.r)
+                                 : keys + ((int64_t)i * p.T + x) * p.r;
+        sm100::bulk_load(kbuf + (uint32_t)(i * ph1_kstride<Tin>(p.r)), kp, kbytes, bar);
+    }
+}
+
 // Scores of token x for the queries j = ch, ch + chunks, ... (Eq. 8-9): lane i
-// takes source i; then the softmax of each of those queries over the n sources.
-// Weights go to aw[j * n + i], lse_j to the output.
+// takes source i, reading its key from kb_s (staged) or global memory; then the
+// softmax of each of those queries over the n sources.  Weights go to
+// aw[i * kPh1MaxSites + j] (a source's weights for every query side by side),
+// lse_j to the output.
 template <typename Tin>
 __device__ __forceinline__ void ph1_score(const Ph1Params &p, const float *__restrict__ q_s, int rp, int64_t x,
-                                          int ch, int lane, float *aw) {
+                                          int ch, int lane, float *aw, const unsigned char *kb_s = nullptr) {
     const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
     const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
     if (ch < p.c)
         for (int i = lane; i < p.n; i += 32) {
-            const Tin *kp = p.sliced ? values + ((int64_t)i * p.T + x) * p.d + (p.d - p.r)
-                                     : keys + ((int64_t)i * p.T + x) * p.r;
-            float ss;
-            const float qk0 = ph1_dot<Tin>(kp, q_s + ch * rp, p.r, p.key_vec != 0, &ss);
+            float ss, qk0;
+            const Tin *kp;
+            if (kb_s) {
+                kp = reinterpret_cast<const Tin *>(kb_s + i * ph1_kstride<Tin>(p.r));
+                qk0 = ph1_dot_s<Tin>(kp, q_s + ch * rp, p.r, &ss);
+            } else {
+                kp = p.sliced ? values + ((int64_t)i * p.T + x) * p.d + (p.d - p.r) : keys + ((int64_t)i * p.T + x) * p.r;
+                qk0 = ph1_dot<Tin>(kp, q_s + ch * rp, p.r, p.key_vec != 0, &ss);
+            }
             const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
-            aw[ch * p.n + i] = rho * qk0;
+            aw[i * kPh1MaxSites + ch] = rho * qk0;
             for (int j = ch + p.chunks; j < p.c; j += p.chunks)  // further queries of this warp (small d)
-                aw[j * p.n + i] = rho * ph1_dot<Tin>(kp, q_s + j * rp, p.r, p.key_vec != 0, nullptr);
+                aw[i * kPh1MaxSites + j] = rho * (kb_s ? ph1_dot_s<Tin>(kp, q_s + j * rp, p.r, nullptr)
+                                              : ph1_dot<Tin>(kp, q_s + j * rp, p.r, p.key_vec != 0, nullptr));
         }
     __syncwarp();
     for (int j = ch; j < p.c; j += p.chunks) {
         float m = -INFINITY;
-        for (int i = lane; i < p.n; i += 32) m = fmaxf(m, aw[j * p.n + i]);
+        for (int i = lane; i < p.n; i += 32) m = fmaxf(m, aw[i * kPh1MaxSites + j]);
         m = warp_max(m);
         float z = 0.f;
-        for (int i = lane; i < p.n; i += 32) z += expf(aw[j * p.n + i] - m);
+        for (int i = lane; i < p.n; i += 32) z += expf(aw[i * kPh1MaxSites + j] - m);
         z = warp_sum(z);
         __syncwarp();
-        for (int i = lane; i < p.n; i += 32) aw[j * p.n + i] = expf(aw[j * p.n + i] - m) / z;
+        for (int i = lane; i < p.n; i += 32) aw[i * kPh1MaxSites + j] = expf(aw[i * kPh1MaxSites + j] - m) / z;
         if (lane == 0) p.lse_pre[(int64_t)j * p.T + x] = m + logf(z);
         __syncwarp();
     }
@@ -110,18 +163,30 @@ __device__ __forceinline__ void ph1_score(const Ph1Params &p, const float *__res
 // Rows stream through a per-lane cp.async ring (each lane copies and reads
 // back its own 16-byte vector of every row), S - 1 rows ahead and across
 // tokens, so the loads of the next token's rows overlap this token's mix.
-template <typename Tin, typename Tout, int S>
+// KS: each group's keys are staged two tokens ahead in shared memory with
+// bulk copies (double-buffered, one mbarrier per buffer), so scoring reads no
+// global memory.
+// C8: exactly eight sites per launch (compile-time loop bounds); else p.c <= 8.
+template <typename Tin, typename Tout, int S, bool KS, bool C8>
 __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_constant__ Ph1Params p) {
     constexpr int E = VecE<Tin>::value;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int rp = round_up(p.r, 4);
-    float *q_s = reinterpret_cast<float *>(smem_raw + (size_t)kWarps * S * 32 * 16);  // [c][r] after the rings
-    float *a_all = q_s + kPh1MaxSites * rp;  // [G][2][kPh1MaxSites][n]: weights, double-buffered by pass
+    const int G_ = kWarps / p.chunks;
+    const int kbuf_bytes = KS ? round_up(p.n * ph1_kstride<Tin>(p.r), 16) : 0;  // one token's keys
+    unsigned char *kb_all = smem_raw + (size_t)kWarps * S * 32 * 16;           // [G][2][kbuf_bytes]
+    uint64_t *kbar_all = reinterpret_cast<uint64_t *>(kb_all + (size_t)G_ * 2 * kbuf_bytes);  // [G][2]
+    float *q_s = reinterpret_cast<float *>(kbar_all + (KS ? 2 * G_ : 0));       // [c][r]
+    float *a_all = q_s + kPh1MaxSites * rp;  // [G][2][n][kPh1MaxSites]: weights, double-buffered by pass
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int G = kWarps / p.chunks;  // tokens per CTA pass
     const int g = warp / p.chunks, ch = warp % p.chunks;
     const int nthr = p.chunks * 32;   // threads of a token group (named barrier 1 + g)
     for (int j = threadIdx.x; j < p.c * p.r; j += kThreads) q_s[(j / p.r) * rp + j % p.r] = p.queries[j];
+    if (KS && threadIdx.x < 2 * G) {
+        sm100::mbar_init(smem_u32(kbar_all + threadIdx.x), 1);
+        sm100::mbar_fence_init();
+    }
     __syncthreads();
 
     const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
@@ -130,6 +195,11 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
     float *aw0 = a_all + (size_t)g * 2 * kPh1MaxSites * p.n;
     const int64_t stride = (int64_t)gridDim.x * G;
     const uint32_t ring_w = smem_u32(smem_raw) + (uint32_t)(warp * S * 32 * 16) + 16u * lane;
+    unsigned char *kb0 = kb_all + (size_t)g * 2 * kbuf_bytes;
+    auto kbuf = [&](int b) { return smem_u32(kb0 + b * kbuf_bytes); };
+    auto kbar = [&](int b) { return smem_u32(kbar_all + 2 * g + b); };
+    // token q of this group (x0 + q * stride) uses key buffer q % 2, for the (q / 2)-th time
+    auto kwait = [&](int q) { sm100::mbar_wait(kbar(q & 1), (uint32_t)(q >> 1) & 1u, 4LL << 30); };
 
     int64_t x = (int64_t)blockIdx.x * G + g;
     int64_t ix = x;  // next row to copy: source ii of token ix
@@ -148,12 +218,24 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
     for (int st = 0; st < S - 1; ++st) issue(st);
     int st_c = 0, st_i = S - 1;
 
-    if (x < p.T) ph1_score<Tin>(p, q_s, rp, x, ch, lane, aw0);
+    if (KS && ch == 0) {
+        if (x < p.T) ph1_stage<Tin>(p, x, lane, kbuf(0), kbar(0));
+        if (x + stride < p.T) ph1_stage<Tin>(p, x + stride, lane, kbuf(1), kbar(1));
+    }
+    if (x < p.T) {
+        if (KS) kwait(0);
+        ph1_score<Tin>(p, q_s, rp, x, ch, lane, aw0, KS ? kb0 : nullptr);
+    }
     group_sync(1 + g, nthr);
     for (int pass = 0; (int64_t)blockIdx.x * G + pass * stride < p.T; ++pass, x += stride) {
         const float *aw = aw0 + (pass & 1) * kPh1MaxSites * p.n;
         float *aw_next = aw0 + ((pass + 1) & 1) * kPh1MaxSites * p.n;
-        if (x + stride < p.T) ph1_score<Tin>(p, q_s, rp, x + stride, ch, lane, aw_next);
+        // buffer pass % 2 held token `pass`, scored by every warp before the last barrier
+        if (KS && ch == 0 && x + 2 * stride < p.T) ph1_stage<Tin>(p, x + 2 * stride, lane, kbuf(pass & 1), kbar(pass & 1));
+        if (x + stride < p.T) {
+            if (KS) kwait(pass + 1);
+            ph1_score<Tin>(p, q_s, rp, x + stride, ch, lane, aw_next, KS ? kb0 + ((pass + 1) & 1) * kbuf_bytes : nullptr);
+        }
         if (x < p.T) {
             float acc[kPh1MaxSites][E];
 #pragma unroll
@@ -168,21 +250,23 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
                 else f.zero();
                 st_c = (st_c + 1 == S) ? 0 : st_c + 1;
                 st_i = (st_i + 1 == S) ? 0 : st_i + 1;
-                float o[E];
+                float o[E], w[kPh1MaxSites];
                 f.get(o);
+                const float4 w0 = *reinterpret_cast<const float4 *>(aw + i * kPh1MaxSites);
+                const float4 w1 = *reinterpret_cast<const float4 *>(aw + i * kPh1MaxSites + 4);
+                w[0] = w0.x, w[1] = w0.y, w[2] = w0.z, w[3] = w0.w, w[4] = w1.x, w[5] = w1.y, w[6] = w1.z, w[7] = w1.w;
 #pragma unroll
                 for (int j = 0; j < kPh1MaxSites; ++j) {
-                    if (j < p.c) {
-                        const float w = aw[j * p.n + i];
+                    if (C8 || j < p.c) {
 #pragma unroll
-                        for (int t = 0; t < E; ++t) acc[j][t] = fmaf(w, o[t], acc[j][t]);
+                        for (int t = 0; t < E; ++t) acc[j][t] = fmaf(w[j], o[t], acc[j][t]);
                     }
                 }
             }
             if (e < p.d) {
 #pragma unroll
                 for (int j = 0; j < kPh1MaxSites; ++j) {
-                    if (j < p.c) {
+                    if (C8 || j < p.c) {
                         Frag<Tout, E> out;
                         out.set(acc[j]);
                         out.store(h_pre + (int64_t)j * p.site_stride + x * p.d + e);
@@ -279,12 +363,22 @@ static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
                                       : (reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
     const int G = kWarps / chunks;
     constexpr int S = kPh1Stages;
-    const size_t smem = (size_t)kWarps * S * 32 * 16 +
+    const int kstride = a.r * (int)sizeof(Tin) + 16;
+    const size_t kbuf_bytes = (size_t)round_up(a.n * kstride, 16);
+    const bool ks = p.key_vec && kbuf_bytes <= 4096;  // keys staged in shared memory
+    const size_t smem = (size_t)kWarps * S * 32 * 16 + (ks ? (size_t)G * 2 * (kbuf_bytes + 8) : 0) +
                         sizeof(float) * ((size_t)kPh1MaxSites * round_up(a.r, 4) + (size_t)G * 2 * kPh1MaxSites * a.n);
-    const void *k = (const void *)block_phase1_kernel<Tin, Tout, S>;
-    if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
+    const void *k = ks ? (const void *)block_phase1_kernel<Tin, Tout, S, true, true>
+                       : (const void *)block_phase1_kernel<Tin, Tout, S, false, true>;  // same resources for C8 or not
+    if (smem > 48 * 1024) {  // every variant this call may launch (8 sites, or the rest)
+        const void *ks_all[4] = {(const void *)block_phase1_kernel<Tin, Tout, S, true, true>,
+                                 (const void *)block_phase1_kernel<Tin, Tout, S, true, false>,
+                                 (const void *)block_phase1_kernel<Tin, Tout, S, false, true>,
+                                 (const void *)block_phase1_kernel<Tin, Tout, S, false, false>};
+        for (const void *kk : ks_all) {
+            cudaError_t e = cudaFuncSetAttribute(kk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (e != cudaSuccess) return e;
+        }
     }
     const int grid = persistent_grid(k, kThreads, smem, (a.T + G - 1) / G, 1 << 30);
     for (int j0 = 0; j0 < a.c; j0 += kPh1MaxSites) {  // groups of at most 8 queries
@@ -292,7 +386,11 @@ static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
         p.queries = a.queries + (size_t)j0 * a.r;
         p.h_pre = static_cast<char *>(a.h_pre) + (size_t)j0 * p.site_stride * sizeof(Tout);
         p.lse_pre = a.lse_pre + (size_t)j0 * a.T;
-        block_phase1_kernel<Tin, Tout, S><<<grid, kThreads, smem, s>>>(p);
+        const bool c8 = p.c == kPh1MaxSites;
+        if (ks && c8) block_phase1_kernel<Tin, Tout, S, true, true><<<grid, kThreads, smem, s>>>(p);
+        else if (ks) block_phase1_kernel<Tin, Tout, S, true, false><<<grid, kThreads, smem, s>>>(p);
+        else if (c8) block_phase1_kernel<Tin, Tout, S, false, true><<<grid, kThreads, smem, s>>>(p);
+        else block_phase1_kernel<Tin, Tout, S, false, false><<<grid, kThreads, smem, s>>>(p);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
