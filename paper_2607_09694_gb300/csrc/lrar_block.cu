@@ -301,13 +301,46 @@ __global__ void __launch_bounds__(kThreads) block_phase2_kernel(const Ph2Params 
     Tout *__restrict__ h = static_cast<Tout *>(p.h);
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     for (int64_t x = (int64_t)blockIdx.x * kWarps + warp; x < p.T; x += nwarps) {
-        // score of the partial summary, Eq. (8)-(9)
-        const Tin *kp = p.sliced ? part + x * p.d + (p.d - p.r) : pkeys + x * p.r;
+        // both rows first: their loads travel while the partial summary is scored
+        Frag<Tin, E> fb[V];
+        Frag<Tp, E> fh[V];
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int e = (lane + 32 * v) * E;
+            if (e < p.d) {
+                fb[v].load_nc(part + x * p.d + e);
+                fh[v].load_nc(h_pre + x * p.d + e);
+            } else {
+                fb[v].zero();
+                fh[v].zero();
+            }
+        }
+        // score of the partial summary, Eq. (8)-(9); an S-LR key is the tail of
+        // the summary row already in registers
         float ss = 0.f, qk = 0.f;
-        for (int j = lane; j < p.r; j += 32) {
-            const float k = to_f(__ldg(kp + j));
-            ss = fmaf(k, k, ss);
-            qk = fmaf(__ldg(p.query + j), k, qk);
+        if (p.sliced) {
+            const int k0 = p.d - p.r;
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e + E > k0 && e < p.d) {
+                    float b[E];
+                    fb[v].get(b);
+#pragma unroll
+                    for (int t = 0; t < E; ++t)
+                        if (e + t >= k0) {
+                            ss = fmaf(b[t], b[t], ss);
+                            qk = fmaf(__ldg(p.query + (e + t - k0)), b[t], qk);
+                        }
+                }
+            }
+        } else {
+            const Tin *kp = pkeys + x * p.r;
+            for (int j = lane; j < p.r; j += 32) {
+                const float k = to_f(__ldg(kp + j));
+                ss = fmaf(k, k, ss);
+                qk = fmaf(__ldg(p.query + j), k, qk);
+            }
         }
         ss = warp_sum(ss);
         qk = warp_sum(qk);
@@ -320,13 +353,9 @@ __global__ void __launch_bounds__(kThreads) block_phase2_kernel(const Ph2Params 
         for (int v = 0; v < V; ++v) {
             const int e = (lane + 32 * v) * E;
             if (e < p.d) {
-                Frag<Tin, E> fb;
-                fb.load_nc(part + x * p.d + e);
-                Frag<Tp, E> fh;
-                fh.load_nc(h_pre + x * p.d + e);
                 float b[E], hp[E], o[E];
-                fb.get(b);
-                fh.get(hp);
+                fb[v].get(b);
+                fh[v].get(hp);
 #pragma unroll
                 for (int t = 0; t < E; ++t) o[t] = fmaf(w2, b[t], w1 * hp[t]);
                 Frag<Tout, E> out;
