@@ -439,6 +439,38 @@ def run_profile_site(args):
                       "fwd_gbs": fb / f / 1e6, "bwd_gbs": bb / b / 1e6}), flush=True)
 
 
+def run_profile_block(args):
+    """Small case of the Block two-phase path for profilers: phase 1 over the
+    last block of the d = 2048 decoder (9 completed sources, 8 sites, r = 64,
+    bf16 h_pre) and phase 2 for one site, --profile-block T tokens."""
+    import torch
+
+    from __graft_entry__ import build
+    from paper_2607_09694_gb300 import lrar, synth
+
+    build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    T, d, r, c, n = args.profile_block, 2048, 64, 8, 9
+    stack = synth.values(n + 1, T, d, 3, "bf16", device=dev)
+    qs = synth.queries(c, r, 3, device=dev)
+    h_pre = torch.empty(c, T, d, dtype=torch.bfloat16, device=dev)
+    lse_pre = torch.empty(c, T, device=dev)
+    h = torch.empty(T, d, dtype=torch.bfloat16, device=dev)
+    lse = torch.empty(T, device=dev)
+    ph1 = lambda: lrar.block_phase1("sliced", stack, None, qs, h_pre, lse_pre, n_completed=n)  # noqa: E731
+    ph2 = lambda: lrar.block_phase2("sliced", h_pre[1], lse_pre[1], stack[n], None, qs[1], h, lse)  # noqa: E731
+    for _ in range(args.warmup):
+        ph1()
+        ph2()
+    m1 = _median_ms(torch, ph1, args.steps)
+    m2 = _median_ms(torch, ph2, args.steps)
+    b1 = T * (n * d * 2 + c * (d * 2 + 4))
+    b2 = T * (3 * d * 2 + 8)
+    print(json.dumps({"profile_block": T, "phase1_ms": m1, "phase1_gbs": b1 / m1 / 1e6, "phase2_ms": m2,
+                      "phase2_gbs": b2 / m2 / 1e6}), flush=True)
+
+
 def run_profile_proj(args):
     """Small case of the fused projection for profilers: --profile-proj m, with
     --tokens T, --site-d d, --site-r r (bf16 operands)."""
@@ -782,6 +814,8 @@ def main():
     ap.add_argument("--site-d", type=int, default=D, help="width d of the --profile-site case")
     ap.add_argument("--site-r", type=int, default=R, help="key rank r of the --profile-site case (not full)")
     ap.add_argument("--suite", action="store_true", help="time every workload's headline site (JSON line each)")
+    ap.add_argument("--profile-block", type=int, default=0,
+                    help="time the Block two-phase path on this many tokens (profiling)")
     ap.add_argument("--profile-proj", type=int, default=0,
                     help="time the fused projection with this input width m (profiling; --tokens, --site-d, --site-r)")
     args = ap.parse_args()
@@ -793,6 +827,8 @@ def main():
         run_profile_site(args)
     elif args.profile_proj:
         run_profile_proj(args)
+    elif args.profile_block:
+        run_profile_block(args)
     elif args.impl == "reference":
         run_reference(args)
     else:
