@@ -109,3 +109,37 @@ def test_slr_d2048_n65_t32768():
     c = synth.CONFIGS["slr_large"]
     vals = synth.values(c["n"], c["T"], c["d"], c["seed"], "bf16")
     _bench_like(_site("slr_large", vals))
+
+
+def test_block_two_phase_d2048_t32768():
+    """The Block decoder's last block at full size (T = 32768, d = 2048, r = 64,
+    c = 8, 9 completed sources, bf16 h_pre as the benchmark's faster setting):
+    phase 1 for the block's eight sites, phase 2 for one of them, on sampled
+    tokens against the oracle's mix over the site's whole source set."""
+    c = synth.CONFIGS["block"]
+    T, d, r, cb = c["T"], c["d"], c["r"], c["block_c"]
+    n = 9
+    dev = torch.device("cuda")
+    stack = synth.values(n + 1, T, d, c["seed"], "bf16")  # 9 completed sources, then a partial summary
+    qs = synth.queries(cb, r, c["seed"], std=0.5)
+    sd = stack.to(dev)
+    h_pre = torch.empty(cb, T, d, dtype=torch.bfloat16, device=dev)
+    lse_pre = torch.empty(cb, T, device=dev)
+    lrar.block_phase1("sliced", sd, None, qs.to(dev), h_pre, lse_pre, n_completed=n)
+    h = torch.empty(T, d, device=dev)
+    lse = torch.empty(T, device=dev)
+    lrar.block_phase2("sliced", h_pre[3], lse_pre[3], sd[n], None, qs[3].to(dev), h, lse)
+    torch.cuda.synchronize()
+    toks = H.sample_tokens(T, k=24, seed=3)
+    idx = torch.as_tensor(toks, dtype=torch.long, device=dev)
+    # phase 1 alone: site 0's mix over the completed sources (h_pre rounded to bf16 once)
+    ref1 = oracle.forward(oracle.SLICED, stack[:n], None, qs[0], H.EPS, r=r, tokens=toks)
+    H.assert_bf16_rounded("h_pre[0]", h_pre[0].index_select(0, idx).double().cpu().numpy(), ref1["h"])
+    H.assert_abs("lse_pre[0]", lse_pre[0].index_select(0, idx).double().cpu().numpy(), ref1["lse"], 1e-4)
+    # both phases: site 3's mix over the completed sources and the partial summary
+    ref = oracle.forward(oracle.SLICED, stack, None, qs[3], H.EPS, r=r, tokens=toks)
+    got = h.index_select(0, idx).double().cpu().numpy()
+    pre_ref = oracle.forward(oracle.SLICED, stack[:n], None, qs[3], H.EPS, r=r, tokens=toks)
+    bound = 0.5 * H.bf16_ulp(pre_ref["h"]) + 1e-5 * H.rms(ref["h"])  # h_pre rounded once, weight <= 1
+    assert np.all(np.abs(got - ref["h"]) <= bound)
+    H.assert_abs("lse", lse.index_select(0, idx).double().cpu().numpy(), ref["lse"], 1e-4)
