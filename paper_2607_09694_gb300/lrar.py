@@ -104,10 +104,17 @@ def dtype_code(t: torch.Tensor | None, default: int = F32) -> int:
 
 
 def _ptr(t) -> int | None:
+    """Device address of a tensor argument (None -> NULL).  Every tensor the
+    library reads or writes must be a contiguous CUDA tensor: a host tensor's
+    address would be dereferenced on the GPU."""
     if t is None:
         return None
     if isinstance(t, int):
         return t
+    if not t.is_cuda:
+        raise LrarError(ERR_INVALID_ARG, "tensor arguments must be CUDA tensors")
+    if not t.is_contiguous():
+        raise LrarError(ERR_INVALID_ARG, "tensor arguments must be contiguous")
     return t.data_ptr()
 
 
@@ -163,7 +170,7 @@ def _table(ts):
     """Host array of device pointers for a list of source tensors (None -> NULL)."""
     if ts is None:
         return None
-    return (ctypes.c_void_p * len(ts))(*[t.data_ptr() for t in ts])
+    return (ctypes.c_void_p * len(ts))(*[_ptr(t) for t in ts])
 
 
 def forward_ptrs(variant, values, keys, query: torch.Tensor | None, h: torch.Tensor, lse: torch.Tensor | None = None,

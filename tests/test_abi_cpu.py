@@ -210,3 +210,15 @@ def test_pointer_tables_rejected_before_launch(lib):
              None) == lrar.ERR_ALIGNMENT
     assert b(1, 1, 1, good, None, FAKE, n, T, d, r, EPS, FAKE, None, 1, None, good, None, FAKE, 0, FAKE, 16,
              None) == lrar.ERR_WORKSPACE
+
+
+def test_binding_rejects_host_and_strided_tensors(lib):
+    """The binding hands the library device addresses only: a host tensor or a
+    non-contiguous view is refused before any call (no GPU needed to check)."""
+    import torch
+
+    v = torch.zeros(2, 4, 64)
+    with pytest.raises(lrar.LrarError) as ei:
+        lrar.forward("sliced", v, None, torch.zeros(4), torch.zeros(4, 64), n_src=2)
+    assert ei.value.code == lrar.ERR_INVALID_ARG
+    assert "CUDA" in str(ei.value)
