@@ -157,6 +157,30 @@ def test_source_permutation(variant, d, r):
     assert np.allclose(b0["dq"], b1["dq"], atol=1e-13)
 
 
+@pytest.mark.parametrize("variant,d,r", [(SLICED, 10, 3), (FULL, 8, 8)])
+def test_hidden_coordinate_permutation(variant, d, r):
+    """§3.4: which r coordinates form the S-LR key is arbitrary up to a
+    permutation of the hidden coordinates.  Permuting the head coordinates
+    among themselves and the key coordinates among themselves (with the query
+    permuted alike) permutes h, the value gradients and dq the same way, and
+    leaves lse unchanged; for full keys any permutation does."""
+    n, T = 5, 4
+    v, _, q, dh = _case(variant, n, T, d, r, seed=12)
+    g = _rng(13)
+    head, tail = np.arange(d - r), np.arange(d - r, d)
+    perm = np.concatenate([g.permutation(head), d - r + g.permutation(r)]) if variant == SLICED \
+        else g.permutation(d)
+    qperm = perm[d - r:] - (d - r)  # the key slice's own coordinates, in the permuted order
+    f0 = oracle.forward(variant, v, None, q, EPS, r=r)
+    f1 = oracle.forward(variant, v[:, :, perm], None, q[qperm], EPS, r=r)
+    assert np.allclose(f0["h"][:, perm], f1["h"], atol=1e-14)
+    assert np.allclose(f0["lse"], f1["lse"], atol=1e-14)
+    b0 = oracle.backward(variant, v, None, q, EPS, dh, r=r)
+    b1 = oracle.backward(variant, v[:, :, perm], None, q[qperm], EPS, dh[:, perm], r=r)
+    assert np.allclose(b0["dvalues"][:, :, perm], b1["dvalues"], atol=1e-13)
+    assert np.allclose(b0["dq"][qperm], b1["dq"], atol=1e-13)
+
+
 def test_key_scale_invariance():
     """RMSNorm makes the score invariant to positive rescaling of a key, up to eps."""
     n, T, d, r = 5, 3, 8, 4
