@@ -598,9 +598,13 @@ __device__ __forceinline__ void full_bwd_row(const Frag<Tin, VecE<Tin>::value> *
         q_get<E>(q_s, v, lane, qv);
 #pragma unroll
         for (int t = 0; t < E; ++t) {
+            if constexpr (!DQS) {  // packed pairs pay where dq stays in registers
+                fma2(ss, qo, o[t], qv[t], o[t], o[t]);  // o.o, q.o
+            } else {
+                ss = fmaf(o[t], o[t], ss);
+                qo = fmaf(qv[t], o[t], qo);
+            }
             g = fmaf(dv[t], o[t], g);
-            ss = fmaf(o[t], o[t], ss);
-            qo = fmaf(qv[t], o[t], qo);
         }
     }
     g = warp_sum(g);
@@ -624,13 +628,22 @@ __device__ __forceinline__ void full_bwd_row(const Frag<Tin, VecE<Tin>::value> *
             else
 #pragma unroll
                 for (int t = 0; t < E; ++t) w[t] = 0.f;
+            if constexpr (!DQS) {
 #pragma unroll
-            for (int t = 0; t < E; ++t) {
-                w[t] = fmaf(a, dv[t], w[t]);
-                w[t] = fmaf(c1, qv[t], w[t]);
-                w[t] = fmaf(-c2, o[t], w[t]);
-                if (DQS) dqf[e + t] = fmaf(c1, o[t], dqf[e + t]);  // this warp's row in shared memory
-                else dqf[v * E + t] = fmaf(c1, o[t], dqf[v * E + t]);
+                for (int t = 0; t < E; t += 2) {
+                    fma2(w[t], w[t + 1], a, a, dv[t], dv[t + 1]);
+                    fma2(w[t], w[t + 1], c1, c1, qv[t], qv[t + 1]);
+                    fma2(w[t], w[t + 1], -c2, -c2, o[t], o[t + 1]);
+                    fma2(dqf[v * E + t], dqf[v * E + t + 1], c1, c1, o[t], o[t + 1]);
+                }
+            } else {
+#pragma unroll
+                for (int t = 0; t < E; ++t) {
+                    w[t] = fmaf(a, dv[t], w[t]);
+                    w[t] = fmaf(c1, qv[t], w[t]);
+                    w[t] = fmaf(-c2, o[t], w[t]);
+                    dqf[e + t] = fmaf(c1, o[t], dqf[e + t]);  // this warp's row in shared memory
+                }
             }
             Frag<Tg, E> out;
             out.set(w);

@@ -190,4 +190,13 @@ __device__ __forceinline__ T *dst_row(const SrcTab &t, int i, int64_t x, int wid
     return static_cast<T *>(const_cast<void *>(t.p[i])) + x * width;
 }
 
+// Two fp32 fused multiply-adds in one packed instruction (d_k = a_k b_k + d_k,
+// each rounded to nearest even: the same results as two fmaf).
+__device__ __forceinline__ void fma2(float &d0, float &d1, float a0, float a1, float b0, float b1) {
+    asm("{\n\t.reg .b64 ra, rb, rc;\n\tmov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%0, %1};\n\t"
+        "fma.rn.f32x2 rc, ra, rb, rc;\n\tmov.b64 {%0, %1}, rc;\n\t}"
+        : "+f"(d0), "+f"(d1)
+        : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+
 }  // namespace lrar

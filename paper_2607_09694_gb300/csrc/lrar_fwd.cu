@@ -273,8 +273,12 @@ __device__ __forceinline__ void full_row_step(const Frag<Tin, VecE<Tin>::value> 
         q_get<E>(q_s, v, lane, qv);  // q is zero past d
 #pragma unroll
         for (int t = 0; t < E; ++t) {
-            ss = fmaf(o[v * E + t], o[v * E + t], ss);
-            qo = fmaf(qv[t], o[v * E + t], qo);
+            if constexpr (V * E <= 32) {  // packed pairs pay where the row fits 32 values per lane
+                fma2(ss, qo, o[v * E + t], qv[t], o[v * E + t], o[v * E + t]);  // o.o, q.o
+            } else {
+                ss = fmaf(o[v * E + t], o[v * E + t], ss);
+                qo = fmaf(qv[t], o[v * E + t], qo);
+            }
         }
     }
     ss = warp_sum(ss);
@@ -289,8 +293,13 @@ __device__ __forceinline__ void full_row_step(const Frag<Tin, VecE<Tin>::value> 
     }
     const float w = expf(s - m);
     z += w;
+    if constexpr (V * E <= 32) {
 #pragma unroll
-    for (int t = 0; t < V * E; ++t) acc[t] = fmaf(w, o[t], acc[t]);
+        for (int t = 0; t < V * E; t += 2) fma2(acc[t], acc[t + 1], w, w, o[t], o[t + 1]);
+    } else {
+#pragma unroll
+        for (int t = 0; t < V * E; ++t) acc[t] = fmaf(w, o[t], acc[t]);
+    }
 }
 
 // One warp per token; each lane streams its own 16-byte vectors of the source
