@@ -222,3 +222,23 @@ def test_binding_rejects_host_and_strided_tensors(lib):
         lrar.forward("sliced", v, None, torch.zeros(4), torch.zeros(4, 64), n_src=2)
     assert ei.value.code == lrar.ERR_INVALID_ARG
     assert "CUDA" in str(ei.value)
+
+
+def _no_cuda_device():
+    try:
+        import torch
+
+        return not torch.cuda.is_available()
+    except Exception:  # pragma: no cover
+        return True
+
+
+@pytest.mark.skipif(not _no_cuda_device(), reason="needs a machine without a usable CUDA device")
+def test_cuda_failures_surface_as_lrar_err_cuda(lib):
+    """A CUDA runtime failure (here: no usable device or driver) is reported as
+    LRAR_ERR_CUDA with the CUDA error's name in the thread's message.  Only run
+    where no device exists: the arguments are placeholder addresses."""
+    assert fwd(lib) == lrar.ERR_CUDA
+    assert b"cuda" in lib.lrar_last_error().lower()
+    assert bwd(lib) == lrar.ERR_CUDA
+    assert lib.lrar_project(1, FAKE, FAKE, 8, 64, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_CUDA
