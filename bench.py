@@ -193,7 +193,7 @@ class Workload:
             if events is not None:
                 events["bwd"][t - 1][0].record()
             lrar.backward(lrar.SLICED, self.values, None, q, self.dh[t - 1], self.dvalues, self.dq[t - 1], self.ws,
-                          n_src=t, r=R, accumulate=(t != N_SITES), eps=EPS)
+                          lse=self.lse[t - 1], n_src=t, r=R, accumulate=(t != N_SITES), eps=EPS)
             if events is not None:
                 events["bwd"][t - 1][1].record()
 
@@ -394,8 +394,8 @@ def time_site(wl, n: int, accumulate: bool, reps: int):
         e[0].record()
         lrar.forward(lrar.SLICED, wl.values, None, q, wl.h[n - 1], wl.lse[n - 1], n_src=n, r=R, eps=EPS)
         e[1].record()
-        lrar.backward(lrar.SLICED, wl.values, None, q, wl.dh[n - 1], wl.dvalues, wl.dq[n - 1], wl.ws, n_src=n, r=R,
-                      accumulate=accumulate, eps=EPS)
+        lrar.backward(lrar.SLICED, wl.values, None, q, wl.dh[n - 1], wl.dvalues, wl.dq[n - 1], wl.ws,
+                      lse=wl.lse[n - 1], n_src=n, r=R, accumulate=accumulate, eps=EPS)
         e[2].record()
     torch.cuda.synchronize()
     f_ms = [e[0].elapsed_time(e[1]) for e in evs]
@@ -732,7 +732,7 @@ def run_e2e(wl, args, dist, dev, step_bytes, world):
             comp.wait_event(E["dh_in"][t - 1])
             q = B["queries"][t - 1] if t > 1 else None
             lrar.backward(lrar.SLICED, B["values"], None, q, B["dh"][t - 1], B["dvalues"], B["dq"][t - 1], wl.ws,
-                          n_src=t, r=R, accumulate=(t != N_SITES), eps=EPS)
+                          lse=B["lse"][t - 1], n_src=t, r=R, accumulate=(t != N_SITES), eps=EPS)
             E["bwd"][t - 1].record(comp)
             s_out.wait_event(E["bwd"][t - 1])
             with torch.cuda.stream(s_out):

@@ -114,7 +114,14 @@ size_t lrar_backward_workspace_size(int variant, int n_src, int64_t T, int d, in
  *              output): at most alpha_i rho_i |q - (s_i/d) kbar_i| sum_j |dh_j|
  *              ulp(h_j)/2 per gradient element
  *   h_dtype    element type of h
- *   lse        [T] float32 from the forward; required for LRAR_FULL, ignored otherwise
+ *   lse        [T] float32 from the forward (4-byte aligned); required for LRAR_FULL.
+ *              LRAR_SLICED may take it: when the gradients are written
+ *              (accumulate = 0) and in_dtype == grad_dtype, alpha_i = exp(s_i - lse)
+ *              comes from each value row's own key slice and the backward makes one
+ *              pass over the values instead of a routing stage, a value pass and a
+ *              key pass (same results up to fp32 rounding order).  It must be the
+ *              forward's lse of the same values and query.  NULL: the sliced
+ *              backward recomputes the routing.  Ignored for LRAR_PROJECTED.
  *   dvalues    [n_src, T, d] grad_dtype, written (accumulate = 0) or added into
  *   dkeys      [n_src, T, r] grad_dtype; LRAR_PROJECTED only, same accumulate rule
  *   dq         [r] float32, written or added into; summed over all T tokens

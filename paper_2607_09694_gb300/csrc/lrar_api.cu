@@ -196,7 +196,7 @@ int backward_impl(int variant, int in_dtype, int grad_dtype, const void *const *
     if (variant == LRAR_FULL && (!h || !lse))
         return fail(LRAR_ERR_INVALID_ARG, "full AttnRes backward needs the forward's h and lse");
     if (!query && n_src > 1) return fail(LRAR_ERR_INVALID_ARG, "query is required when n_src > 1");
-    if (!aligned16(dh) || !aligned4(dq) || (variant == LRAR_FULL && (!aligned16(h) || !aligned4(lse))) ||
+    if (!aligned16(dh) || !aligned4(dq) || (variant == LRAR_FULL && !aligned16(h)) || (lse && !aligned4(lse)) ||
         (query && !aligned4(query)))
         return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (query, lse and dq 4-byte)");
     if (!workspace || workspace_bytes < lrar_backward_workspace_size(variant, n_src, T, d, r))
@@ -218,7 +218,7 @@ int backward_impl(int variant, int in_dtype, int grad_dtype, const void *const *
     a.eps = eps;
     a.dh = dh;
     a.h = variant == LRAR_FULL ? h : nullptr;
-    a.lse = variant == LRAR_FULL ? lse : nullptr;
+    a.lse = variant == LRAR_PROJECTED ? nullptr : lse;  // SLICED: one pass over the values when given
     a.dvalues = dvalues;
     a.dkeys = variant == LRAR_PROJECTED ? dkeys : nullptr;
     a.dq = dq;

@@ -13,7 +13,9 @@
 // 16-byte vector that does not lie wholly in the key slice; (3) the key pass,
 // with gbar known, forms ds_i and dL/dk_i lane-per-key-coordinate, writes the
 // key slice of dvalues (SLICED: alpha_i dh + dL/dk_i in one rounding) or dkeys
-// (PROJECTED), and accumulates dq.
+// (PROJECTED), and accumulates dq.  Sliced keys with the forward's lse and
+// written gradients skip (1) and fold (3) into the same pass
+// (bwd_slr_onepass_kernel): alpha_i = exp(s_i - lse) from the row's own slice.
 //
 // Full keys (r = d): ds_i needs gbar before row i can be written, and gbar =
 // <dh, h> because h = sum_i alpha_i o_i, so a single pass needs the forward's
@@ -804,6 +806,238 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_full_pipe_kernel(const __grid
     full_dq_partial<T, V, DQS>(p, dqf, scratch, lane, warp);
 }
 
+// ---------------------------------------------------- sliced, one pass ----
+// Sliced keys, one dtype for inputs and gradients, with the forward's lse: the
+// key of row i is that row's last r coordinates, so the row streamed for the
+// value gradient carries its key and no routing stage is needed.  The
+// NV = r / E lanes holding the slice (one 16-byte vector each; an aligned
+// group of lanes because NV divides 32 and r divides d) form |k_i|^2 and
+// q.k_i with a butterfly over the group, which gives rho_i, s_i and
+// alpha_i = exp(s_i - lse).  Every lane writes alpha_i dh (+ old) for its
+// vectors before the slice, and the slice lanes park the row's key vector
+// (and old gradient vector) in a per-warp stash in shared memory.  After the
+// token's last row gbar = sum_i alpha_i g_i is exact, and all 32 lanes finish
+// the slices from the stash (ds_i, dL/dk_i, old + alpha_i dh + dL/dk_i in one
+// rounding, dq) as key_pass_vec does from global memory.  Every value row and
+// every gradient row crosses HBM once.  The launcher runs the writing form
+// (ACC = false); see launch_bwd_t for the accumulating one.
+//
+// Shared memory: ring [kWarps][S][P][V][32] cells | q [rp] | dq [kWarps][rp] |
+// tables [kWarps][4][n4] (alpha, s, rho, g) | per warp: stash [n][P][NV]
+// cells and the token's dh slice [NV] cells.
+template <int V, bool ACC> struct OnePassStages {
+    static constexpr int raw = 40 / (V * (ACC ? 2 : 1));  // a ring of about 160 KB per CTA
+    static constexpr int value = raw < 2 ? 2 : (raw > 8 ? 8 : raw);
+};
+
+inline size_t onepass_smem(int S, int P, int V, int n, int r, int nv) {
+    const int rp = round_up(r, 4), n4 = round_up(n, 4);
+    return (size_t)kWarps * S * P * V * 32 * 16 + sizeof(float) * (size_t)rp * (1 + kWarps) +
+           (size_t)kWarps * (sizeof(float) * 4 * n4 + (size_t)16 * nv * (n * P + 1));
+}
+
+template <typename T, int V, int S, bool ACC>
+__global__ void __launch_bounds__(kThreads, 1) bwd_slr_onepass_kernel(const __grid_constant__ BwdParams p) {
+    constexpr int E = VecE<T>::value;
+    constexpr int P = ACC ? 2 : 1;
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int rp = round_up(p.r, 4), n4 = round_up(p.n, 4);
+    const int nv = p.r / E;
+    float *q_s = reinterpret_cast<float *>(smem_raw + (size_t)kWarps * S * P * V * 32 * 16);
+    float *dq_all = q_s + rp;           // [kWarps][rp]
+    float *tab = dq_all + kWarps * rp;  // [kWarps][4][n4]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    float *a_s = tab + warp * 4 * n4;
+    float *s_s = a_s + n4;
+    float *rho_s = s_s + n4;
+    float *g_s = rho_s + n4;
+    const uint32_t stash_w = smem_u32(tab + kWarps * 4 * n4) + (uint32_t)(warp * nv * (p.n * P + 1) * 16);
+    const uint32_t dhs_w = stash_w + (uint32_t)(p.n * P * nv * 16);
+    const uint32_t ring_w = smem_u32(smem_raw) + (uint32_t)(warp * S * P * V * 32 * 16) + 16u * lane;
+    for (int j = threadIdx.x; j < p.r; j += kThreads) q_s[j] = p.query ? p.query[j] : 0.f;
+    __syncthreads();
+
+    const T *__restrict__ dh = static_cast<const T *>(p.dh);
+    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+    const int tail0 = p.d - p.r;  // a whole number of vectors
+    const int tv0 = tail0 / E;    // first slice vector of a row
+    const int lead = tv0 % 32;    // lanes lead .. lead + nv - 1 hold the slice, all in register slot vk
+    const int vk = tv0 / 32;
+    const int kvi = lane - lead;
+    const bool has_key = kvi >= 0 && kvi < nv;
+    const int qi = has_key ? kvi * E : 0;  // r >= E, so q_s[qi + t] is in range for every lane
+    float qv[E];
+#pragma unroll
+    for (int t = 0; t < E; ++t) qv[t] = has_key ? q_s[qi + t] : 0.f;
+    // slice pass: lane takes slice vector kp of sources lane / nv, lane / nv + kst, ...
+    const int kp = lane % nv, kst = 32 / nv, j0 = kp * E;
+    float dq_r[E];
+#pragma unroll
+    for (int t = 0; t < E; ++t) dq_r[t] = 0.f;
+    auto stash = [&](int i, int plane, int c) -> uint32_t {
+        return stash_w + (uint32_t)(((i * P + plane) * nv + c) * 16);
+    };
+
+    const int64_t x0 = (int64_t)blockIdx.x * kWarps + warp;
+    int64_t ix = x0;  // next row to copy: source ii of token ix
+    int ii = 0;
+    auto cell = [&](int st, int plane, int v) -> uint32_t {
+        return ring_w + (uint32_t)((((st * P + plane) * V + v) * 32) * 16);
+    };
+    auto issue = [&](int st) {
+        if (ix < p.T) {
+            const T *row = src_row<T>(p.vt, ii, ix, p.d);
+            const T *old = ACC ? dst_row<T>(p.dvt, ii, ix, p.d) : nullptr;
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) {
+                    cp_async16(cell(st, 0, v), row + e);
+                    if (ACC) cp_async16(cell(st, P - 1, v), old + e);
+                }
+            }
+            if (++ii == p.n) {
+                ii = 0;
+                ix += nwarps;
+            }
+        }
+        cp_async_commit();
+    };
+#pragma unroll
+    for (int st = 0; st < S - 1; ++st) issue(st);
+    int st_c = 0, st_i = S - 1;
+
+    for (int64_t x = x0; x < p.T; x += nwarps) {
+        const int64_t row_off = x * p.d;
+        Frag<T, E> dhr[V];
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int e = (lane + 32 * v) * E;
+            if (e < p.d) dhr[v].load_nc(dh + row_off + e);
+            else dhr[v].zero();
+        }
+        const float lse = __ldg(p.lse + x);
+#pragma unroll
+        for (int v = 0; v < V; ++v)
+            if (v == vk && has_key) st_shared16(dhs_w + (uint32_t)(kvi * 16), dhr[v].a);
+
+        for (int i = 0; i < p.n; ++i) {
+            issue(st_i);
+            cp_async_wait<S - 1>();  // this lane's copies of row i have landed
+            Frag<T, E> f[V], old[V];
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) f[v].a = ld_shared16(cell(st_c, 0, v));
+                else f[v].zero();
+                if (ACC && e < p.d) old[v].a = ld_shared16(cell(st_c, P - 1, v));
+                else old[v].zero();
+            }
+            float g0 = 0.f, g1 = 0.f, ss = 0.f, qk = 0.f;
+#pragma unroll
+            for (int v = 0; v < V; ++v) {  // vectors past d are zero
+                float o[E], dv[E];
+                f[v].get(o);
+                dhr[v].get(dv);
+#pragma unroll
+                for (int t = 0; t < E; t += 2) fma2(g0, g1, dv[t], dv[t + 1], o[t], o[t + 1]);
+                if (v == vk && has_key) {
+#pragma unroll
+                    for (int t = 0; t < E; ++t) {
+                        ss = fmaf(o[t], o[t], ss);
+                        qk = fmaf(qv[t], o[t], qk);
+                    }
+                    st_shared16(stash(i, 0, kvi), f[v].a);
+                    if (ACC) st_shared16(stash(i, 1, kvi), old[v].a);
+                }
+            }
+            for (int off = 1; off < nv; off <<= 1) {  // the slice group is aligned: partners stay inside
+                ss += __shfl_xor_sync(0xffffffffu, ss, off);
+                qk += __shfl_xor_sync(0xffffffffu, qk, off);
+            }
+            const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
+            const float s = __shfl_sync(0xffffffffu, rho * qk, lead);
+            const float a = expf(s - lse);
+            T *drow = dst_row<T>(p.dvt, i, x, p.d);
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < tail0) {
+                    float dv[E], w[E];
+                    dhr[v].get(dv);
+                    if (ACC) old[v].get(w);
+                    else
+#pragma unroll
+                        for (int t = 0; t < E; ++t) w[t] = 0.f;
+#pragma unroll
+                    for (int t = 0; t < E; ++t) w[t] = fmaf(a, dv[t], w[t]);
+                    Frag<T, E> out;
+                    out.set(w);
+                    out.store(drow + e);
+                }
+            }
+            const float g = warp_sum(g0 + g1);
+            if (lane == lead) {
+                a_s[i] = a;
+                s_s[i] = s;
+                rho_s[i] = rho;
+                g_s[i] = g;
+            }
+            st_c = (st_c + 1 == S) ? 0 : st_c + 1;
+            st_i = (st_i + 1 == S) ? 0 : st_i + 1;
+        }
+        __syncwarp();  // stash, tables and the dh slice are visible to the whole warp
+
+        float part = 0.f;
+        for (int k = lane; k < p.n; k += 32) part = fmaf(a_s[k], g_s[k], part);
+        const float gbar = warp_sum(part);
+        float dhv[E];
+        {
+            Frag<T, E> hf;
+            hf.a = ld_shared16(dhs_w + (uint32_t)(kp * 16));
+            hf.get(dhv);
+        }
+        for (int k = lane / nv; k < p.n; k += kst) {
+            Frag<T, E> kf, of;
+            kf.a = ld_shared16(stash(k, 0, kp));
+            if (ACC) of.a = ld_shared16(stash(k, 1, kp));
+            else of.zero();
+            const float a = a_s[k], s = s_s[k], rho = rho_s[k];
+            const float ds = a * (g_s[k] - gbar);
+            const float c1 = ds * rho, c2 = s * p.inv_r;
+            float kv[E], w[E];
+            kf.get(kv);
+            of.get(w);
+#pragma unroll
+            for (int t = 0; t < E; ++t) {
+                const float kbar = rho * kv[t];
+                const float dk = c1 * (q_s[j0 + t] - c2 * kbar);
+                dq_r[t] = fmaf(ds, kbar, dq_r[t]);
+                w[t] += fmaf(a, dhv[t], dk);
+            }
+            Frag<T, E> out;
+            out.set(w);
+            out.store(dst_row<T>(p.dvt, k, x, p.d) + tail0 + j0);
+        }
+        __syncwarp();  // the next token overwrites stash, tables and dh slice
+    }
+    cp_async_wait_all();
+    // lanes sharing a slice vector combine their dq parts with a fixed butterfly
+#pragma unroll
+    for (int t = 0; t < E; ++t)
+        for (int off = nv; off < 32; off <<= 1) dq_r[t] += __shfl_xor_sync(0xffffffffu, dq_r[t], off);
+    if (lane < nv)
+#pragma unroll
+        for (int t = 0; t < E; ++t) dq_all[warp * rp + j0 + t] = dq_r[t];
+    __syncthreads();
+    for (int j = threadIdx.x; j < p.r; j += kThreads) {
+        float acc = 0.f;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) acc += dq_all[w * rp + j];
+        p.partials[(int64_t)blockIdx.x * p.r + j] = acc;
+    }
+}
+
 // Full keys with gradients in another dtype than the inputs: rows loaded into
 // registers, U at a time.
 template <typename Tin, typename Tg, int V, int U>
@@ -946,6 +1180,35 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     size_t smem;
     int rq;
     constexpr bool kPipe = LRAR_BWD_PIPE && std::is_same<Tin, Tg>::value;
+    // Sliced keys with the forward's lse, gradients written (not accumulated):
+    // one pass over the values when the slice is whole vectors forming an
+    // aligned lane group (r / E divides 32, r divides d) and the per-warp stash
+    // fits in shared memory.  The accumulating form of the same kernel
+    // (ACC = true, equally exact) measured 2-3 % slower than the routing + value
+    // pass + key pass kernel at n = 49 on GB300 (one CTA per SM against two),
+    // so accumulating calls take bwd_lr_pipe_kernel.
+    if constexpr (kPipe && V <= 4) {
+        constexpr int OSN = OnePassStages<V, false>::value;
+        const int nvk = a.r / E;
+        if (a.variant == kSliced && a.lse && !a.accumulate && p.key_vec && nvk >= 1 && nvk <= 32 &&
+            32 % nvk == 0 && a.d % a.r == 0) {
+            const size_t smem1 = onepass_smem(OSN, 1, V, a.n, a.r, nvk);
+            int dev = 0, optin = 0;
+            cudaGetDevice(&dev);
+            cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+            if (smem1 <= (size_t)optin) {
+                const void *k1 = (const void *)bwd_slr_onepass_kernel<Tin, V, OSN, false>;
+                cudaError_t e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
+                if (e != cudaSuccess) return e;
+                const int grid = persistent_grid(k1, kThreads, smem1, work, kMaxPartials);
+                bwd_slr_onepass_kernel<Tin, V, OSN, false><<<grid, kThreads, smem1, s>>>(p);
+                e = cudaGetLastError();
+                if (e != cudaSuccess) return e;
+                dq_reduce_kernel<<<(a.r + 7) / 8, 256, 0, s>>>(a.partials, grid, a.r, a.dq, a.accumulate);
+                return cudaGetLastError();
+            }
+        }
+    }
     constexpr int SA = BwdStages<V, true>::value, SN = BwdStages<V, false>::value;
     // with dq in shared memory (V E > 32) the rings leave it room
     constexpr int FB = V * E > 32 ? 32 : 48;

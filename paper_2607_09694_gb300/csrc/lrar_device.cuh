@@ -63,6 +63,10 @@ __device__ __forceinline__ uint4 ld_shared16(uint32_t smem_addr) {
                  : "memory");
     return v;
 }
+__device__ __forceinline__ void st_shared16(uint32_t smem_addr, uint4 v) {
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(smem_addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

@@ -72,11 +72,13 @@ def sample_tokens(T: int, k: int = 48, seed: int = 0) -> np.ndarray:
 
 
 def run_gpu(si, out_dtype="f32", grad_dtype="f32", accumulate=False, init=None, n_src=None, eps=EPS,
-            stream=None, tokens=None):
+            stream=None, tokens=None, bwd_lse=True):
     """Forward + backward of one site through the C ABI.  `init` (dict of CPU
     tensors dvalues/dkeys/dq) seeds the gradient buffers when accumulating;
     otherwise they start as NaN so that any element left unwritten shows.
-    With `tokens`, only those token rows of h / lse / dvalues / dkeys come back."""
+    With `tokens`, only those token rows of h / lse / dvalues / dkeys come back.
+    bwd_lse=False calls the backward without the forward's lse (the sliced
+    backward then routes first and finishes the key slices in a second pass)."""
     dev = torch.device("cuda")
     n = si.n if n_src is None else n_src
     v = si.values.to(dev)
@@ -98,7 +100,7 @@ def run_gpu(si, out_dtype="f32", grad_dtype="f32", accumulate=False, init=None, 
         dq = torch.full((rq,), float("nan"), dtype=torch.float32, device=dev)
     ws = torch.empty(max(1, lrar.workspace_size(si.variant, n, T, d, si.r) // 4), dtype=torch.float32, device=dev)
     lrar.forward(si.variant, v, k, q, h, lse, n_src=n, r=si.r, eps=eps, stream=stream)
-    lrar.backward(si.variant, v, k, q, dh, dv, dq, ws, dkeys=dk, h=h, lse=lse, n_src=n, r=si.r,
+    lrar.backward(si.variant, v, k, q, dh, dv, dq, ws, dkeys=dk, h=h, lse=lse if bwd_lse else None, n_src=n, r=si.r,
                   accumulate=accumulate, eps=eps, stream=stream)
     torch.cuda.synchronize()
     if tokens is not None:

@@ -176,6 +176,32 @@ def test_sliced_key_widths(r, grad):
         _check(si, got, ref, si.n, "ulp")
 
 
+@pytest.mark.parametrize("r", [8, 16, 32])
+@pytest.mark.parametrize("accumulate", [False, True])
+@pytest.mark.parametrize("with_lse", [True, False])
+def test_sliced_one_pass_and_two_pass(r, accumulate, with_lse):
+    """Given the forward's lse, the writing sliced backward (one dtype for
+    inputs and gradients) takes one pass over the values: alpha_i =
+    exp(s_i - lse) from each row's own key slice, the slices finished from
+    shared memory once gbar is known.  Without lse, or when accumulating: a
+    routing stage, the value pass and a second pass over the key slices.  Both
+    round every bf16 gradient element once."""
+    si = synth.site("slr", n=49, T=333, r=r)
+    init = _init(si, dtype=torch.bfloat16) if accumulate else None
+    got = H.run_gpu(si, "bf16", "bf16", accumulate=accumulate, init=init, bwd_lse=with_lse)
+    _check(si, got, H.run_oracle(si), si.n, "ulp", init=init)
+
+
+@pytest.mark.parametrize("n,d,r", [(128, 1024, 16), (40, 512, 64), (7, 1000, 8), (3, 96, 32), (1, 256, 16)])
+def test_sliced_one_pass_shapes(n, d, r):
+    """The one-pass sliced backward at its edges: 128 sources (the per-warp
+    stash no longer fits shared memory, so two passes run), eight slice lanes
+    (r = 64 at d = 512), a row that does not fill the lanes' vectors
+    (d = 1000), a row of twelve vectors, and the single-source site."""
+    si = synth.site("slr", n=n, T=150, d=d, r=r)
+    _check(si, H.run_gpu(si, "bf16", "bf16"), H.run_oracle(si), si.n, "ulp")
+
+
 @pytest.mark.parametrize("r", [1, 4, 8, 16, 64])
 def test_projected_key_widths(r):
     si = synth.site("plr", n=12, T=260, r=r)

@@ -88,8 +88,8 @@ def test_sweep_equals_the_stacked_calls_and_its_graph():
         lrar.forward("sliced", v, None, qd[t - 1] if t > 1 else None, h[t - 1], lse[t - 1], n_src=t, r=r)
     dq.zero_()
     for t in range(n, 0, -1):
-        lrar.backward("sliced", v, None, qd[t - 1] if t > 1 else None, dhd[t - 1], dv, dq[t - 1], ws, n_src=t, r=r,
-                      accumulate=t != n)
+        lrar.backward("sliced", v, None, qd[t - 1] if t > 1 else None, dhd[t - 1], dv, dq[t - 1], ws, lse=lse[t - 1],
+                      n_src=t, r=r, accumulate=t != n)
     torch.cuda.synchronize()
     assert torch.equal(sw.h, h) and torch.equal(sw.lse, lse) and torch.equal(sw.dq, dq)
     assert torch.equal(torch.stack(sw.dsources), dv)
