@@ -405,7 +405,8 @@ def time_site(wl, n: int, accumulate: bool, reps: int):
 
 def run_profile_site(args):
     """Small single-site case for profilers: --profile-site n sources, --tokens T,
-    --site-variant / --site-d / --site-r (bf16 storage, accumulating backward)."""
+    --site-variant / --site-d / --site-r (bf16 storage; accumulating backward,
+    or with --site-write a backward that writes the gradients)."""
     import torch
 
     from __graft_entry__ import build
@@ -427,15 +428,17 @@ def run_profile_site(args):
     dq = torch.empty(r, device=dev)
     ws = torch.empty(max(1, lrar.workspace_size(variant, n, T, d, r) // 4), device=dev)
     fwd = lambda: lrar.forward(variant, vals, keys, q, h, lse, r=r)
-    bwd = lambda: lrar.backward(variant, vals, keys, q, dh, dv, dq, ws, dkeys=dk, h=h, lse=lse, r=r, accumulate=True)
+    acc = not args.site_write
+    bwd = lambda: lrar.backward(variant, vals, keys, q, dh, dv, dq, ws, dkeys=dk, h=h, lse=lse, r=r, accumulate=acc)
     for _ in range(args.warmup):
         fwd()
         bwd()
     f = _median_ms(torch, fwd, args.steps)
     b = _median_ms(torch, bwd, args.steps)
-    shp = sites.SiteShape(variant, n, T, d, r, out_bytes=2)
+    shp = sites.SiteShape(variant, n, T, d, r, out_bytes=2, accumulate=int(acc))
     fb, bb = sites.forward_bytes(shp), sites.backward_bytes(shp)
-    print(json.dumps({"profile_site": n, "variant": variant, "T": T, "d": d, "r": r, "fwd_ms": f, "bwd_ms": b,
+    print(json.dumps({"profile_site": n, "variant": variant, "T": T, "d": d, "r": r, "accumulate": int(acc),
+                      "fwd_ms": f, "bwd_ms": b,
                       "fwd_gbs": fb / f / 1e6, "bwd_gbs": bb / b / 1e6}), flush=True)
 
 
@@ -813,6 +816,7 @@ def main():
                     help="key variant of the --profile-site case")
     ap.add_argument("--site-d", type=int, default=D, help="width d of the --profile-site case")
     ap.add_argument("--site-r", type=int, default=R, help="key rank r of the --profile-site case (not full)")
+    ap.add_argument("--site-write", action="store_true", help="--profile-site: the backward writes the gradients")
     ap.add_argument("--suite", action="store_true", help="time every workload's headline site (JSON line each)")
     ap.add_argument("--profile-block", type=int, default=0,
                     help="time the Block two-phase path on this many tokens (profiling)")
