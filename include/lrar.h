@@ -79,7 +79,8 @@ enum lrar_status {
  *             (d <= 2048 for bfloat16 input, <= 1024 for float32)
  *   eps       RMSNorm epsilon, > 0
  *   h         [T, d] out_dtype, written
- *   lse       [T] float32, written when non-NULL (LRAR_FULL's backward needs it)
+ *   lse       [T] float32, written when non-NULL (LRAR_FULL's backward needs it;
+ *             LRAR_SLICED's writing backward uses it to skip its routing stage)
  *   stream    cudaStream_t
  */
 int lrar_forward(int variant, int in_dtype, int out_dtype, const void *values, const void *keys,
