@@ -242,3 +242,21 @@ def test_cuda_failures_surface_as_lrar_err_cuda(lib):
     assert b"cuda" in lib.lrar_last_error().lower()
     assert bwd(lib) == lrar.ERR_CUDA
     assert lib.lrar_project(1, FAKE, FAKE, 8, 64, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_CUDA
+
+
+def test_plain_c_client_compiles_links_and_runs(lib, tmp_path):
+    """tests/c_client.c includes include/lrar.h as C11 (-pedantic -Werror),
+    links against liblrar.so and gets INVALID_ARG back with a message."""
+    import shutil
+    import subprocess
+
+    if shutil.which("gcc") is None:
+        pytest.skip("no C compiler")
+    exe = str(tmp_path / "c_client")
+    libdir = os.path.dirname(lrar.LIB_PATH)
+    subprocess.run(["gcc", "-std=c11", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I", os.path.join(ROOT, "include"),
+                    os.path.join(ROOT, "tests", "c_client.c"), "-L", libdir, "-llrar", f"-Wl,-rpath,{libdir}",
+                    "-o", exe], check=True)
+    out = subprocess.run([exe], capture_output=True, text=True)
+    assert out.returncode == 0, out.stdout + out.stderr
+    assert "invalid argument" in out.stdout
