@@ -26,8 +26,10 @@
  *
  * Conventions shared by every entry point:
  *   - Calls are asynchronous and ordered on `stream` (a cudaStream_t; NULL is
- *     the legacy default stream).  No call synchronises the host, allocates
- *     memory or keeps state between calls; the library is thread-safe.
+ *     the legacy default stream).  No call synchronises the host or allocates
+ *     memory, and no call keeps state between calls except
+ *     lrar_backward_noalloc (its fixed scratch array and the cached address of
+ *     it, described there); the library is thread-safe.
  *   - Return value: LRAR_OK (0) or a negative LRAR_ERR_* code.  Argument
  *     checks run before anything is launched; on error nothing is launched and
  *     outputs are untouched.  lrar_last_error() gives a message for the
@@ -48,9 +50,18 @@
 extern "C" {
 #endif
 
-#define LRAR_VERSION 1
+#define LRAR_VERSION 2
 #define LRAR_MAX_SOURCES 128
 #define LRAR_MAX_BLOCK_SITES 64
+
+/*
+ * Bits a kernel may OR into a caller's optional device status word (the
+ * `status` arguments below).  The library never clears the word: the caller
+ * zeroes it, runs the calls, and reads it back when it wants to know.
+ */
+#define LRAR_STATUS_WAIT_TIMEOUT 1 /* a bounded wait inside a kernel gave up (about 2 s); outputs are invalid */
+#define LRAR_STATUS_LSE_MISMATCH 2 /* a backward that took alpha from a supplied lse found a token whose
+                                      weights sum to more than 1e-3 away from 1 (an lse of other inputs) */
 
 enum lrar_variant { LRAR_FULL = 0, LRAR_SLICED = 1, LRAR_PROJECTED = 2 };
 enum lrar_dtype { LRAR_F32 = 0, LRAR_BF16 = 1 };
@@ -130,12 +141,18 @@ size_t lrar_backward_workspace_size(int variant, int n_src, int64_t T, int d, in
  *              receives gradient from every later site)
  *   workspace  device scratch of at least lrar_backward_workspace_size() bytes,
  *              16-byte aligned; contents on entry are ignored
+ *   status     optional device int (4-byte aligned), may be NULL: where alpha is
+ *              taken from the supplied lse (LRAR_FULL; LRAR_SLICED's one-pass
+ *              form), each token checks that its weights sum to 1 within 1e-3 and
+ *              ORs LRAR_STATUS_LSE_MISMATCH in when they do not -- the sign of an
+ *              lse that belongs to other values or another query.  The gradients
+ *              are then not valid.  Never written otherwise.
  *   Other arguments as for lrar_forward.  values, dvalues and dkeys must not overlap.
  */
 int lrar_backward(int variant, int in_dtype, int grad_dtype, const void *values, const void *keys,
                   const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh,
                   const void *h, int h_dtype, const float *lse, void *dvalues, void *dkeys, float *dq,
-                  int accumulate, void *workspace, size_t workspace_bytes, void *stream);
+                  int accumulate, void *workspace, size_t workspace_bytes, int *status, void *stream);
 
 /*
  * lrar_backward for callers that cannot allocate device memory.  The paper has
@@ -151,18 +168,24 @@ int lrar_backward(int variant, int in_dtype, int grad_dtype, const void *values,
  *   - Problems whose workspace would exceed 4 MiB (lrar_backward_workspace_size()
  *     > 4 MiB, i.e. a dq width -- r, or d for LRAR_FULL -- above 1024) are
  *     rejected with LRAR_ERR_UNSUPPORTED before anything runs.
- *   - The first call on each device looks up the scratch's device address with
- *     that device current; make that first call before any stream capture.
+ *   - The first call on each device that passes the argument checks looks up
+ *     the scratch's device address with that device current, and keeps it for
+ *     the life of the process; make that first call before any stream capture.
+ *     A reset of the device (cudaDeviceReset, or a reset of its primary
+ *     context) invalidates the kept address: do not use this call on a device
+ *     after such a reset.
  *   - All calls on a device share the one scratch array.  None of it needs to
  *     start at zero (every partial sum is written before it is read), but calls
  *     that may run at the same time on the GPU (different streams, or host
  *     threads without ordering between them) race on it: serialise them.
- * Results, errors and all other rules are those of lrar_backward.
+ * Results, errors and all other rules are those of lrar_backward; arguments
+ * are checked (with lrar_backward's codes and messages) before the device is
+ * touched.
  */
 int lrar_backward_noalloc(int variant, int in_dtype, int grad_dtype, const void *values, const void *keys,
                           const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh,
                           const void *h, int h_dtype, const float *lse, void *dvalues, void *dkeys, float *dq,
-                          int accumulate, void *stream);
+                          int accumulate, int *status, void *stream);
 
 /*
  * Block AttnRes source assembly (§3.1, Eq. 5-6) and its gradient fan-out:
@@ -199,6 +222,12 @@ int lrar_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *s
  *               sources only (float32 keeps phase 2 exact; bfloat16 rounds it)
  *   lse_pre     [n_sites, T] float32, written: log sum_i exp(score) over them
  *   n_sites     1..LRAR_MAX_BLOCK_SITES
+ *   status      optional device int (4-byte aligned), may be NULL: the kernel
+ *               stages each token's keys with bulk copies and waits for them
+ *               with a bound (about 2 s); a wait that runs out ORs
+ *               LRAR_STATUS_WAIT_TIMEOUT in, stops the launch's further copies,
+ *               and the launch drains the copies in flight and returns (h_pre
+ *               and lse_pre are then not valid).  Never written otherwise.
  * Phase 2 (one site):
  *   h_pre, lse_pre  that site's rows of the phase-1 outputs ([T, d], [T])
  *   partial     [T, d] in_dtype: the partial-block summary (for the first site
@@ -210,7 +239,7 @@ int lrar_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *s
  */
 int lrar_block_phase1(int variant, int in_dtype, int pre_dtype, const void *values, const void *keys,
                       const float *queries, int n_completed, int n_sites, int64_t T, int d, int r, float eps,
-                      void *h_pre, float *lse_pre, void *stream);
+                      void *h_pre, float *lse_pre, int *status, void *stream);
 int lrar_block_phase2(int variant, int in_dtype, int pre_dtype, int out_dtype, const void *h_pre,
                       const float *lse_pre, const void *partial, const void *partial_key, const float *query,
                       int64_t T, int d, int r, float eps, void *h, float *lse, void *stream);
@@ -255,7 +284,7 @@ int lrar_backward_ptrs(int variant, int in_dtype, int grad_dtype, const void *co
                        const void *const *keys, const float *query, int n_src, int64_t T, int d, int r, float eps,
                        const void *dh, const void *h, int h_dtype, const float *lse, void *const *dvalues,
                        void *const *dkeys, float *dq, int accumulate, void *workspace, size_t workspace_bytes,
-                       void *stream);
+                       int *status, void *stream);
 
 /*
  * P-LR fused output projection (§3.3, Eq. 11-12) on the tensor cores:
@@ -269,9 +298,9 @@ int lrar_backward_ptrs(int variant, int in_dtype, int grad_dtype, const void *co
  *           (m = d for attention, the SwiGLU hidden width for the FFN)
  *   w       [d + r, m] row-major: the d rows of W_O, then the r rows of W_K
  *   o       [T, d] (may be NULL when d == 0);  keys [T, r] (NULL when r == 0)
- *   status  optional device int: set to 1 if a pipeline wait inside the kernel
- *           gave up (about 2 s; then the outputs are not valid).  Never written
- *           otherwise, so the caller zeroes it beforehand.
+ *   status  optional device int (4-byte aligned): LRAR_STATUS_WAIT_TIMEOUT is
+ *           ORed in if a pipeline wait inside the kernel gave up (about 2 s; the
+ *           outputs are then not valid).  Never written otherwise.
  * in_dtype must be LRAR_BF16 (LRAR_ERR_UNSUPPORTED otherwise); m, d and r must
  * be multiples of 8 and a, w, o, keys 16-byte aligned (LRAR_ERR_ALIGNMENT).
  * T == 0 is a no-op.  No counterpart of the depth mix's other rules: the call

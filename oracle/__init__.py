@@ -50,7 +50,7 @@ def _load():
             vp, i64p, dp = ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p
             i, i64, dbl = ctypes.c_int, ctypes.c_int64, ctypes.c_double
             lib.oracle_forward.argtypes = [i, i, vp, vp, dp, i, i64, i, i, dbl, i64p, i64, dp, dp, dp]
-            lib.oracle_backward.argtypes = [i, i, vp, vp, dp, i, i64, i, i, dbl, vp, i64p, i64, dp, dp, dp, dp]
+            lib.oracle_backward.argtypes = [i, i, vp, vp, dp, i, i64, i, i, dbl, vp, i64p, i64, dp, dp, dp, dp, dp]
             lib.oracle_diagnostics.argtypes = [i, i, vp, vp, dp, i, i64, i, i, dbl, i64p, i64, dp, dp]
             lib.oracle_block_sources.argtypes = [i, vp, i, i64, i, i, dp]
             lib.oracle_block_fanout.argtypes = [dp, i, i64, i, i, dp]
@@ -142,7 +142,9 @@ def forward(variant, values, keys, q, eps, r=None, tokens=None, want_alpha=False
 
 
 def backward(variant, values, keys, q, eps, dh, r=None, tokens=None, want_dvalues=True, want_ds=False):
-    """Gradients of sum <dh, h>: dict(dvalues [n,n_tok,d], dkeys [n,n_tok,r], dq [r], ds [n_tok,n])."""
+    """Gradients of sum <dh, h>: dict(dvalues [n,n_tok,d], dkeys [n,n_tok,r], dq [r], ds [n_tok,n],
+    dq_abs [r]).  dq_abs[j] = sum over tokens and sources of |ds_i kbar_ij|, the
+    magnitude of the terms that dq[j] sums (what bounds the rounding of that sum)."""
     va, dt = _as_array(values)
     ka, kdt = _as_array(keys)
     da, ddt = _as_array(dh)
@@ -156,12 +158,13 @@ def backward(variant, values, keys, q, eps, dh, r=None, tokens=None, want_dvalue
     dv = np.zeros((n, n_tok, d)) if want_dvalues else None
     dk = np.zeros((n, n_tok, r)) if variant == PROJECTED else None
     dq = np.zeros(r)
+    dq_abs = np.zeros(r)
     ds = np.zeros((n_tok, n)) if want_ds else None
     rc = _load().oracle_backward(variant, dt, _ptr(va), _ptr(ka), _ptr(qa), n, T, d, r, float(eps), _ptr(da),
-                                 _ptr(tk), n_tok, _ptr(dv), _ptr(dk), _ptr(dq), _ptr(ds))
+                                 _ptr(tk), n_tok, _ptr(dv), _ptr(dk), _ptr(dq), _ptr(ds), _ptr(dq_abs))
     if rc != 0:
         raise ValueError("oracle_backward rejected its arguments")
-    return {"dvalues": dv, "dkeys": dk, "dq": dq, "ds": ds}
+    return {"dvalues": dv, "dkeys": dk, "dq": dq, "ds": ds, "dq_abs": dq_abs}
 
 
 def diagnostics(variant, values, keys, q, eps, r=None, tokens=None):

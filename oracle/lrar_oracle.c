@@ -229,18 +229,21 @@ int oracle_forward(int variant, int dtype, const void *values, const void *keys,
 int oracle_backward(int variant, int dtype, const void *values, const void *keys, const double *q,
                     int n, int64_t T, int d, int r, double eps, const void *dh,
                     const int64_t *tokens, int64_t n_tok,
-                    double *dvalues, double *dkeys, double *dq, double *ds) {
+                    double *dvalues, double *dkeys, double *dq, double *ds, double *dq_abs) {
     if (check_args(variant, dtype, values, keys, q, n, T, d, r, eps) || !dh) return -1;
     if (!tokens) n_tok = T;
     if (n_tok < 0) return -1;
     int nt = nthreads();
-    double *dq_part = calloc((size_t)nt * r, sizeof(double));
+    /* per thread: r partial sums of dq, then r sums of |ds_i kbar_ij| (the
+     * magnitude of the terms dq adds up, for judging its rounding) */
+    double *dq_part = calloc((size_t)nt * 2 * r, sizeof(double));
     if (!dq_part) return -1;
     int err = 0;
 #pragma omp parallel reduction(| : err)
     {
         scratch_t w;
-        double *dqp = dq_part + (size_t)thread_id() * r;
+        double *dqp = dq_part + (size_t)thread_id() * 2 * r;
+        double *dqa = dqp + r;
         int ok = scratch_alloc(&w, n, d, r) == 0;
         if (!ok) err |= 1;
         /* every thread reaches the work-sharing loop, even without scratch */
@@ -274,7 +277,10 @@ int oracle_backward(int variant, int dtype, const void *values, const void *keys
                     const double *kbi = w.kbar + (size_t)i * r;
                     double rho = w.rho[i];
                     /* Score s_i = q . kbar_i: dL/dq += ds_i kbar_i, dL/dkbar_i = ds_i q. */
-                    for (int j = 0; j < r; ++j) dqp[j] += w.ds[i] * kbi[j];
+                    for (int j = 0; j < r; ++j) {
+                        dqp[j] += w.ds[i] * kbi[j];
+                        dqa[j] += fabs(w.ds[i] * kbi[j]);
+                    }
                     /* Eq. (8), RMSNorm: kbar = rho k with rho = (k.k/r + eps)^(-1/2),
                      * so d kbar_a / d k_b = rho [a==b] + k_a drho/dk_b and
                      * drho/dk_b = -rho^3 k_b / r.  Apply the transpose to dkbar. */
@@ -296,12 +302,14 @@ int oracle_backward(int variant, int dtype, const void *values, const void *keys
         }
         scratch_free(&w);
     }
-    if (dq) {
-        for (int j = 0; j < r; ++j) {
-            double acc = 0.0;
-            for (int t = 0; t < nt; ++t) acc += dq_part[(size_t)t * r + j];
-            dq[j] = acc;
+    for (int j = 0; j < r; ++j) {
+        double acc = 0.0, mag = 0.0;
+        for (int t = 0; t < nt; ++t) {
+            acc += dq_part[(size_t)t * 2 * r + j];
+            mag += dq_part[(size_t)t * 2 * r + r + j];
         }
+        if (dq) dq[j] = acc;
+        if (dq_abs) dq_abs[j] = mag;
     }
     free(dq_part);
     return err ? -1 : 0;

@@ -28,7 +28,8 @@ def _nvcc() -> str:
 
 def _inputs() -> list[str]:
     files = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".cu", ".cuh", ".h"))]
-    return files + [os.path.join(INCLUDE, "lrar.h"), os.path.abspath(__file__)]
+    headers = [os.path.join(INCLUDE, f) for f in os.listdir(INCLUDE) if f.endswith(".h")]
+    return files + headers + [os.path.abspath(__file__)]
 
 
 def stale() -> bool:

@@ -9,6 +9,7 @@
 #include <unordered_map>
 
 #include "lrar.h"
+#include "lrar_testing.h"
 #include "lrar_device.cuh"
 #include "lrar_launch.h"
 
@@ -166,17 +167,25 @@ int forward_impl(int variant, int in_dtype, int out_dtype, const void *const *va
     return LRAR_OK;
 }
 
-// Checks of the backward that do not depend on how the sources are passed;
-// returns 1 (with *early set to the status) when nothing is left to launch.
-int backward_common(int variant, int in_dtype, int grad_dtype, int n_src, int64_t T, int d, int r, float eps,
-                    int h_dtype, float *dq, int accumulate, void *stream, bool *done) {
-    *done = false;
+// Scalar checks of the backward (every form of it).
+int backward_scalars(int variant, int in_dtype, int grad_dtype, int n_src, int64_t T, int d, int r, float eps,
+                     int h_dtype, float *dq, int accumulate) {
     int rc = check_shape(variant, in_dtype, n_src, T, d, r, eps);
     if (rc) return rc;
     if (!dtype_ok(grad_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown gradient dtype %d", grad_dtype);
     if (accumulate != 0 && accumulate != 1) return fail(LRAR_ERR_INVALID_ARG, "accumulate must be 0 or 1");
     if (variant == LRAR_FULL && !dtype_ok(h_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown h dtype %d", h_dtype);
     if (!dq) return fail(LRAR_ERR_INVALID_ARG, "dq is required");
+    return LRAR_OK;
+}
+
+// Checks of the backward that do not depend on how the sources are passed;
+// returns 1 (with *early set to the status) when nothing is left to launch.
+int backward_common(int variant, int in_dtype, int grad_dtype, int n_src, int64_t T, int d, int r, float eps,
+                    int h_dtype, float *dq, int accumulate, void *stream, bool *done) {
+    *done = false;
+    int rc = backward_scalars(variant, in_dtype, grad_dtype, n_src, T, d, r, eps, h_dtype, dq, accumulate);
+    if (rc) return rc;
     if (T == 0) {  // dq is a sum over no tokens
         *done = true;
         if (!accumulate) {
@@ -188,17 +197,36 @@ int backward_common(int variant, int in_dtype, int grad_dtype, int n_src, int64_
     return LRAR_OK;
 }
 
-int backward_impl(int variant, int in_dtype, int grad_dtype, const void *const *values, const void *const *keys,
-                  const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh, const void *h,
-                  int h_dtype, const float *lse, void *const *dvalues, void *const *dkeys, float *dq,
-                  int accumulate, void *workspace, size_t workspace_bytes, void *stream) {
+// Pointer checks of the backward's per-call tensors (dh, h, lse, query, dq).
+int backward_tensors(int variant, const float *query, int n_src, const void *dh, const void *h, const float *lse,
+                     const float *dq, const int *status) {
     if (!dh) return fail(LRAR_ERR_INVALID_ARG, "dh is required");
     if (variant == LRAR_FULL && (!h || !lse))
         return fail(LRAR_ERR_INVALID_ARG, "full AttnRes backward needs the forward's h and lse");
     if (!query && n_src > 1) return fail(LRAR_ERR_INVALID_ARG, "query is required when n_src > 1");
     if (!aligned16(dh) || !aligned4(dq) || (variant == LRAR_FULL && !aligned16(h)) || (lse && !aligned4(lse)) ||
-        (query && !aligned4(query)))
+        (query && !aligned4(query)) || (status && !aligned4(status)))
+        return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (query, lse, dq and status 4-byte)");
+    return LRAR_OK;
+}
+
+// Pointer checks of the stacked backward's source and gradient buffers.
+int backward_stacks(int variant, const void *values, const void *keys, const void *dvalues, const void *dkeys) {
+    if (!values || !dvalues) return fail(LRAR_ERR_INVALID_ARG, "values, dh and dvalues are required");
+    if (variant == LRAR_PROJECTED && (!keys || !dkeys))
+        return fail(LRAR_ERR_INVALID_ARG, "projected keys and dkeys are required");
+    if (!aligned16(values) || !aligned16(dvalues) ||
+        (variant == LRAR_PROJECTED && (!aligned16(keys) || !aligned16(dkeys))))
         return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (query, lse and dq 4-byte)");
+    return LRAR_OK;
+}
+
+int backward_impl(int variant, int in_dtype, int grad_dtype, const void *const *values, const void *const *keys,
+                  const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh, const void *h,
+                  int h_dtype, const float *lse, void *const *dvalues, void *const *dkeys, float *dq,
+                  int accumulate, void *workspace, size_t workspace_bytes, int *status, void *stream) {
+    int rc = backward_tensors(variant, query, n_src, dh, h, lse, dq, status);
+    if (rc) return rc;
     if (!workspace || workspace_bytes < lrar_backward_workspace_size(variant, n_src, T, d, r))
         return fail(LRAR_ERR_WORKSPACE, "workspace needs %zu bytes (got %zu)",
                     lrar_backward_workspace_size(variant, n_src, T, d, r), workspace ? workspace_bytes : (size_t)0);
@@ -224,6 +252,7 @@ int backward_impl(int variant, int in_dtype, int grad_dtype, const void *const *
     a.dq = dq;
     a.accumulate = accumulate;
     a.partials = static_cast<float *>(workspace);
+    a.status = status;
     cudaError_t e = lrar::launch_backward(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "lrar_backward");
     return LRAR_OK;
@@ -271,17 +300,12 @@ LRAR_API size_t lrar_backward_workspace_size(int variant, int n_src, int64_t T, 
 LRAR_API int lrar_backward(int variant, int in_dtype, int grad_dtype, const void *values, const void *keys,
                            const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh,
                            const void *h, int h_dtype, const float *lse, void *dvalues, void *dkeys, float *dq,
-                           int accumulate, void *workspace, size_t workspace_bytes, void *stream) {
+                           int accumulate, void *workspace, size_t workspace_bytes, int *status, void *stream) {
     bool done;
     int rc = backward_common(variant, in_dtype, grad_dtype, n_src, T, d, r, eps, h_dtype, dq, accumulate, stream,
                              &done);
     if (rc || done) return rc;
-    if (!values || !dvalues) return fail(LRAR_ERR_INVALID_ARG, "values, dh and dvalues are required");
-    if (variant == LRAR_PROJECTED && (!keys || !dkeys))
-        return fail(LRAR_ERR_INVALID_ARG, "projected keys and dkeys are required");
-    if (!aligned16(values) || !aligned16(dvalues) ||
-        (variant == LRAR_PROJECTED && (!aligned16(keys) || !aligned16(dkeys))))
-        return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (query, lse and dq 4-byte)");
+    if ((rc = backward_stacks(variant, values, keys, dvalues, dkeys))) return rc;
     const int esz = esize(in_dtype), gsz = esize(grad_dtype);
     const void *vt[LRAR_MAX_SOURCES], *kt[LRAR_MAX_SOURCES], *dvt[LRAR_MAX_SOURCES], *dkt[LRAR_MAX_SOURCES];
     const bool pl = variant == LRAR_PROJECTED;
@@ -291,14 +315,29 @@ LRAR_API int lrar_backward(int variant, int in_dtype, int grad_dtype, const void
     stack_table(pl ? dkeys : nullptr, n_src, T, r, gsz, dkt);
     return backward_impl(variant, in_dtype, grad_dtype, vt, kt, query, n_src, T, d, r, eps, dh, h, h_dtype, lse,
                          const_cast<void *const *>(dvt), const_cast<void *const *>(dkt), dq, accumulate, workspace,
-                         workspace_bytes, stream);
+                         workspace_bytes, status, stream);
 }
+
+namespace lrar {
+
+int check_backward(int variant, int in_dtype, int grad_dtype, const void *values, const void *keys,
+                   const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh, const void *h,
+                   int h_dtype, const float *lse, const void *dvalues, const void *dkeys, const float *dq,
+                   int accumulate, const int *status) {
+    int rc = backward_scalars(variant, in_dtype, grad_dtype, n_src, T, d, r, eps, h_dtype, const_cast<float *>(dq),
+                              accumulate);
+    if (rc || T == 0) return rc;
+    if ((rc = backward_stacks(variant, values, keys, dvalues, dkeys))) return rc;
+    return backward_tensors(variant, query, n_src, dh, h, lse, dq, status);
+}
+
+}  // namespace lrar
 
 LRAR_API int lrar_backward_ptrs(int variant, int in_dtype, int grad_dtype, const void *const *values,
                                 const void *const *keys, const float *query, int n_src, int64_t T, int d, int r,
                                 float eps, const void *dh, const void *h, int h_dtype, const float *lse,
                                 void *const *dvalues, void *const *dkeys, float *dq, int accumulate, void *workspace,
-                                size_t workspace_bytes, void *stream) {
+                                size_t workspace_bytes, int *status, void *stream) {
     bool done;
     int rc = backward_common(variant, in_dtype, grad_dtype, n_src, T, d, r, eps, h_dtype, dq, accumulate, stream,
                              &done);
@@ -310,7 +349,7 @@ LRAR_API int lrar_backward_ptrs(int variant, int in_dtype, int grad_dtype, const
         if ((rc = check_table(const_cast<const void *const *>(dkeys), n_src, "dkeys"))) return rc;
     }
     return backward_impl(variant, in_dtype, grad_dtype, values, keys, query, n_src, T, d, r, eps, dh, h, h_dtype, lse,
-                         dvalues, dkeys, dq, accumulate, workspace, workspace_bytes, stream);
+                         dvalues, dkeys, dq, accumulate, workspace, workspace_bytes, status, stream);
 }
 
 LRAR_API size_t lrar_diagnostics_workspace_size(int n_src) {
@@ -363,9 +402,11 @@ LRAR_API int lrar_diagnostics(int variant, int in_dtype, const void *values, con
     return LRAR_OK;
 }
 
-LRAR_API int lrar_block_phase1(int variant, int in_dtype, int pre_dtype, const void *values, const void *keys,
-                               const float *queries, int n_completed, int n_sites, int64_t T, int d, int r, float eps,
-                               void *h_pre, float *lse_pre, void *stream) {
+namespace {
+
+int block_phase1_impl(int variant, int in_dtype, int pre_dtype, const void *values, const void *keys,
+                      const float *queries, int n_completed, int n_sites, int64_t T, int d, int r, float eps,
+                      void *h_pre, float *lse_pre, int *status, long long wait_cycles, bool stall, void *stream) {
     if (variant == LRAR_FULL)
         return fail(LRAR_ERR_UNSUPPORTED, "the two-phase block path serves low-rank keys (sliced, projected)");
     int rc = check_shape(variant, in_dtype, n_completed, T, d, r, eps);
@@ -373,6 +414,7 @@ LRAR_API int lrar_block_phase1(int variant, int in_dtype, int pre_dtype, const v
     if (!dtype_ok(pre_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown phase-1 output dtype %d", pre_dtype);
     if (n_sites < 1 || n_sites > LRAR_MAX_BLOCK_SITES)
         return fail(LRAR_ERR_INVALID_ARG, "n_sites must be in 1..%d (got %d)", LRAR_MAX_BLOCK_SITES, n_sites);
+    if (status && !aligned4(status)) return fail(LRAR_ERR_ALIGNMENT, "status must be 4-byte aligned");
     if (T == 0) return LRAR_OK;
     if (!values || !queries || !h_pre || !lse_pre)
         return fail(LRAR_ERR_INVALID_ARG, "values, queries, h_pre and lse_pre are required");
@@ -395,9 +437,34 @@ LRAR_API int lrar_block_phase1(int variant, int in_dtype, int pre_dtype, const v
     a.eps = eps;
     a.h_pre = h_pre;
     a.lse_pre = lse_pre;
+    a.status = status;
+    a.wait_cycles = wait_cycles;
+    a.stall = stall;
+    if (stall && !lrar::block_phase1_stages_keys(a))
+        return fail(LRAR_ERR_UNSUPPORTED, "this shape reads keys from global memory: no waits to stall");
     cudaError_t e = lrar::launch_block_phase1(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "lrar_block_phase1");
     return LRAR_OK;
+}
+
+}  // namespace
+
+LRAR_API int lrar_block_phase1(int variant, int in_dtype, int pre_dtype, const void *values, const void *keys,
+                               const float *queries, int n_completed, int n_sites, int64_t T, int d, int r, float eps,
+                               void *h_pre, float *lse_pre, int *status, void *stream) {
+    return block_phase1_impl(variant, in_dtype, pre_dtype, values, keys, queries, n_completed, n_sites, T, d, r, eps,
+                             h_pre, lse_pre, status, lrar::kWaitCycles, false, stream);
+}
+
+LRAR_API int lrar_test_block_phase1_stalled(int variant, int in_dtype, int pre_dtype, const void *values,
+                                            const void *keys, const float *queries, int n_completed, int n_sites,
+                                            int64_t T, int d, int r, float eps, void *h_pre, float *lse_pre,
+                                            int *status, long long wait_cycles, void *stream) {
+    if (!status) return fail(LRAR_ERR_INVALID_ARG, "the stalled phase 1 reports through status: it is required");
+    if (wait_cycles < 1 || wait_cycles > (1LL << 32))
+        return fail(LRAR_ERR_INVALID_ARG, "wait_cycles must be in 1 .. 2^32");
+    return block_phase1_impl(variant, in_dtype, pre_dtype, values, keys, queries, n_completed, n_sites, T, d, r, eps,
+                             h_pre, lse_pre, status, wait_cycles, true, stream);
 }
 
 LRAR_API int lrar_block_phase2(int variant, int in_dtype, int pre_dtype, int out_dtype, const void *h_pre,
@@ -438,8 +505,10 @@ LRAR_API int lrar_block_phase2(int variant, int in_dtype, int pre_dtype, int out
     return LRAR_OK;
 }
 
-LRAR_API int lrar_project(int in_dtype, const void *a, const void *w, int64_t T, int m, int d, int r, void *o,
-                          void *keys, int *status, void *stream) {
+namespace {
+
+int project_impl(int tile, int in_dtype, const void *a, const void *w, int64_t T, int m, int d, int r, void *o,
+                 void *keys, int *status, void *stream) {
     if (!dtype_ok(in_dtype)) return fail(LRAR_ERR_INVALID_ARG, "unknown input dtype %d", in_dtype);
     if (in_dtype != LRAR_BF16) return fail(LRAR_ERR_UNSUPPORTED, "lrar_project takes bfloat16 operands");
     if (T < 0 || m < 1 || d < 0 || r < 0 || d + r < 1)
@@ -453,8 +522,23 @@ LRAR_API int lrar_project(int in_dtype, const void *a, const void *w, int64_t T,
     if (!aligned16(a) || !aligned16(w) || (o && !aligned16(o)) || (keys && !aligned16(keys)))
         return fail(LRAR_ERR_ALIGNMENT, "a, w, o and keys must be 16-byte aligned");
     if (status && !aligned4(status)) return fail(LRAR_ERR_ALIGNMENT, "status must be 4-byte aligned");
+    if (tile != 0 && !lrar::project_tile_ok(tile))
+        return fail(LRAR_ERR_INVALID_ARG, "tile must be 160, 176, 192, 224, 240 or 256 (got %d)", tile);
     if (T == 0) return LRAR_OK;
-    return lrar::launch_project(a, w, T, m, d, r, o, keys, status, static_cast<cudaStream_t>(stream));
+    return lrar::launch_project(a, w, T, m, d, r, o, keys, status, tile, static_cast<cudaStream_t>(stream));
+}
+
+}  // namespace
+
+LRAR_API int lrar_project(int in_dtype, const void *a, const void *w, int64_t T, int m, int d, int r, void *o,
+                          void *keys, int *status, void *stream) {
+    return project_impl(0, in_dtype, a, w, T, m, d, r, o, keys, status, stream);
+}
+
+LRAR_API int lrar_test_project_tile(int tile, int in_dtype, const void *a, const void *w, int64_t T, int m, int d,
+                                    int r, void *o, void *keys, int *status, void *stream) {
+    if (tile == 0) return fail(LRAR_ERR_INVALID_ARG, "tile must be 160, 176, 192, 224, 240 or 256 (got 0)");
+    return project_impl(tile, in_dtype, a, w, T, m, d, r, o, keys, status, stream);
 }
 
 LRAR_API int lrar_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *src, int64_t count,

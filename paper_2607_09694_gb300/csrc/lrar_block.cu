@@ -18,6 +18,7 @@
 // element.  The chunk warps split the c queries for scoring and share the
 // weights through shared memory (double-buffered, one named barrier per pass),
 // and each pass scores the next token while the current token's rows load.
+#include "lrar.h"
 #include "lrar_device.cuh"
 #include "lrar_launch.h"
 #include "lrar_sm100.cuh"
@@ -36,6 +37,9 @@ struct Ph1Params {
     int n, c, d, r, chunks;
     float eps, inv_r;
     int sliced, key_vec;
+    int *status;            // optional: LRAR_STATUS_WAIT_TIMEOUT when a key wait gives up
+    long long wait_cycles;  // bound of each key wait
+    int stall;              // test hook: key waits go to a barrier that never completes
 };
 
 __device__ __forceinline__ void group_sync(int id, int threads) {
@@ -165,7 +169,16 @@ __device__ __forceinline__ void ph1_score(const Ph1Params &p, const float *__res
 // tokens, so the loads of the next token's rows overlap this token's mix.
 // KS: each group's keys are staged two tokens ahead in shared memory with
 // bulk copies (double-buffered, one mbarrier per buffer), so scoring reads no
-// global memory.
+// global memory.  Each wait for them is bounded (p.wait_cycles) and decided
+// for the whole warp; one that runs out ORs LRAR_STATUS_WAIT_TIMEOUT into
+// *p.status and raises the CTA's abort flag, after which no warp waits again
+// and no group issues another copy (a group's copy into a buffer follows the
+// barrier that ends the pass in which its warps waited for that buffer's
+// previous token, so a give-up is seen before the buffer is reused).  The
+// issuing warp counts the phases it issued and saw complete per buffer (at
+// most one per buffer is left unconfirmed after a give-up) and waits, bounded,
+// for that one before the CTA exits, so no copy lands in freed shared memory.
+// The outputs of a launch that gave up are not valid.
 // C8: exactly eight sites per launch (compile-time loop bounds); else p.c <= 8.
 template <typename Tin, typename Tout, int S, bool KS, bool C8>
 __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_constant__ Ph1Params p) {
@@ -182,10 +195,20 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
     const int G = kWarps / p.chunks;  // tokens per CTA pass
     const int g = warp / p.chunks, ch = warp % p.chunks;
     const int nthr = p.chunks * 32;   // threads of a token group (named barrier 1 + g)
+    __shared__ int abort_s;           // set once a key wait of this CTA gave up
+    __shared__ __align__(8) uint64_t never_bar;  // test hook: a barrier nothing arrives on
+    volatile int *abort = &abort_s;
     for (int j = threadIdx.x; j < p.c * p.r; j += kThreads) q_s[(j / p.r) * rp + j % p.r] = p.queries[j];
     if (KS && threadIdx.x < 2 * G) {
         sm100::mbar_init(smem_u32(kbar_all + threadIdx.x), 1);
         sm100::mbar_fence_init();
+    }
+    if (threadIdx.x == 0) {
+        abort_s = 0;
+        if (KS) {
+            sm100::mbar_init(smem_u32(&never_bar), 1);
+            sm100::mbar_fence_init();
+        }
     }
     __syncthreads();
 
@@ -198,8 +221,31 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
     unsigned char *kb0 = kb_all + (size_t)g * 2 * kbuf_bytes;
     auto kbuf = [&](int b) { return smem_u32(kb0 + b * kbuf_bytes); };
     auto kbar = [&](int b) { return smem_u32(kbar_all + 2 * g + b); };
-    // token q of this group (x0 + q * stride) uses key buffer q % 2, for the (q / 2)-th time
-    auto kwait = [&](int q) { sm100::mbar_wait(kbar(q & 1), (uint32_t)(q >> 1) & 1u, 4LL << 30); };
+    // token q of this group (x0 + q * stride) uses key buffer q % 2, for the (q / 2)-th time;
+    // the issuing warp (ch == 0) counts phases issued and seen complete per buffer
+    uint32_t issued0 = 0u, issued1 = 0u, seen0 = 0u, seen1 = 0u;
+    auto kwait = [&](int q) {
+        if (__any_sync(0xffffffffu, *abort != 0)) return;  // the CTA gave up: no further waits (warp-uniform)
+        const uint32_t bar = p.stall ? smem_u32(&never_bar) : kbar(q & 1);
+        const uint32_t par = p.stall ? 0u : (uint32_t)(q >> 1) & 1u;
+        const bool ok = __all_sync(0xffffffffu, sm100::mbar_wait(bar, par, p.wait_cycles, abort));
+        if (ok) {
+            if (ch == 0) {
+                if (q & 1) seen1 = (uint32_t)(q >> 1) + 1u;
+                else seen0 = (uint32_t)(q >> 1) + 1u;
+            }
+        } else if (lane == 0) {
+            *abort = 1;
+            if (p.status) atomicOr(p.status, LRAR_STATUS_WAIT_TIMEOUT);
+        }
+    };
+    // the issuing warp stages token xx into buffer b unless the CTA gave up (warp-uniform)
+    auto stage = [&](int64_t xx, int b) {
+        if (__any_sync(0xffffffffu, *abort != 0)) return;
+        ph1_stage<Tin>(p, xx, lane, kbuf(b), kbar(b));
+        if (b) ++issued1;
+        else ++issued0;
+    };
 
     int64_t x = (int64_t)blockIdx.x * G + g;
     int64_t ix = x;  // next row to copy: source ii of token ix
@@ -219,8 +265,8 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
     int st_c = 0, st_i = S - 1;
 
     if (KS && ch == 0) {
-        if (x < p.T) ph1_stage<Tin>(p, x, lane, kbuf(0), kbar(0));
-        if (x + stride < p.T) ph1_stage<Tin>(p, x + stride, lane, kbuf(1), kbar(1));
+        if (x < p.T) stage(x, 0);
+        if (x + stride < p.T) stage(x + stride, 1);
     }
     if (x < p.T) {
         if (KS) kwait(0);
@@ -231,7 +277,7 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
         const float *aw = aw0 + (pass & 1) * kPh1MaxSites * p.n;
         float *aw_next = aw0 + ((pass + 1) & 1) * kPh1MaxSites * p.n;
         // buffer pass % 2 held token `pass`, scored by every warp before the last barrier
-        if (KS && ch == 0 && x + 2 * stride < p.T) ph1_stage<Tin>(p, x + 2 * stride, lane, kbuf(pass & 1), kbar(pass & 1));
+        if (KS && ch == 0 && x + 2 * stride < p.T) stage(x + 2 * stride, pass & 1);
         if (x + stride < p.T) {
             if (KS) kwait(pass + 1);
             ph1_score<Tin>(p, q_s, rp, x + stride, ch, lane, aw_next, KS ? kb0 + ((pass + 1) & 1) * kbuf_bytes : nullptr);
@@ -277,6 +323,13 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
         group_sync(1 + g, nthr);  // next weights complete; this pass's weights free for reuse
     }
     cp_async_wait_all();
+    if (KS && ch == 0)  // drain: the one phase per buffer a give-up may have left unconfirmed
+        for (int b = 0; b < 2; ++b) {
+            const uint32_t iss = b ? issued1 : issued0, done = b ? seen1 : seen0;
+            if (iss > done && !__all_sync(0xffffffffu, sm100::mbar_wait(kbar(b), (iss - 1u) & 1u, p.wait_cycles)) &&
+                lane == 0 && p.status)
+                atomicOr(p.status, LRAR_STATUS_WAIT_TIMEOUT);
+        }
 }
 
 struct Ph2Params {
@@ -368,6 +421,25 @@ __global__ void __launch_bounds__(kThreads) block_phase2_kernel(const Ph2Params 
 }
 
 // --------------------------------------------------------------- launch ----
+// Keys as whole 16-byte vectors (vector loads, and bulk copies when staged).
+template <typename Tin>
+static bool ph1_key_vec(const BlockPh1Args &a) {
+    constexpr int esz = sizeof(Tin);
+    return (a.r * esz) % 16 == 0 && (a.variant == kSliced ? ((a.d - a.r) * esz) % 16 == 0
+                                                          : (reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
+}
+
+// A token's keys are staged in shared memory when they are whole vectors and fit 4 KB.
+template <typename Tin>
+static bool ph1_stages_keys_t(const BlockPh1Args &a) {
+    const size_t kbuf_bytes = (size_t)round_up(a.n * (a.r * (int)sizeof(Tin) + 16), 16);
+    return ph1_key_vec<Tin>(a) && kbuf_bytes <= 4096;
+}
+
+bool block_phase1_stages_keys(const BlockPh1Args &a) {
+    return a.in_dtype == kBF16 ? ph1_stages_keys_t<bf16>(a) : ph1_stages_keys_t<float>(a);
+}
+
 template <typename Tin, typename Tout>
 static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
     constexpr int E = VecE<Tin>::value;
@@ -386,15 +458,15 @@ static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
     p.eps = a.eps;
     p.inv_r = 1.f / (float)a.r;
     p.sliced = a.variant == kSliced;
-    constexpr int esz = sizeof(Tin);
-    p.key_vec = (a.r * esz) % 16 == 0 &&
-                (a.variant == kSliced ? ((a.d - a.r) * esz) % 16 == 0
-                                      : (reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
+    p.status = a.status;
+    p.wait_cycles = a.wait_cycles;
+    p.stall = a.stall ? 1 : 0;
+    p.key_vec = ph1_key_vec<Tin>(a);
     const int G = kWarps / chunks;
     constexpr int S = kPh1Stages;
     const int kstride = a.r * (int)sizeof(Tin) + 16;
     const size_t kbuf_bytes = (size_t)round_up(a.n * kstride, 16);
-    const bool ks = p.key_vec && kbuf_bytes <= 4096;  // keys staged in shared memory
+    const bool ks = ph1_stages_keys_t<Tin>(a);  // keys staged in shared memory
     const size_t smem = (size_t)kWarps * S * 32 * 16 + (ks ? (size_t)G * 2 * (kbuf_bytes + 8) : 0) +
                         sizeof(float) * ((size_t)kPh1MaxSites * round_up(a.r, 4) + (size_t)G * 2 * kPh1MaxSites * a.n);
     const void *k = ks ? (const void *)block_phase1_kernel<Tin, Tout, S, true, true>

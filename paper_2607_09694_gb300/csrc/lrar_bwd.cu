@@ -28,6 +28,7 @@
 // bitwise reproducible on a given device.
 #include <type_traits>
 
+#include "lrar.h"
 #include "lrar_device.cuh"
 #include "lrar_launch.h"
 
@@ -38,11 +39,21 @@ struct BwdParams {
     const void *dh, *h;
     const float *query, *lse;
     float *partials;
+    int *status;  // optional: LRAR_STATUS_LSE_MISMATCH when a token's weights from lse do not sum to 1
     int64_t T;
     int n, d, r;
     float eps, inv_r;
     int sliced, key_vec, accumulate, h_bf16;
 };
+
+// Weights taken from a supplied lse sum to 1 up to fp32 rounding when the lse
+// belongs to the same values and query; a sum further than this from 1 marks
+// an lse of other inputs.
+constexpr float kLseSumTol = 1e-3f;
+
+__device__ __forceinline__ void check_alpha_sum(const BwdParams &p, float asum, int lane) {
+    if (lane == 0 && p.status && !(fabsf(asum - 1.f) <= kLseSumTol)) atomicOr(p.status, LRAR_STATUS_LSE_MISMATCH);
+}
 
 // Routing stage, identical arithmetic to the forward's (see lrar_fwd.cu).
 template <typename Tin>
@@ -580,11 +591,11 @@ __global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(c
 // One source row of the full-key backward, with lse and gbar = <dh, h> known:
 // alpha_i, g_i = <dh, o_i>, ds_i (Eq. 11-12), and the value gradient
 // alpha_i dh + ds_i rho_i (q - (s_i / d) kbar_i) written in one pass (the key
-// is the value, Eq. 13).  Operands stay packed and are unpacked one vector at
+// is the value, Eq. 13).  Returns alpha_i (warp-uniform).  Operands stay packed and are unpacked one vector at
 // a time; q_s (laid out by q_slot) is zero past d.  dq accumulates in dqf: V * E registers, or with
 // DQS the warp's d floats in shared memory.
 template <typename Tin, typename Tg, int V, bool DQS = false>
-__device__ __forceinline__ void full_bwd_row(const Frag<Tin, VecE<Tin>::value> *f,
+__device__ __forceinline__ float full_bwd_row(const Frag<Tin, VecE<Tin>::value> *f,
                                              const Frag<Tg, VecE<Tin>::value> *old,
                                              const Frag<Tin, VecE<Tin>::value> *dhr,
                                              const float *__restrict__ q_s, float *dqf, float gbar, float lse,
@@ -652,6 +663,7 @@ __device__ __forceinline__ void full_bwd_row(const Frag<Tin, VecE<Tin>::value> *
             out.store(drow + e);
         }
     }
+    return a;
 }
 
 // gbar = <dh, h> = sum_i alpha_i g_i for one token, from the saved output.
@@ -783,6 +795,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_full_pipe_kernel(const __grid
         }
         const float gbar = full_gbar<T, V>(p, dhr, x, lane);
         const float lse = __ldg(p.lse + x);
+        float asum = 0.f;
         for (int i = 0; i < p.n; ++i) {
             issue(st_i);
             cp_async_wait<S - 1>();
@@ -795,11 +808,12 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_full_pipe_kernel(const __grid
                 if (ACC && e < p.d) old[v].a = ld_shared16(cell(st_c, P - 1, v));
                 else old[v].zero();
             }
-            full_bwd_row<T, T, V, DQS>(f, old, dhr, q_s, dqf, gbar, lse, inv_d, p.eps,
-                                       dst_row<T>(p.dvt, i, x, p.d), p.d, lane, ACC);
+            asum += full_bwd_row<T, T, V, DQS>(f, old, dhr, q_s, dqf, gbar, lse, inv_d, p.eps,
+                                               dst_row<T>(p.dvt, i, x, p.d), p.d, lane, ACC);
             st_c = (st_c + 1 == S) ? 0 : st_c + 1;
             st_i = (st_i + 1 == S) ? 0 : st_i + 1;
         }
+        check_alpha_sum(p, asum, lane);
     }
     cp_async_wait_all();
     __syncthreads();  // every warp is done with the ring before it becomes dq scratch
@@ -921,6 +935,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_slr_onepass_kernel(const __gr
         for (int v = 0; v < V; ++v)
             if (v == vk && has_key) st_shared16(dhs_w + (uint32_t)(kvi * 16), dhr[v].a);
 
+        float asum = 0.f;
         for (int i = 0; i < p.n; ++i) {
             issue(st_i);
             cp_async_wait<S - 1>();  // this lane's copies of row i have landed
@@ -958,6 +973,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_slr_onepass_kernel(const __gr
             const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
             const float s = __shfl_sync(0xffffffffu, rho * qk, lead);
             const float a = expf(s - lse);
+            asum += a;
             T *drow = dst_row<T>(p.dvt, i, x, p.d);
 #pragma unroll
             for (int v = 0; v < V; ++v) {
@@ -987,6 +1003,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_slr_onepass_kernel(const __gr
             st_i = (st_i + 1 == S) ? 0 : st_i + 1;
         }
         __syncwarp();  // stash, tables and the dh slice are visible to the whole warp
+        check_alpha_sum(p, asum, lane);
 
         float part = 0.f;
         for (int k = lane; k < p.n; k += 32) part = fmaf(a_s[k], g_s[k], part);
@@ -1068,6 +1085,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(co
         }
         const float gbar = full_gbar<Tin, V>(p, dhr, x, lane);
         const float lse = __ldg(p.lse + x);
+        float asum = 0.f;
         int i = 0;
         for (; i + U <= p.n; i += U) {
             Frag<Tin, E> f[U][V];
@@ -1084,8 +1102,8 @@ __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(co
                 }
 #pragma unroll
             for (int u = 0; u < U; ++u)
-                full_bwd_row<Tin, Tg, V>(f[u], old[u], dhr, q_s, dqf, gbar, lse, inv_d, p.eps,
-                                         dst_row<Tg>(p.dvt, i + u, x, p.d), p.d, lane, p.accumulate);
+                asum += full_bwd_row<Tin, Tg, V>(f[u], old[u], dhr, q_s, dqf, gbar, lse, inv_d, p.eps,
+                                                 dst_row<Tg>(p.dvt, i + u, x, p.d), p.d, lane, p.accumulate);
         }
         for (; i < p.n; ++i) {
             Frag<Tin, E> f[V];
@@ -1098,9 +1116,10 @@ __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(co
                 if (p.accumulate && e < p.d) old[v].load(dst_row<Tg>(p.dvt, i, x, p.d) + e);
                 else old[v].zero();
             }
-            full_bwd_row<Tin, Tg, V>(f, old, dhr, q_s, dqf, gbar, lse, inv_d, p.eps,
-                                     dst_row<Tg>(p.dvt, i, x, p.d), p.d, lane, p.accumulate);
+            asum += full_bwd_row<Tin, Tg, V>(f, old, dhr, q_s, dqf, gbar, lse, inv_d, p.eps,
+                                             dst_row<Tg>(p.dvt, i, x, p.d), p.d, lane, p.accumulate);
         }
+        check_alpha_sum(p, asum, lane);
     }
     full_dq_partial<Tin, V>(p, dqf, scratch, lane, warp);
 }
@@ -1156,6 +1175,7 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     p.query = a.query;
     p.lse = a.lse;
     p.partials = a.partials;
+    p.status = a.status;
     p.T = a.T;
     p.n = a.n;
     p.d = a.d;

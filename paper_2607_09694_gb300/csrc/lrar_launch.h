@@ -48,6 +48,7 @@ struct BwdArgs {
     float *dq;
     int accumulate;
     float *partials;  // workspace: [kMaxPartials][rq] floats
+    int *status;      // optional: LRAR_STATUS_LSE_MISMATCH is ORed in by kernels that take alpha from lse
 };
 
 struct BlockPh1Args {
@@ -61,7 +62,18 @@ struct BlockPh1Args {
     float eps;
     void *h_pre;     // [c, T, d]
     float *lse_pre;  // [c, T]
+    int *status;     // optional: LRAR_STATUS_WAIT_TIMEOUT is ORed in when a key wait gives up
+    long long wait_cycles;  // bound of each key wait (SM clock cycles)
+    bool stall;      // test hook: key waits wait on a barrier nothing completes
 };
+
+// Bound of a kernel's waits on its own asynchronous copies: about 2 s at the
+// GB300's 2.07 GHz SM clock, far beyond any copy's latency.
+constexpr long long kWaitCycles = 4LL << 30;
+
+// Whether a phase-1 launch with these arguments stages keys in shared memory
+// (and so waits for bulk copies).
+bool block_phase1_stages_keys(const BlockPh1Args &a);
 
 struct BlockPh2Args {
     int variant, in_dtype, pre_dtype, out_dtype;
@@ -83,10 +95,20 @@ cudaError_t launch_block_phase2(const BlockPh2Args &a, cudaStream_t s);
 // Sets the calling thread's lrar_last_error() message; returns `code`.
 int record_error(int code, const char *message);
 
+// Every argument check of lrar_backward on a stacked buffer except those of
+// the workspace, in the same order and with the same messages; launches
+// nothing.  LRAR_OK for T == 0 once the scalar arguments are valid.
+int check_backward(int variant, int in_dtype, int grad_dtype, const void *values, const void *keys,
+                   const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh, const void *h,
+                   int h_dtype, const float *lse, const void *dvalues, const void *dkeys, const float *dq,
+                   int accumulate, const int *status);
+
 // P-LR fused output projection on the tensor cores (lrar_proj.cu); returns an
 // LRAR status (argument checks done by the caller).
+// tile: 0 picks the width from the shape, else one of the compiled widths.
 int launch_project(const void *a, const void *w, int64_t T, int m, int d, int r, void *o, void *keys, int *status,
-                   cudaStream_t s);
+                   int tile, cudaStream_t s);
+bool project_tile_ok(int tile);
 
 // Largest d one warp covers (the kernels keep a whole token row per warp).
 int max_width(int in_dtype);

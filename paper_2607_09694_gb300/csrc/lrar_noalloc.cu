@@ -21,9 +21,13 @@
 //     reduction reads it), but calls that may run at the same time on the GPU
 //     (on different streams, or issued by different host threads without
 //     ordering) race on it and must be serialised by the caller;
-//   * the first call on each device looks up the array's device address
-//     (cudaGetSymbolAddress) with that device current; make that first call
-//     before any stream capture.
+//   * the first call on each device that gets past the argument checks looks
+//     up the array's device address (cudaGetSymbolAddress) with that device
+//     current and keeps it for the life of the process; make that first call
+//     before any stream capture.  A reset of the device or of its primary
+//     context (cudaDeviceReset) unloads the library's device code and leaves
+//     the kept address stale, so the call must not be used on a device after
+//     such a reset.
 #include <mutex>
 
 #include "lrar.h"
@@ -69,15 +73,22 @@ int scratch_address(void **out) {
 LRAR_API int lrar_backward_noalloc(int variant, int in_dtype, int grad_dtype, const void *values, const void *keys,
                                    const float *query, int n_src, int64_t T, int d, int r, float eps, const void *dh,
                                    const void *h, int h_dtype, const float *lse, void *dvalues, void *dkeys,
-                                   float *dq, int accumulate, void *stream) {
+                                   float *dq, int accumulate, int *status, void *stream) {
+    // lrar_backward's own checks first, so that a bad argument gets its code and
+    // message without touching the device
+    int rc = lrar::check_backward(variant, in_dtype, grad_dtype, values, keys, query, n_src, T, d, r, eps, dh, h,
+                                  h_dtype, lse, dvalues, dkeys, dq, accumulate, status);
+    if (rc != LRAR_OK) return rc;
+    if (T == 0)  // nothing to reduce: lrar_backward only sets dq (no workspace involved)
+        return lrar_backward(variant, in_dtype, grad_dtype, values, keys, query, n_src, T, d, r, eps, dh, h, h_dtype,
+                             lse, dvalues, dkeys, dq, accumulate, nullptr, 0, status, stream);
     const size_t need = lrar_backward_workspace_size(variant, n_src, T, d, r);
     if (need > kScratchBytes)
         return lrar::record_error(LRAR_ERR_UNSUPPORTED,
                                   "lrar_backward_noalloc: needs more scratch than its fixed 4 MiB (dq width > 1024); "
                                   "use lrar_backward with a workspace");
     void *scratch = nullptr;
-    const int rc = scratch_address(&scratch);
-    if (rc != LRAR_OK) return rc;
+    if ((rc = scratch_address(&scratch)) != LRAR_OK) return rc;
     return lrar_backward(variant, in_dtype, grad_dtype, values, keys, query, n_src, T, d, r, eps, dh, h, h_dtype, lse,
-                         dvalues, dkeys, dq, accumulate, scratch, kScratchBytes, stream);
+                         dvalues, dkeys, dq, accumulate, scratch, kScratchBytes, status, stream);
 }

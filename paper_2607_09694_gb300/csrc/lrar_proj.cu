@@ -23,7 +23,6 @@
 // shared abort flag that ends the other roles' waits, and the kernel drains
 // its copies and MMAs and frees TMEM before it returns.
 #include <cmath>
-#include <cstdlib>
 #include <mutex>
 
 #include "lrar.h"
@@ -42,7 +41,7 @@ constexpr int kPThreads = 192;                  // 6 warps
 constexpr uint32_t kAccCols = 256;              // TMEM columns per accumulator (>= the tile width)
 constexpr uint32_t kTmemCols = 2 * kAccCols;    // two accumulators: the whole TMEM of the SM
 constexpr int kABytes = kPM * kPK * 2;          // 16 KB
-constexpr long long kWaitLimit = 4LL << 30;     // SM cycles (about 2 s) before a wait gives up
+constexpr long long kWaitLimit = kWaitCycles;   // SM cycles (about 2 s) before a wait gives up
 
 // Tile width BN (columns of Y), picked per call by the host (tile_efficiency).
 template <int BN> struct ProjTile {
@@ -61,12 +60,12 @@ struct ProjParams {
     bf16 *keys;  // [T, r]
     int64_t T;
     int m, d, r;
-    int *status;  // set to 1 when a wait ran out (may be null)
+    int *status;  // LRAR_STATUS_WAIT_TIMEOUT is ORed in when a wait ran out (may be null)
 };
 
 __device__ __forceinline__ void give_up(int *status, volatile int *abort) {
     *abort = 1;
-    if (status) atomicExch(status, 1);
+    if (status) atomicOr(status, LRAR_STATUS_WAIT_TIMEOUT);
 }
 
 template <int kPN>
@@ -218,7 +217,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
         // the copies still in flight before the CTA's shared memory goes away.
         for (int64_t g = issued - kPStages > 0 ? issued - kPStages : 0; g < issued; ++g)
             if (!mbar_wait(full((int)(g % kPStages)), (uint32_t)(g / kPStages) & 1u, kWaitLimit)) {
-                if (p.status) atomicExch(p.status, 1);
+                if (p.status) atomicOr(p.status, LRAR_STATUS_WAIT_TIMEOUT);
             }
     }
     if (warp == 5) {
@@ -299,8 +298,14 @@ constexpr int kTileWidths[] = {160, 176, 192, 224, 240, 256};
 
 }  // namespace
 
+bool project_tile_ok(int tile) {
+    for (int c : kTileWidths)
+        if (c == tile) return true;
+    return false;
+}
+
 int launch_project(const void *a, const void *w, int64_t T, int m, int d, int r, void *o, void *keys, int *status,
-                   cudaStream_t s) {
+                   int tile, cudaStream_t s) {
     CUtensorMap map_a;
     if (!make_map(&map_a, a, T, m, kPM))
         return record_error(LRAR_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point or arguments)");
@@ -316,7 +321,7 @@ int launch_project(const void *a, const void *w, int64_t T, int m, int d, int r,
             bn = c;
         }
     }
-    if (const char *force = getenv("LRAR_PROJ_TILE")) bn = atoi(force);  // tuning override
+    if (tile != 0) bn = tile;  // forced by the test hook (checked by the caller)
     switch (bn) {
         case 160: return launch_project_t<160>(map_a, w, T, m, d, r, o, keys, status, s);
         case 176: return launch_project_t<176>(map_a, w, T, m, d, r, o, keys, status, s);
@@ -324,7 +329,7 @@ int launch_project(const void *a, const void *w, int64_t T, int m, int d, int r,
         case 224: return launch_project_t<224>(map_a, w, T, m, d, r, o, keys, status, s);
         case 240: return launch_project_t<240>(map_a, w, T, m, d, r, o, keys, status, s);
         case 256: return launch_project_t<256>(map_a, w, T, m, d, r, o, keys, status, s);
-        default: return record_error(LRAR_ERR_INVALID_ARG, "LRAR_PROJ_TILE must be 160, 176, 192, 224, 240 or 256");
+        default: return record_error(LRAR_ERR_INVALID_ARG, "tile must be 160, 176, 192, 224, 240 or 256");
     }
 }
 

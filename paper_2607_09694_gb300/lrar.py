@@ -21,6 +21,7 @@ DEFAULT_EPS = 1e-6
 
 OK = 0
 ERR_INVALID_ARG, ERR_ALIGNMENT, ERR_UNSUPPORTED, ERR_CUDA, ERR_WORKSPACE = -1, -2, -3, -4, -5
+STATUS_WAIT_TIMEOUT, STATUS_LSE_MISMATCH = 1, 2  # bits of the optional device status words
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "liblrar.so")
@@ -28,6 +29,7 @@ EXPORTS = ("lrar_forward", "lrar_backward", "lrar_backward_workspace_size", "lra
            "lrar_strerror", "lrar_last_error", "lrar_version", "lrar_backward_noalloc", "lrar_diagnostics",
            "lrar_diagnostics_workspace_size", "lrar_block_phase1", "lrar_block_phase2", "lrar_project",
            "lrar_forward_ptrs", "lrar_backward_ptrs")
+TEST_HOOKS = ("lrar_test_project_tile", "lrar_test_block_phase1_stalled")  # include/lrar_testing.h
 MAX_BLOCK_SITES = 64
 
 _lock = threading.Lock()
@@ -53,12 +55,19 @@ def load(path: str | None = None):
         vp, i, i64, f32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
         lib.lrar_forward.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, vp]
         lib.lrar_forward.restype = i
-        lib.lrar_backward.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, i, vp, vp, vp, vp, i, vp, sz, vp]
+        lib.lrar_backward.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, i, vp, vp, vp, vp, i, vp, sz, vp,
+                                      vp]
         lib.lrar_backward.restype = i
-        lib.lrar_backward_noalloc.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, i, vp, vp, vp, vp, i, vp]
+        lib.lrar_backward_noalloc.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, i, vp, vp, vp, vp, i, vp,
+                                              vp]
         lib.lrar_backward_noalloc.restype = i
-        lib.lrar_block_phase1.argtypes = [i, i, i, vp, vp, vp, i, i, i64, i, i, f32, vp, vp, vp]
+        lib.lrar_block_phase1.argtypes = [i, i, i, vp, vp, vp, i, i, i64, i, i, f32, vp, vp, vp, vp]
         lib.lrar_block_phase1.restype = i
+        lib.lrar_test_block_phase1_stalled.argtypes = [i, i, i, vp, vp, vp, i, i, i64, i, i, f32, vp, vp, vp,
+                                                       ctypes.c_longlong, vp]
+        lib.lrar_test_block_phase1_stalled.restype = i
+        lib.lrar_test_project_tile.argtypes = [i, i, vp, vp, i64, i, i, i, vp, vp, vp, vp]
+        lib.lrar_test_project_tile.restype = i
         lib.lrar_block_phase2.argtypes = [i, i, i, i, vp, vp, vp, vp, vp, i64, i, i, f32, vp, vp, vp]
         lib.lrar_block_phase2.restype = i
         lib.lrar_diagnostics.argtypes = [i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, vp, sz, vp]
@@ -70,7 +79,7 @@ def load(path: str | None = None):
         lib.lrar_forward_ptrs.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, vp]
         lib.lrar_forward_ptrs.restype = i
         lib.lrar_backward_ptrs.argtypes = [i, i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, i, vp, vp, vp, vp, i, vp,
-                                           sz, vp]
+                                           sz, vp, vp]
         lib.lrar_backward_ptrs.restype = i
         lib.lrar_project.argtypes = [i, vp, vp, i64, i, i, i, vp, vp, vp, vp]
         lib.lrar_project.restype = i
@@ -151,9 +160,10 @@ def backward(variant, values: torch.Tensor, keys: torch.Tensor | None, query: to
              dh: torch.Tensor, dvalues: torch.Tensor, dq: torch.Tensor, workspace: torch.Tensor,
              dkeys: torch.Tensor | None = None, h: torch.Tensor | None = None, lse: torch.Tensor | None = None,
              n_src: int | None = None, r: int | None = None, accumulate: bool = False,
-             eps: float = DEFAULT_EPS, stream=None) -> None:
+             eps: float = DEFAULT_EPS, status: torch.Tensor | None = None, stream=None) -> None:
     """lrar_backward for the first n_src sources of `values`; gradients go to the
-    first n_src slices of `dvalues` (and `dkeys`)."""
+    first n_src slices of `dvalues` (and `dkeys`).  status: optional int32
+    device scalar that collects STATUS_LSE_MISMATCH."""
     variant = _variant(variant)
     _, T, d = values.shape
     n = values.shape[0] if n_src is None else n_src
@@ -163,7 +173,7 @@ def backward(variant, values: torch.Tensor, keys: torch.Tensor | None, query: to
     _check(load().lrar_backward(variant, dtype_code(values), dtype_code(dvalues), _ptr(values), _ptr(keys),
                                 _ptr(query), n, T, d, r, eps, _ptr(dh), _ptr(h), dtype_code(h), _ptr(lse),
                                 _ptr(dvalues), _ptr(dkeys), _ptr(dq), int(bool(accumulate)), _ptr(workspace),
-                                ws_bytes, _stream(stream)))
+                                ws_bytes, _ptr(status), _stream(stream)))
 
 
 def _table(ts):
@@ -188,7 +198,8 @@ def forward_ptrs(variant, values, keys, query: torch.Tensor | None, h: torch.Ten
 
 def backward_ptrs(variant, values, keys, query: torch.Tensor | None, dh: torch.Tensor, dvalues, dq: torch.Tensor,
                   workspace: torch.Tensor, dkeys=None, h: torch.Tensor | None = None, lse: torch.Tensor | None = None,
-                  r: int | None = None, accumulate: bool = False, eps: float = DEFAULT_EPS, stream=None) -> None:
+                  r: int | None = None, accumulate: bool = False, eps: float = DEFAULT_EPS,
+                  status: torch.Tensor | None = None, stream=None) -> None:
     """lrar_backward_ptrs: like backward, with sources and their gradients as
     lists of separate tensors (gradient i goes to dvalues[i], dkeys[i])."""
     variant = _variant(variant)
@@ -200,13 +211,14 @@ def backward_ptrs(variant, values, keys, query: torch.Tensor | None, dh: torch.T
     _check(load().lrar_backward_ptrs(variant, dtype_code(values[0]), dtype_code(dvalues[0]), _table(values),
                                      _table(keys), _ptr(query), n, T, d, r, eps, _ptr(dh), _ptr(h), dtype_code(h),
                                      _ptr(lse), _table(dvalues), _table(dkeys), _ptr(dq), int(bool(accumulate)),
-                                     _ptr(workspace), ws_bytes, _stream(stream)))
+                                     _ptr(workspace), ws_bytes, _ptr(status), _stream(stream)))
 
 
 def backward_noalloc(variant, values: torch.Tensor, keys: torch.Tensor | None, query: torch.Tensor | None,
                      dh: torch.Tensor, dvalues: torch.Tensor, dq: torch.Tensor, dkeys: torch.Tensor | None = None,
                      h: torch.Tensor | None = None, lse: torch.Tensor | None = None, n_src: int | None = None,
-                     r: int | None = None, accumulate: bool = False, eps: float = DEFAULT_EPS, stream=None) -> None:
+                     r: int | None = None, accumulate: bool = False, eps: float = DEFAULT_EPS,
+                     status: torch.Tensor | None = None, stream=None) -> None:
     """lrar_backward_noalloc: lrar_backward without a workspace, for callers
     that cannot allocate device memory (scratch is the library's fixed 4 MiB
     array per device; calls that may overlap on the GPU race on it)."""
@@ -218,20 +230,22 @@ def backward_noalloc(variant, values: torch.Tensor, keys: torch.Tensor | None, q
     _check(load().lrar_backward_noalloc(variant, dtype_code(values), dtype_code(dvalues), _ptr(values), _ptr(keys),
                                         _ptr(query), n, T, d, r, eps, _ptr(dh), _ptr(h), dtype_code(h), _ptr(lse),
                                         _ptr(dvalues), _ptr(dkeys), _ptr(dq), int(bool(accumulate)),
-                                        _stream(stream)))
+                                        _ptr(status), _stream(stream)))
 
 
 def block_phase1(variant, values: torch.Tensor, keys: torch.Tensor | None, queries: torch.Tensor,
                  h_pre: torch.Tensor, lse_pre: torch.Tensor, n_completed: int | None = None,
-                 eps: float = DEFAULT_EPS, stream=None) -> None:
+                 eps: float = DEFAULT_EPS, status: torch.Tensor | None = None, stream=None) -> None:
     """lrar_block_phase1: mixes of the first n_completed sources of `values` for
-    every query row of `queries` [n_sites, r] -> h_pre [n_sites, T, d], lse_pre [n_sites, T]."""
+    every query row of `queries` [n_sites, r] -> h_pre [n_sites, T, d], lse_pre [n_sites, T].
+    status: optional int32 device scalar that collects STATUS_WAIT_TIMEOUT."""
     variant = _variant(variant)
     _, T, d = values.shape
     n = values.shape[0] if n_completed is None else n_completed
     c, r = queries.shape
     _check(load().lrar_block_phase1(variant, dtype_code(values), dtype_code(h_pre), _ptr(values), _ptr(keys),
-                                    _ptr(queries), n, c, T, d, r, eps, _ptr(h_pre), _ptr(lse_pre), _stream(stream)))
+                                    _ptr(queries), n, c, T, d, r, eps, _ptr(h_pre), _ptr(lse_pre), _ptr(status),
+                                    _stream(stream)))
 
 
 def block_phase2(variant, h_pre: torch.Tensor, lse_pre: torch.Tensor, partial: torch.Tensor,
@@ -290,3 +304,31 @@ def project(a: torch.Tensor, w: torch.Tensor, o: torch.Tensor | None, keys: torc
 
 def version() -> int:
     return int(load().lrar_version())
+
+
+# ------------------------------------------------------------ test hooks ----
+# include/lrar_testing.h: variants of the calls above that let the tests reach
+# paths ordinary inputs do not choose.  Not part of the library's interface.
+def test_project_tile(tile: int, a: torch.Tensor, w: torch.Tensor, o: torch.Tensor | None,
+                      keys: torch.Tensor | None, status: torch.Tensor | None = None, stream=None) -> None:
+    """lrar_test_project_tile: project() with the tile width forced."""
+    T, m = a.shape
+    d = 0 if o is None else o.shape[-1]
+    r = 0 if keys is None else keys.shape[-1]
+    if w.shape[0] != d + r or w.shape[-1] != m:
+        raise ValueError(f"w must be [{d + r}, {m}], got {tuple(w.shape)}")
+    _check(load().lrar_test_project_tile(int(tile), dtype_code(a), _ptr(a), _ptr(w), T, m, d, r, _ptr(o),
+                                         _ptr(keys), _ptr(status), _stream(stream)))
+
+
+def test_block_phase1_stalled(variant, values: torch.Tensor, keys: torch.Tensor | None, queries: torch.Tensor,
+                              h_pre: torch.Tensor, lse_pre: torch.Tensor, status: torch.Tensor, wait_cycles: int,
+                              n_completed: int | None = None, eps: float = DEFAULT_EPS, stream=None) -> None:
+    """lrar_test_block_phase1_stalled: block_phase1() whose key waits all run out."""
+    variant = _variant(variant)
+    _, T, d = values.shape
+    n = values.shape[0] if n_completed is None else n_completed
+    c, r = queries.shape
+    _check(load().lrar_test_block_phase1_stalled(variant, dtype_code(values), dtype_code(h_pre), _ptr(values),
+                                                 _ptr(keys), _ptr(queries), n, c, T, d, r, eps, _ptr(h_pre),
+                                                 _ptr(lse_pre), _ptr(status), int(wait_cycles), _stream(stream)))

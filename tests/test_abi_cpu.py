@@ -20,16 +20,21 @@ def lib():
     return lrar.load()
 
 
-def _declared():
-    text = open(os.path.join(ROOT, "include", "lrar.h")).read()
+def _declared(header="lrar.h"):
+    text = open(os.path.join(ROOT, "include", header)).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
     return sorted(set(re.findall(r"\b(lrar_[a-z0-9_]+)\s*\(", text)))
 
 
+def _all_declared():
+    headers = sorted(f for f in os.listdir(os.path.join(ROOT, "include")) if f.endswith(".h"))
+    return sorted(set(n for h in headers for n in _declared(h)))
+
+
 def test_every_declared_symbol_is_exported(lib):
-    names = _declared()
-    assert set(names) == set(lrar.EXPORTS)
-    for n in names:
+    assert set(_declared("lrar.h")) == set(lrar.EXPORTS)
+    assert set(_declared("lrar_testing.h")) == set(lrar.TEST_HOOKS)
+    for n in _all_declared():
         assert hasattr(lib, n), n
 
 
@@ -38,11 +43,11 @@ def test_only_declared_symbols_are_exported(lib):
 
     out = subprocess.run(["nm", "-D", "--defined-only", lrar.LIB_PATH], capture_output=True, text=True).stdout
     syms = {line.split()[-1] for line in out.splitlines() if " T " in line}
-    assert syms == set(_declared())
+    assert syms == set(_all_declared())
 
 
 def test_version_and_strings(lib):
-    assert lib.lrar_version() == 1
+    assert lib.lrar_version() == 2
     for code in (0, -1, -2, -3, -4, -5):
         assert lib.lrar_strerror(code)
     assert b"unknown" in lib.lrar_strerror(-99)
@@ -54,11 +59,11 @@ def fwd(lib, variant=1, ind=1, outd=1, values=FAKE, keys=None, query=FAKE, n=4, 
 
 
 def bwd(lib, variant=1, ind=1, gd=1, values=FAKE, keys=None, query=FAKE, n=4, T=8, d=64, r=4, eps=EPS, dh=FAKE,
-        h=None, hd=1, lse=None, dv=FAKE, dk=None, dq=FAKE, acc=0, ws=FAKE, wsb=None):
+        h=None, hd=1, lse=None, dv=FAKE, dk=None, dq=FAKE, acc=0, ws=FAKE, wsb=None, st=None):
     if wsb is None:
         wsb = lib.lrar_backward_workspace_size(variant, n, T, d, r)
     return lib.lrar_backward(variant, ind, gd, values, keys, query, n, T, d, r, eps, dh, h, hd, lse, dv, dk, dq, acc,
-                             ws, wsb, None)
+                             ws, wsb, st, None)
 
 
 @pytest.mark.parametrize("kw,code", [
@@ -109,6 +114,7 @@ def test_forward_empty_is_noop(lib):
     (dict(wsb=16), lrar.ERR_WORKSPACE),
     (dict(ws=FAKE + 8), lrar.ERR_ALIGNMENT),
     (dict(dv=FAKE + 2), lrar.ERR_ALIGNMENT),
+    (dict(st=FAKE + 2), lrar.ERR_ALIGNMENT),
     (dict(n=200), lrar.ERR_UNSUPPORTED),
 ])
 def test_backward_rejects(lib, kw, code):
@@ -205,11 +211,11 @@ def test_pointer_tables_rejected_before_launch(lib):
     b = lib.lrar_backward_ptrs
     ws = lib.lrar_backward_workspace_size(1, n, T, d, r)
     assert b(1, 1, 1, good, None, FAKE, n, T, d, r, EPS, FAKE, None, 1, None, None, None, FAKE, 0, FAKE, ws,
-             None) == lrar.ERR_INVALID_ARG  # dvalues table
+             None, None) == lrar.ERR_INVALID_ARG  # dvalues table
     assert b(1, 1, 1, good, None, FAKE, n, T, d, r, EPS, FAKE, None, 1, None, odd_entry, None, FAKE, 0, FAKE, ws,
-             None) == lrar.ERR_ALIGNMENT
+             None, None) == lrar.ERR_ALIGNMENT
     assert b(1, 1, 1, good, None, FAKE, n, T, d, r, EPS, FAKE, None, 1, None, good, None, FAKE, 0, FAKE, 16,
-             None) == lrar.ERR_WORKSPACE
+             None, None) == lrar.ERR_WORKSPACE
 
 
 def test_binding_rejects_host_and_strided_tensors(lib):
@@ -260,3 +266,54 @@ def test_plain_c_client_compiles_links_and_runs(lib, tmp_path):
     out = subprocess.run([exe], capture_output=True, text=True)
     assert out.returncode == 0, out.stdout + out.stderr
     assert "invalid argument" in out.stdout
+
+
+@pytest.mark.parametrize("kw", [
+    dict(gd=5), dict(acc=2), dict(dq=None), dict(dv=None), dict(dh=None), dict(n=0), dict(eps=0.0), dict(st=FAKE + 1),
+    dict(variant=2, keys=FAKE, dk=None), dict(variant=0, d=64, r=64, h=FAKE, lse=None), dict(dv=FAKE + 2),
+    dict(n=200),
+])
+def test_noalloc_rejects_like_the_workspace_backward(lib, kw):
+    """lrar_backward_noalloc runs lrar_backward's argument checks before it
+    looks up its scratch on the device: a bad call returns the same code and
+    message as lrar_backward, with or without a device present."""
+    code = bwd(lib, **kw)
+    msg = lib.lrar_last_error()
+    assert code < 0
+    a = dict(variant=1, ind=1, gd=1, values=FAKE, keys=None, query=FAKE, n=4, T=8, d=64, r=4, eps=EPS, dh=FAKE,
+             h=None, hd=1, lse=None, dv=FAKE, dk=None, dq=FAKE, acc=0, st=None)
+    a.update(kw)
+    got = lib.lrar_backward_noalloc(a["variant"], a["ind"], a["gd"], a["values"], a["keys"], a["query"], a["n"],
+                                    a["T"], a["d"], a["r"], a["eps"], a["dh"], a["h"], a["hd"], a["lse"], a["dv"],
+                                    a["dk"], a["dq"], a["acc"], a["st"], None)
+    assert got == code
+    assert lib.lrar_last_error() == msg
+
+
+def test_block_phase1_rejects(lib):
+    f = lib.lrar_block_phase1
+    args = [1, 1, 1, FAKE, None, FAKE, 4, 8, 16, 64, 8, EPS, FAKE, FAKE]
+    assert f(*args, FAKE + 2, None) == lrar.ERR_ALIGNMENT           # status
+    assert f(0, *args[1:], None, None) == lrar.ERR_UNSUPPORTED     # full keys
+    bad = list(args)
+    bad[7] = 0
+    assert f(*bad, None, None) == lrar.ERR_INVALID_ARG             # n_sites
+    bad = list(args)
+    bad[3] = None
+    assert f(*bad, None, None) == lrar.ERR_INVALID_ARG             # values
+    bad = list(args)
+    bad[8] = 0
+    bad[3] = None
+    assert f(*bad, None, None) == lrar.OK                          # T == 0
+
+
+def test_test_hooks_reject(lib):
+    t = lib.lrar_test_project_tile
+    assert t(0, 1, FAKE, FAKE, 8, 64, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_INVALID_ARG
+    assert t(200, 1, FAKE, FAKE, 8, 64, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_INVALID_ARG
+    assert t(160, 1, FAKE, FAKE, 0, 64, 64, 16, FAKE, FAKE, None, None) == lrar.OK  # T == 0
+    s = lib.lrar_test_block_phase1_stalled
+    args = [1, 1, 1, FAKE, None, FAKE, 4, 8, 16, 64, 8, EPS, FAKE, FAKE]
+    assert s(*args, None, 1000, None) == lrar.ERR_INVALID_ARG      # status required
+    assert s(*args, FAKE, 0, None) == lrar.ERR_INVALID_ARG         # wait bound
+    assert s(*args[:9], 64, 7, EPS, FAKE, FAKE, FAKE, 1000, None) == lrar.ERR_UNSUPPORTED  # r = 7: no staging

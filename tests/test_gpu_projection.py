@@ -18,13 +18,16 @@ def _operands(T, m, N, seed):
     return a, w
 
 
-def _run(T, m, d, r, seed=3):
+def _run(T, m, d, r, seed=3, tile=0):
     a, w = _operands(T, m, d + r, seed)
     dev = torch.device("cuda")
     o = torch.full((T, d), float("nan"), dtype=torch.bfloat16, device=dev) if d else None
     k = torch.full((T, r), float("nan"), dtype=torch.bfloat16, device=dev) if r else None
     status = torch.zeros(1, dtype=torch.int32, device=dev)
-    lrar.project(a.to(dev), w.to(dev), o, k, status=status)
+    if tile:
+        lrar.test_project_tile(tile, a.to(dev), w.to(dev), o, k, status=status)
+    else:
+        lrar.project(a.to(dev), w.to(dev), o, k, status=status)
     torch.cuda.synchronize()
     assert status.item() == 0, "a pipeline wait in the projection kernel gave up"
     return a, w, o, k
@@ -45,8 +48,8 @@ def _check(name, got, ref, a, w_rows):
     assert err.mean() <= 0.5 * H.bf16_ulp(ref).mean(), name
 
 
-def _compare(T, m, d, r, seed=3, tokens=None):
-    a, w, o, k = _run(T, m, d, r, seed)
+def _compare(T, m, d, r, seed=3, tokens=None, tile=0):
+    a, w, o, k = _run(T, m, d, r, seed, tile)
     ref = oracle.projection(a if tokens is None else a[tokens], w, d)
     if d:
         _check("o", o.cpu() if tokens is None else o.cpu()[tokens], ref["o"],
@@ -68,11 +71,10 @@ def test_ragged_edges():
 
 
 @pytest.mark.parametrize("width", [160, 176, 192, 224, 240, 256])
-def test_every_tile_width(width, monkeypatch):
-    """Each compiled tile width (forced through LRAR_PROJ_TILE) on ragged T, m and
-    N, the value/key split falling inside a tile."""
-    monkeypatch.setenv("LRAR_PROJ_TILE", str(width))
-    _compare(300, 1000, 1024, 16, seed=4)
+def test_every_tile_width(width):
+    """Each compiled tile width (forced through the lrar_test_project_tile hook)
+    on ragged T, m and N, the value/key split falling inside a tile."""
+    _compare(300, 1000, 1024, 16, seed=4, tile=width)
 
 
 def test_swiglu_output_projection():

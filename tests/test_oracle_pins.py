@@ -82,7 +82,7 @@ def test_single_source_is_identity(variant, d, r):
     assert np.array_equal(f["h"], v[0])
     b = oracle.backward(variant, v, k, q, EPS, dh, r=r)
     assert np.allclose(b["dvalues"][0], dh, atol=1e-15)
-    assert np.max(np.abs(b["dq"])) < 1e-15
+    assert np.max(np.abs(b["dq"])) < 1e-15 and np.max(b["dq_abs"]) < 1e-15
     if variant == PROJECTED:
         assert np.max(np.abs(b["dkeys"])) < 1e-15
 
@@ -112,6 +112,13 @@ def test_two_sources_closed_form():
     b = oracle.backward(PROJECTED, v, keys, q, EPS, dh, want_ds=True)
     gi = v[:, 0, :] @ dh[0]
     assert abs(b["ds"][0, 1] - a1 * (1 - a1) * (gi[1] - gi[0])) < 1e-13
+    # dq = sum_i ds_i kbar_i with ds_0 = -ds_1 and kbar_i = kappa_i u; the two
+    # terms share a sign (kappa_0 > 0 > kappa_1), so the magnitude of the terms
+    # summed, dq_abs = sum_i |ds_i kbar_i|, equals |dq| here
+    kap = c / np.sqrt(c * c + EPS)
+    ds1 = a1 * (1 - a1) * (gi[1] - gi[0])
+    assert np.allclose(b["dq"], ds1 * (kap[1] - kap[0]) * u, rtol=1e-12, atol=1e-15)
+    assert np.allclose(b["dq_abs"], abs(ds1) * (abs(kap[0]) + abs(kap[1])) * np.ones(r), rtol=1e-12, atol=1e-15)
 
 
 def test_zero_key_scores_zero():
@@ -197,9 +204,14 @@ def test_key_scale_invariance():
 def test_score_gradients_sum_to_zero(variant, d, r):
     """Softmax is invariant to adding a constant to every score, so sum_i ds_i = 0."""
     v, k, q, dh = _case(variant, 7, 5, d, r, seed=12)
-    ds = oracle.backward(variant, v, k, q, EPS, dh, r=r, want_ds=True)["ds"]
+    out = oracle.backward(variant, v, k, q, EPS, dh, r=r, want_ds=True)
+    ds = out["ds"]
     assert np.max(np.abs(ds.sum(axis=1))) < 1e-13
     assert np.max(np.abs(ds)) > 1e-3
+    # the magnitude of the terms of dq bounds |dq| (triangle inequality) and,
+    # over many tokens of mixed sign, exceeds it
+    assert np.all(out["dq_abs"] >= np.abs(out["dq"]) - 1e-15)
+    assert np.all(out["dq_abs"] > np.abs(out["dq"]))
 
 
 def test_key_gradient_is_orthogonal_to_key():

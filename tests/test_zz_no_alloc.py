@@ -10,10 +10,10 @@ The file name puts it last in collection, so that a run stopping at the first
 failure has already run every other test; it also passes on its own in a
 fresh process (the first call on the device does the scratch set-up).
 """
+import numpy as np
 import pytest
 import torch
 
-import gpu_helpers as H
 from paper_2607_09694_gb300 import lrar, synth
 
 pytestmark = pytest.mark.gpu
@@ -56,13 +56,16 @@ def _backward(si, noalloc):
 
 def test_consecutive_calls_match_the_workspace_backward():
     """Back-to-back calls with different shapes share the scratch; each result
-    matches lrar_backward on the same inputs (1e-2 x RMS, the bf16-input bound)."""
+    equals lrar_backward's on the same inputs bit for bit: both run the same
+    kernels on the same grid, and dq's partial sums are reduced in a fixed
+    order, so a stale or overlapping partial-sum row would show as a
+    difference.  (Accuracy against the oracle is covered by the parity tests.)"""
     sites = [_site(c) for c in CASES]
     refs = [_backward(si, noalloc=False) for si in sites]
     for si, ref in zip(sites + sites[:1], refs + refs[:1]):  # four calls in a row, first case again last
         got = _backward(si, noalloc=True)
         for name in ref:
-            H.assert_rms(f"{si.variant}:{name}", got[name], ref[name])
+            assert np.array_equal(got[name], ref[name]), f"{si.variant}:{name}"
 
 
 def test_rejects_problems_beyond_the_scratch():
