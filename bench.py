@@ -647,6 +647,82 @@ def run_suite(args):
               "per_site_ms": tn, "two_phase_ms": tt, "speedup": tn / tt, "per_site_bytes": naive_bytes,
               "two_phase_bytes": tp_bytes, "per_site_gbs": naive_bytes / tn / 1e6,
               "two_phase_gbs": tp_bytes / tt / 1e6})
+    del stack, h_pre, lse_pre
+    torch.cuda.empty_cache()
+    run_block_step(emit, dev, max(3, reps // 2))
+
+
+def run_block_step(emit, dev, reps: int):
+    """The Block AttnRes training step of the 32-layer, d = 2048 decoder
+    (M = 64 sub-layer outputs, c = 8, S-LR r = 64, T = 32768, bf16 outputs, h
+    and gradients) through sweep.BlockSweep: per step the assembly after each
+    sub-layer and the mix at each of the 65 sites (forward), then the backward
+    at each site in reverse and the fan-out of the summary gradients to the
+    members.  The outputs are written afresh before every step (untimed), as
+    the sub-layers would; bytes of the mix and of the assembly / fan-out (a9)
+    are reported separately."""
+    import torch
+
+    from paper_2607_09694_gb300 import sites, synth
+    from paper_2607_09694_gb300.sweep import BlockSweep
+
+    T, d, r, c, M = 32768, 2048, 64, 8, 64
+    fresh = synth.values(M + 1, T, d, 3, "bf16", device=dev)
+    outs = [torch.empty(T, d, dtype=torch.bfloat16, device=dev) for _ in range(M + 1)]
+    qs = synth.queries(M + 1, r, 3, device=dev)
+    dh = synth.upstream(T, d, 3, "bf16", sites=M + 1, device=dev)
+    h = torch.empty(M + 1, T, d, dtype=torch.bfloat16, device=dev)
+    lse = torch.empty(M + 1, T, device=dev)
+    douts = [torch.empty(T, d, dtype=torch.bfloat16, device=dev) for _ in range(M + 1)]
+    sw = BlockSweep("sliced", outs, qs, [dh[t] for t in range(M + 1)], h, lse, douts, c, r=r)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(reps + 1)]
+    for a, b, e in ev:
+        for i in range(M + 1):
+            outs[i].copy_(fresh[i])
+        sw.rearm()
+        a.record()
+        sw.forward()
+        b.record()
+        sw.backward()
+        e.record()
+    torch.cuda.synchronize()
+    fwd = statistics.median(a.elapsed_time(b) for a, b, _ in ev[1:])
+    bwd = statistics.median(b.elapsed_time(e) for _, b, e in ev[1:])
+    mix_f = mix_b = 0
+    for t in range(1, M + 2):
+        shp = sites.SiteShape("sliced", sites.block_num_sources(t, c), T, d, r, accumulate=int(t != M + 1))
+        mix_f += sites.forward_bytes(shp)
+        mix_b += sites.backward_bytes(shp)
+    asm = sum(sites.block_accumulate_bytes(T, d, 2, True) for i in range(1, M + 1) if not sites.block_opens_slot(i, c))
+    fan = (M + 1) * sites.block_accumulate_bytes(T, d, 2, False)
+    emit({"suite": "Block S-LR training step, 65 sites, d2048 r64 c8 T32768 (site by site)",
+          "fwd_ms": fwd, "bwd_ms": bwd, "step_ms": fwd + bwd, "mix_fwd_bytes": mix_f, "assembly_bytes": asm,
+          "mix_bwd_bytes": mix_b, "fanout_bytes": fan, "fwd_gbs": (mix_f + asm) / fwd / 1e6,
+          "bwd_gbs": (mix_b + fan) / bwd / 1e6, "step_gbs": (mix_f + asm + mix_b + fan) / (fwd + bwd) / 1e6,
+          "tokens_per_s_per_site": T * (M + 1) / ((fwd + bwd) / 1e3)})
+    del fresh, outs, dh, h, douts, sw
+    torch.cuda.empty_cache()
+
+
+def run_block_step_only(args):
+    import torch
+
+    from __graft_entry__ import build
+
+    build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    peak, _ = _peaks()
+
+    def emit(d):
+        d["peak_gbs"] = peak
+        for k in list(d):
+            if k.endswith("_gbs") and k != "peak_gbs":
+                d[k.replace("_gbs", "_frac")] = d[k] / peak
+        print(json.dumps(d), flush=True)
+
+    run_block_step(emit, dev, max(3, args.steps))
 
 
 def run_graph(wl, step_bytes, reps: int = 10):
@@ -818,6 +894,8 @@ def main():
     ap.add_argument("--site-r", type=int, default=R, help="key rank r of the --profile-site case (not full)")
     ap.add_argument("--site-write", action="store_true", help="--profile-site: the backward writes the gradients")
     ap.add_argument("--suite", action="store_true", help="time every workload's headline site (JSON line each)")
+    ap.add_argument("--block-step", action="store_true",
+                    help="time only the Block AttnRes training step of the d = 2048 decoder (a --suite line)")
     ap.add_argument("--profile-block", type=int, default=0,
                     help="time the Block two-phase path on this many tokens (profiling)")
     ap.add_argument("--profile-proj", type=int, default=0,
@@ -825,6 +903,9 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.block_step:
+        run_block_step_only(args)
+        return
     if args.suite:
         run_suite(args)
     elif args.profile_site:

@@ -234,12 +234,21 @@ int lrar_block_accumulate(int dst_dtype, void *dst, int src_dtype, const void *s
  *               of a block the partial block is empty: use h_pre as h directly)
  *   partial_key [T, r] in_dtype: its projected key (LRAR_PROJECTED), else ignored
  *   query       [r] float32: the site's query
- *   h           [T, d] out_dtype, written; lse [T] float32, written when non-NULL
+ *   h           [T, d] out_dtype, written; lse [T] float32, written when non-NULL.
+ *               h may be h_pre and lse may be lse_pre (in place, pre_dtype ==
+ *               out_dtype): each element is read before it is written.
  * Other arguments and errors as for lrar_forward; LRAR_FULL is LRAR_ERR_UNSUPPORTED.
  */
 int lrar_block_phase1(int variant, int in_dtype, int pre_dtype, const void *values, const void *keys,
                       const float *queries, int n_completed, int n_sites, int64_t T, int d, int r, float eps,
                       void *h_pre, float *lse_pre, int *status, void *stream);
+/* Phase 1 with the completed sources as separate tensors: values (and, for
+ * LRAR_PROJECTED, keys) are HOST arrays of n_completed device pointers to [T, d]
+ * (keys: [T, r]) matrices, 16-byte aligned, read during the call (the rules of
+ * lrar_forward_ptrs).  Everything else as lrar_block_phase1. */
+int lrar_block_phase1_ptrs(int variant, int in_dtype, int pre_dtype, const void *const *values,
+                           const void *const *keys, const float *queries, int n_completed, int n_sites, int64_t T,
+                           int d, int r, float eps, void *h_pre, float *lse_pre, int *status, void *stream);
 int lrar_block_phase2(int variant, int in_dtype, int pre_dtype, int out_dtype, const void *h_pre,
                       const float *lse_pre, const void *partial, const void *partial_key, const float *query,
                       int64_t T, int d, int r, float eps, void *h, float *lse, void *stream);

@@ -404,7 +404,8 @@ LRAR_API int lrar_diagnostics(int variant, int in_dtype, const void *values, con
 
 namespace {
 
-int block_phase1_impl(int variant, int in_dtype, int pre_dtype, const void *values, const void *keys,
+// values / keys: stacked buffers (tables == false) or host arrays of n_completed pointers (tables == true).
+int block_phase1_impl(int variant, int in_dtype, int pre_dtype, const void *values, const void *keys, bool tables,
                       const float *queries, int n_completed, int n_sites, int64_t T, int d, int r, float eps,
                       void *h_pre, float *lse_pre, int *status, long long wait_cycles, bool stall, void *stream) {
     if (variant == LRAR_FULL)
@@ -419,15 +420,28 @@ int block_phase1_impl(int variant, int in_dtype, int pre_dtype, const void *valu
     if (!values || !queries || !h_pre || !lse_pre)
         return fail(LRAR_ERR_INVALID_ARG, "values, queries, h_pre and lse_pre are required");
     if (variant == LRAR_PROJECTED && !keys) return fail(LRAR_ERR_INVALID_ARG, "projected keys are required");
-    if (!aligned16(values) || !aligned16(h_pre) || (variant == LRAR_PROJECTED && !aligned16(keys)) ||
-        !aligned4(queries) || !aligned4(lse_pre))
+    const void *vt[LRAR_MAX_SOURCES], *kt[LRAR_MAX_SOURCES];
+    const void *const *vtab = vt, *const *ktab = kt;
+    if (tables) {
+        vtab = static_cast<const void *const *>(values);
+        ktab = static_cast<const void *const *>(keys);
+        int rc2 = check_table(vtab, n_completed, "values");
+        if (rc2) return rc2;
+        if (variant == LRAR_PROJECTED && (rc2 = check_table(ktab, n_completed, "keys"))) return rc2;
+    } else {
+        if (!aligned16(values) || (variant == LRAR_PROJECTED && !aligned16(keys)))
+            return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (queries and lse_pre 4-byte)");
+        stack_table(values, n_completed, T, d, esize(in_dtype), vt);
+        stack_table(variant == LRAR_PROJECTED ? keys : nullptr, n_completed, T, r, esize(in_dtype), kt);
+    }
+    if (!aligned16(h_pre) || !aligned4(queries) || !aligned4(lse_pre))
         return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (queries and lse_pre 4-byte)");
     lrar::BlockPh1Args a;
     a.variant = variant;
     a.in_dtype = in_dtype;
     a.pre_dtype = pre_dtype;
-    a.values = values;
-    a.keys = variant == LRAR_PROJECTED ? keys : nullptr;
+    a.values = vtab;
+    a.keys = variant == LRAR_PROJECTED ? ktab : nullptr;
     a.queries = queries;
     a.n = n_completed;
     a.c = n_sites;
@@ -452,8 +466,16 @@ int block_phase1_impl(int variant, int in_dtype, int pre_dtype, const void *valu
 LRAR_API int lrar_block_phase1(int variant, int in_dtype, int pre_dtype, const void *values, const void *keys,
                                const float *queries, int n_completed, int n_sites, int64_t T, int d, int r, float eps,
                                void *h_pre, float *lse_pre, int *status, void *stream) {
-    return block_phase1_impl(variant, in_dtype, pre_dtype, values, keys, queries, n_completed, n_sites, T, d, r, eps,
-                             h_pre, lse_pre, status, lrar::kWaitCycles, false, stream);
+    return block_phase1_impl(variant, in_dtype, pre_dtype, values, keys, false, queries, n_completed, n_sites, T, d,
+                             r, eps, h_pre, lse_pre, status, lrar::kWaitCycles, false, stream);
+}
+
+LRAR_API int lrar_block_phase1_ptrs(int variant, int in_dtype, int pre_dtype, const void *const *values,
+                                    const void *const *keys, const float *queries, int n_completed, int n_sites,
+                                    int64_t T, int d, int r, float eps, void *h_pre, float *lse_pre, int *status,
+                                    void *stream) {
+    return block_phase1_impl(variant, in_dtype, pre_dtype, values, keys, true, queries, n_completed, n_sites, T, d,
+                             r, eps, h_pre, lse_pre, status, lrar::kWaitCycles, false, stream);
 }
 
 LRAR_API int lrar_test_block_phase1_stalled(int variant, int in_dtype, int pre_dtype, const void *values,
@@ -463,8 +485,8 @@ LRAR_API int lrar_test_block_phase1_stalled(int variant, int in_dtype, int pre_d
     if (!status) return fail(LRAR_ERR_INVALID_ARG, "the stalled phase 1 reports through status: it is required");
     if (wait_cycles < 1 || wait_cycles > (1LL << 32))
         return fail(LRAR_ERR_INVALID_ARG, "wait_cycles must be in 1 .. 2^32");
-    return block_phase1_impl(variant, in_dtype, pre_dtype, values, keys, queries, n_completed, n_sites, T, d, r, eps,
-                             h_pre, lse_pre, status, wait_cycles, true, stream);
+    return block_phase1_impl(variant, in_dtype, pre_dtype, values, keys, false, queries, n_completed, n_sites, T, d,
+                             r, eps, h_pre, lse_pre, status, wait_cycles, true, stream);
 }
 
 LRAR_API int lrar_block_phase2(int variant, int in_dtype, int pre_dtype, int out_dtype, const void *h_pre,

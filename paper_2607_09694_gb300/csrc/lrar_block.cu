@@ -13,11 +13,14 @@
 //            h = exp(lse_j - lse) h_pre_j + exp(s_P - lse) b_P.
 //
 // The result is the site's mix over [completed sources, b_P] (Eq. 8-10).
+//
 // Phase 1 tiles a token's row over the warps of a group: warp (g, ch) of a CTA
-// owns the 32 x 16-byte chunk ch of token g's rows and keeps c accumulators per
-// element.  The chunk warps split the c queries for scoring and share the
-// weights through shared memory (double-buffered, one named barrier per pass),
-// and each pass scores the next token while the current token's rows load.
+// owns the 32 x 16-byte chunk ch of token g's rows and keeps up to 8
+// accumulators per element, one per site, so every row read serves all the
+// block's sites.  The chunk warps split the c queries for scoring, each lane
+// working on one (source, key vector) pair, and score the group's next token
+// while its rows load; the weights pass through shared memory,
+// double-buffered, behind one named barrier per token.
 #include "lrar.h"
 #include "lrar_device.cuh"
 #include "lrar_launch.h"
@@ -26,10 +29,11 @@
 namespace lrar {
 
 constexpr int kPh1MaxSites = 8;  // queries per phase-1 launch (more are split by the host)
-constexpr int kPh1Stages = 12;   // ring depth of phase 1 (rows in flight per lane + 1)
+constexpr int kPh1Stages = 16;   // ring depth of phase 1 (rows in flight per lane + 1; a power of two)
+static_assert((kPh1Stages & (kPh1Stages - 1)) == 0, "the ring index wraps with a mask");
 
 struct Ph1Params {
-    const void *values, *keys;
+    SrcTab vt, kt;         // completed sources [T, d] each; P-LR keys [T, r] each
     const float *queries;  // [c][r]
     void *h_pre;           // [c][T][d]
     float *lse_pre;        // [c][T]
@@ -46,63 +50,17 @@ __device__ __forceinline__ void group_sync(int id, int threads) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
-// Scores of token x for the queries j = ch, ch + chunks, ... (Eq. 8-9): lane i
-// takes source i; then the softmax of each of those queries over the n sources.
-// Weights go to aw[j * n + i], lse_j to the output.
+// Key of source i at token x: the last r coordinates of the row (S-LR, Eq. 14)
+// or the P-LR key row.
 template <typename Tin>
-__device__ __forceinline__ float ph1_dot(const Tin *__restrict__ kp, const float *__restrict__ qj, int r, bool vec,
-                                         float *ss) {
-    constexpr int E = VecE<Tin>::value;
-    float qk = 0.f, s2 = 0.f;
-    if (vec) {
-#pragma unroll 4
-        for (int jj = 0; jj < r; jj += E) {
-            Frag<Tin, E> f;
-            f.load_nc(kp + jj);
-            float k[E];
-            f.get(k);
-#pragma unroll
-            for (int t = 0; t < E; ++t) {
-                s2 = fmaf(k[t], k[t], s2);
-                qk = fmaf(qj[jj + t], k[t], qk);
-            }
-        }
-    } else {
-        for (int jj = 0; jj < r; ++jj) {
-            const float k = to_f(__ldg(kp + jj));
-            s2 = fmaf(k, k, s2);
-            qk = fmaf(qj[jj], k, qk);
-        }
-    }
-    if (ss) *ss = s2;
-    return qk;
-}
-
-// The same over a key staged in shared memory (whole 16-byte vectors).
-template <typename Tin>
-__device__ __forceinline__ float ph1_dot_s(const Tin *kp, const float *__restrict__ qj, int r, float *ss) {
-    constexpr int E = VecE<Tin>::value;
-    float qk = 0.f, s2 = 0.f;
-#pragma unroll 4
-    for (int jj = 0; jj < r; jj += E) {
-        Frag<Tin, E> f;
-        f.a = *reinterpret_cast<const uint4 *>(kp + jj);
-        float k[E];
-        f.get(k);
-#pragma unroll
-        for (int t = 0; t < E; ++t) {
-            s2 = fmaf(k[t], k[t], s2);
-            qk = fmaf(qj[jj + t], k[t], qk);
-        }
-    }
-    if (ss) *ss = s2;
-    return qk;
+__device__ __forceinline__ const Tin *ph1_key(const Ph1Params &p, int i, int64_t x) {
+    return p.sliced ? src_row<Tin>(p.vt, i, x, p.d) + (p.d - p.r) : src_row<Tin>(p.kt, i, x, p.r);
 }
 
 // Staged keys of one token: key i at byte i * kstride of a group's buffer
 // (r * sizeof(Tin) bytes, then 16 bytes of padding against bank conflicts).
 template <typename Tin>
-__device__ __forceinline__ int ph1_kstride(int r) {
+__host__ __device__ __forceinline__ int ph1_kstride(int r) {
     return r * (int)sizeof(Tin) + 16;
 }
 
@@ -110,45 +68,101 @@ __device__ __forceinline__ int ph1_kstride(int r) {
 // (one warp: lane 0 announces the bytes, lane i copies key i).
 template <typename Tin>
 __device__ __forceinline__ void ph1_stage(const Ph1Params &p, int64_t x, int lane, uint32_t kbuf, uint32_t bar) {
-    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
-    const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
     const uint32_t kbytes = (uint32_t)(p.r * (int)sizeof(Tin));
     if (lane == 0) sm100::mbar_arrive_expect_tx(bar, kbytes * (uint32_t)p.n);
     __syncwarp();
-    for (int i = lane; i < p.n; i += 32) {
-        const Tin *kp = p.sliced ? values + ((int64_t)i * p.T + x) * p.d + (p.d - p.r)
-                                 : keys + ((int64_t)i * p.T + x) * p.r;
-        sm100::bulk_load(kbuf + (uint32_t)(i * ph1_kstride<Tin>(p.r)), kp, kbytes, bar);
+    for (int i = lane; i < p.n; i += 32)
+        sm100::bulk_load(kbuf + (uint32_t)(i * ph1_kstride<Tin>(p.r)), ph1_key<Tin>(p, i, x), kbytes, bar);
+}
+
+// Scores of token x for QW queries j = j0, j0 + jstep, ... (Eq. 8-9), by one
+// warp: s_ij goes to aw[i * kPh1MaxSites + j].  Keys that are whole 16-byte
+// vectors and whose row of nv = r / E vectors divides a warp are scored lane
+// per (source, key vector): each lane forms its vector's part of |k_i|^2 and of
+// q_j . k_i, and the nv lanes of a source combine them with a fixed butterfly.
+// Other keys take a lane per source.  kb_s: the token's keys staged in shared
+// memory (null: read from global memory).
+template <typename Tin, int QW>
+__device__ __forceinline__ void ph1_scores(const Ph1Params &p, const float *__restrict__ q_s, int rp, int64_t x,
+                                           int lane, int j0, int jstep, float *aw, const unsigned char *kb_s) {
+    constexpr int E = VecE<Tin>::value;
+    const int nv = p.r / E;
+    if (p.key_vec && nv <= 32 && (32 % nv) == 0) {
+        const int per = 32 / nv;  // sources per round
+        const int v = lane % nv;
+        for (int i0 = 0; i0 < p.n; i0 += per) {
+            const int i = i0 + lane / nv;
+            float k[E];
+            if (i < p.n) {
+                Frag<Tin, E> f;
+                if (kb_s) f.a = *reinterpret_cast<const uint4 *>(kb_s + i * ph1_kstride<Tin>(p.r) + v * 16);
+                else f.load_nc(ph1_key<Tin>(p, i, x) + v * E);
+                f.get(k);
+            } else {
+#pragma unroll
+                for (int t = 0; t < E; ++t) k[t] = 0.f;
+            }
+            float ss = 0.f, qk[QW];
+#pragma unroll
+            for (int t = 0; t < E; ++t) ss = fmaf(k[t], k[t], ss);
+#pragma unroll
+            for (int u = 0; u < QW; ++u) {
+                qk[u] = 0.f;
+                const float *qj = q_s + (j0 + u * jstep) * rp + v * E;
+#pragma unroll
+                for (int t = 0; t < E; t += 4) {
+                    const float4 q4 = *reinterpret_cast<const float4 *>(qj + t);
+                    qk[u] = fmaf(q4.x, k[t], qk[u]);
+                    qk[u] = fmaf(q4.y, k[t + 1], qk[u]);
+                    qk[u] = fmaf(q4.z, k[t + 2], qk[u]);
+                    qk[u] = fmaf(q4.w, k[t + 3], qk[u]);
+                }
+            }
+            for (int off = 1; off < nv; off <<= 1) {  // the source's lanes form an aligned group
+                ss += __shfl_xor_sync(0xffffffffu, ss, off);
+#pragma unroll
+                for (int u = 0; u < QW; ++u) qk[u] += __shfl_xor_sync(0xffffffffu, qk[u], off);
+            }
+            if (v == 0 && i < p.n) {
+                const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
+#pragma unroll
+                for (int u = 0; u < QW; ++u) aw[i * kPh1MaxSites + j0 + u * jstep] = rho * qk[u];
+            }
+        }
+    } else {
+        for (int i = lane; i < p.n; i += 32) {
+            const Tin *kp = ph1_key<Tin>(p, i, x);
+            float ss = 0.f, qk[QW];
+#pragma unroll
+            for (int u = 0; u < QW; ++u) qk[u] = 0.f;
+            for (int t = 0; t < p.r; ++t) {
+                const float kt = to_f(__ldg(kp + t));
+                ss = fmaf(kt, kt, ss);
+#pragma unroll
+                for (int u = 0; u < QW; ++u) qk[u] = fmaf(q_s[(j0 + u * jstep) * rp + t], kt, qk[u]);
+            }
+            const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
+#pragma unroll
+            for (int u = 0; u < QW; ++u) aw[i * kPh1MaxSites + j0 + u * jstep] = rho * qk[u];
+        }
     }
 }
 
-// Scores of token x for the queries j = ch, ch + chunks, ... (Eq. 8-9): lane i
-// takes source i, reading its key from kb_s (staged) or global memory; then the
-// softmax of each of those queries over the n sources.  Weights go to
-// aw[i * kPh1MaxSites + j] (a source's weights for every query side by side),
-// lse_j to the output.
+// Scores and softmax of token x for this warp's queries j = ch, ch + chunks,
+// ... < c (the chunk warps of a group share the queries): weights alpha_ij to
+// aw[i * kPh1MaxSites + j], lse_j to lse_pre.
 template <typename Tin>
-__device__ __forceinline__ void ph1_score(const Ph1Params &p, const float *__restrict__ q_s, int rp, int64_t x,
-                                          int ch, int lane, float *aw, const unsigned char *kb_s = nullptr) {
-    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
-    const Tin *__restrict__ keys = static_cast<const Tin *>(p.keys);
-    if (ch < p.c)
-        for (int i = lane; i < p.n; i += 32) {
-            float ss, qk0;
-            const Tin *kp;
-            if (kb_s) {
-                kp = reinterpret_cast<const Tin *>(kb_s + i * ph1_kstride<Tin>(p.r));
-                qk0 = ph1_dot_s<Tin>(kp, q_s + ch * rp, p.r, &ss);
-            } else {
-                kp = p.sliced ? values + ((int64_t)i * p.T + x) * p.d + (p.d - p.r) : keys + ((int64_t)i * p.T + x) * p.r;
-                qk0 = ph1_dot<Tin>(kp, q_s + ch * rp, p.r, p.key_vec != 0, &ss);
-            }
-            const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
-            aw[i * kPh1MaxSites + ch] = rho * qk0;
-            for (int j = ch + p.chunks; j < p.c; j += p.chunks)  // further queries of this warp (small d)
-                aw[i * kPh1MaxSites + j] = rho * (kb_s ? ph1_dot_s<Tin>(kp, q_s + j * rp, p.r, nullptr)
-                                              : ph1_dot<Tin>(kp, q_s + j * rp, p.r, p.key_vec != 0, nullptr));
-        }
+__device__ __forceinline__ void ph1_score_warp(const Ph1Params &p, const float *__restrict__ q_s, int rp, int64_t x,
+                                               int ch, int lane, float *aw, const unsigned char *kb_s) {
+    const int nq = ch < p.c ? (p.c - ch + p.chunks - 1) / p.chunks : 0;
+    switch (nq) {  // queries of this warp: 8 / chunks when c = 8
+        case 0: break;
+        case 1: ph1_scores<Tin, 1>(p, q_s, rp, x, lane, ch, p.chunks, aw, kb_s); break;
+        case 2: ph1_scores<Tin, 2>(p, q_s, rp, x, lane, ch, p.chunks, aw, kb_s); break;
+        case 3: ph1_scores<Tin, 3>(p, q_s, rp, x, lane, ch, p.chunks, aw, kb_s); break;
+        case 4: ph1_scores<Tin, 4>(p, q_s, rp, x, lane, ch, p.chunks, aw, kb_s); break;
+        default: ph1_scores<Tin, 8>(p, q_s, rp, x, lane, ch, p.chunks, aw, kb_s); break;  // 5..8: chunks == 1
+    }
     __syncwarp();
     for (int j = ch; j < p.c; j += p.chunks) {
         float m = -INFINITY;
@@ -157,50 +171,58 @@ __device__ __forceinline__ void ph1_score(const Ph1Params &p, const float *__res
         float z = 0.f;
         for (int i = lane; i < p.n; i += 32) z += expf(aw[i * kPh1MaxSites + j] - m);
         z = warp_sum(z);
-        __syncwarp();
         for (int i = lane; i < p.n; i += 32) aw[i * kPh1MaxSites + j] = expf(aw[i * kPh1MaxSites + j] - m) / z;
         if (lane == 0) p.lse_pre[(int64_t)j * p.T + x] = m + logf(z);
-        __syncwarp();
     }
+    __syncwarp();
 }
 
-// Rows stream through a per-lane cp.async ring (each lane copies and reads
-// back its own 16-byte vector of every row), S - 1 rows ahead and across
-// tokens, so the loads of the next token's rows overlap this token's mix.
-// KS: each group's keys are staged two tokens ahead in shared memory with
-// bulk copies (double-buffered, one mbarrier per buffer), so scoring reads no
-// global memory.  Each wait for them is bounded (p.wait_cycles) and decided
-// for the whole warp; one that runs out ORs LRAR_STATUS_WAIT_TIMEOUT into
-// *p.status and raises the CTA's abort flag, after which no warp waits again
-// and no group issues another copy (a group's copy into a buffer follows the
-// barrier that ends the pass in which its warps waited for that buffer's
-// previous token, so a give-up is seen before the buffer is reused).  The
-// issuing warp counts the phases it issued and saw complete per buffer (at
-// most one per buffer is left unconfirmed after a give-up) and waits, bounded,
-// for that one before the CTA exits, so no copy lands in freed shared memory.
-// The outputs of a launch that gave up are not valid.
-// C8: exactly eight sites per launch (compile-time loop bounds); else p.c <= 8.
-template <typename Tin, typename Tout, int S, bool KS, bool C8>
+// Phase 1 (§3.5): per token of a group, the group's warps mix its n rows into
+// c sites and score the group's next token, each warp its share of the queries.
+//   Rows stream through a per-lane cp.async ring (each lane copies and reads
+//   back its own 16-byte vector of every row), S - 1 rows ahead and across
+//   tokens, so the next token's rows travel while this one is mixed.
+//   KS: each group's keys are staged two tokens ahead in shared memory with
+//   bulk copies (double-buffered, one mbarrier per buffer) by the group's warp
+//   0, so scoring reads no global memory.  Each warp's wait for them is
+//   bounded (p.wait_cycles) and decided for the whole warp; one that runs out
+//   ORs LRAR_STATUS_WAIT_TIMEOUT into *p.status and raises the CTA's abort
+//   flag, after which no warp waits again and no group issues another copy.
+//   A copy into a buffer follows the barrier that ends the pass in which its
+//   previous token was waited for, so a give-up is always seen before the
+//   buffer is reused, and each buffer holds at most one phase that no wait
+//   confirmed; the issuing warp waits (bounded) for that one before the CTA
+//   exits, so no copy lands in released shared memory.  A launch that gave up
+//   writes outputs that are not valid.
+//   C8: exactly eight sites (compile-time loop bounds); else p.c <= 8.
+//   FULLW: every lane's vector lies inside the row (d = chunks * 32 * E).
+template <typename Tin, typename Tout, int S, bool KS, bool C8, bool FULLW>
 __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_constant__ Ph1Params p) {
     constexpr int E = VecE<Tin>::value;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int rp = round_up(p.r, 4);
-    const int G_ = kWarps / p.chunks;
+    const int G = kWarps / p.chunks;  // token groups per CTA
     const int kbuf_bytes = KS ? round_up(p.n * ph1_kstride<Tin>(p.r), 16) : 0;  // one token's keys
     unsigned char *kb_all = smem_raw + (size_t)kWarps * S * 32 * 16;           // [G][2][kbuf_bytes]
-    uint64_t *kbar_all = reinterpret_cast<uint64_t *>(kb_all + (size_t)G_ * 2 * kbuf_bytes);  // [G][2]
-    float *q_s = reinterpret_cast<float *>(kbar_all + (KS ? 2 * G_ : 0));       // [c][r]
-    float *a_all = q_s + kPh1MaxSites * rp;  // [G][2][n][kPh1MaxSites]: weights, double-buffered by pass
+    uint64_t *kbar_all = reinterpret_cast<uint64_t *>(kb_all + (size_t)G * 2 * kbuf_bytes);  // [G][2]
+    int *conf_all = reinterpret_cast<int *>(kbar_all + (KS ? 2 * G : 0));     // [G][2] phases seen complete
+    // q_s starts 16-byte aligned: the barriers and counters take round_up(G * 2 * 12, 16) bytes
+    float *q_s = reinterpret_cast<float *>(reinterpret_cast<unsigned char *>(kbar_all) +
+                                           (KS ? round_up(G * 2 * (8 + 4), 16) : 0));  // [8][rp], zero past c and r
+    float *a_all = q_s + kPh1MaxSites * rp;  // [G][2][n][8]: weights, double-buffered by token
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int G = kWarps / p.chunks;  // tokens per CTA pass
     const int g = warp / p.chunks, ch = warp % p.chunks;
-    const int nthr = p.chunks * 32;   // threads of a token group (named barrier 1 + g)
+    const int nthr = p.chunks * 32;  // threads of a token group (named barrier 1 + g)
     __shared__ int abort_s;           // set once a key wait of this CTA gave up
     __shared__ __align__(8) uint64_t never_bar;  // test hook: a barrier nothing arrives on
     volatile int *abort = &abort_s;
-    for (int j = threadIdx.x; j < p.c * p.r; j += kThreads) q_s[(j / p.r) * rp + j % p.r] = p.queries[j];
+    for (int j = threadIdx.x; j < kPh1MaxSites * rp; j += kThreads) {
+        const int jj = j / rp, t = j % rp;
+        q_s[j] = (jj < p.c && t < p.r) ? p.queries[jj * p.r + t] : 0.f;
+    }
     if (KS && threadIdx.x < 2 * G) {
         sm100::mbar_init(smem_u32(kbar_all + threadIdx.x), 1);
+        conf_all[threadIdx.x] = 0;
         sm100::mbar_fence_init();
     }
     if (threadIdx.x == 0) {
@@ -212,47 +234,46 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
     }
     __syncthreads();
 
-    const Tin *__restrict__ values = static_cast<const Tin *>(p.values);
     Tout *__restrict__ h_pre = static_cast<Tout *>(p.h_pre);
     const int e = (ch * 32 + lane) * E;  // this lane's first element of the row
     float *aw0 = a_all + (size_t)g * 2 * kPh1MaxSites * p.n;
     const int64_t stride = (int64_t)gridDim.x * G;
     const uint32_t ring_w = smem_u32(smem_raw) + (uint32_t)(warp * S * 32 * 16) + 16u * lane;
     unsigned char *kb0 = kb_all + (size_t)g * 2 * kbuf_bytes;
+    int *conf = conf_all + 2 * g;
     auto kbuf = [&](int b) { return smem_u32(kb0 + b * kbuf_bytes); };
     auto kbar = [&](int b) { return smem_u32(kbar_all + 2 * g + b); };
-    // token q of this group (x0 + q * stride) uses key buffer q % 2, for the (q / 2)-th time;
-    // the issuing warp (ch == 0) counts phases issued and seen complete per buffer
-    uint32_t issued0 = 0u, issued1 = 0u, seen0 = 0u, seen1 = 0u;
+    // token q of this group (x0 + q * stride) uses key buffer q % 2, for the (q / 2)-th time
     auto kwait = [&](int q) {
-        if (__any_sync(0xffffffffu, *abort != 0)) return;  // the CTA gave up: no further waits (warp-uniform)
+        if (__any_sync(0xffffffffu, *abort != 0)) return;  // the CTA gave up: no further waits
         const uint32_t bar = p.stall ? smem_u32(&never_bar) : kbar(q & 1);
         const uint32_t par = p.stall ? 0u : (uint32_t)(q >> 1) & 1u;
-        const bool ok = __all_sync(0xffffffffu, sm100::mbar_wait(bar, par, p.wait_cycles, abort));
-        if (ok) {
-            if (ch == 0) {
-                if (q & 1) seen1 = (uint32_t)(q >> 1) + 1u;
-                else seen0 = (uint32_t)(q >> 1) + 1u;
-            }
+        if (__all_sync(0xffffffffu, sm100::mbar_wait(bar, par, p.wait_cycles, abort))) {
+            if (lane == 0 && ch == 0) conf[q & 1] = (q >> 1) + 1;
         } else if (lane == 0) {
             *abort = 1;
             if (p.status) atomicOr(p.status, LRAR_STATUS_WAIT_TIMEOUT);
         }
     };
-    // the issuing warp stages token xx into buffer b unless the CTA gave up (warp-uniform)
-    auto stage = [&](int64_t xx, int b) {
+    uint32_t issued0 = 0u, issued1 = 0u;  // the issuing warp's phases per buffer
+    auto stage = [&](int64_t xx, int b) {  // warp 0 of the group, unless the CTA gave up
         if (__any_sync(0xffffffffu, *abort != 0)) return;
         ph1_stage<Tin>(p, xx, lane, kbuf(b), kbar(b));
         if (b) ++issued1;
         else ++issued0;
     };
+    auto score = [&](int q, int64_t xx, float *aw) {  // token q = xx of the group: this warp's queries
+        if (KS) kwait(q);
+        ph1_score_warp<Tin>(p, q_s, rp, xx, ch, lane, aw, KS ? kb0 + (q & 1) * kbuf_bytes : nullptr);
+    };
 
     int64_t x = (int64_t)blockIdx.x * G + g;
-    int64_t ix = x;  // next row to copy: source ii of token ix
+    // the ring: row ii of token ix is the next to copy
+    int64_t ix = x;
     int ii = 0;
     auto issue = [&](int st) {
         if (ix < p.T) {
-            if (e < p.d) cp_async16(ring_w + 16u * 32u * st, values + ((int64_t)ii * p.T + ix) * p.d + e);
+            if (FULLW || e < p.d) cp_async16(ring_w + 16u * 32u * st, src_row<Tin>(p.vt, ii, ix, p.d) + e);
             if (++ii == p.n) {
                 ii = 0;
                 ix += stride;
@@ -262,26 +283,19 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
     };
 #pragma unroll
     for (int st = 0; st < S - 1; ++st) issue(st);
-    int st_c = 0, st_i = S - 1;
+    int st = 0;  // ring slot of the next row to mix; slot st - 1 (mod S) is refilled
 
     if (KS && ch == 0) {
         if (x < p.T) stage(x, 0);
         if (x + stride < p.T) stage(x + stride, 1);
     }
-    if (x < p.T) {
-        if (KS) kwait(0);
-        ph1_score<Tin>(p, q_s, rp, x, ch, lane, aw0, KS ? kb0 : nullptr);
-    }
+    if (x < p.T) score(0, x, aw0);
     group_sync(1 + g, nthr);
     for (int pass = 0; (int64_t)blockIdx.x * G + pass * stride < p.T; ++pass, x += stride) {
         const float *aw = aw0 + (pass & 1) * kPh1MaxSites * p.n;
-        float *aw_next = aw0 + ((pass + 1) & 1) * kPh1MaxSites * p.n;
-        // buffer pass % 2 held token `pass`, scored by every warp before the last barrier
+        // buffer pass % 2 held token `pass`, scored before the last barrier
         if (KS && ch == 0 && x + 2 * stride < p.T) stage(x + 2 * stride, pass & 1);
-        if (x + stride < p.T) {
-            if (KS) kwait(pass + 1);
-            ph1_score<Tin>(p, q_s, rp, x + stride, ch, lane, aw_next, KS ? kb0 + ((pass + 1) & 1) * kbuf_bytes : nullptr);
-        }
+        if (x + stride < p.T) score(pass + 1, x + stride, aw0 + ((pass + 1) & 1) * kPh1MaxSites * p.n);
         if (x < p.T) {
             float acc[kPh1MaxSites][E];
 #pragma unroll
@@ -289,13 +303,12 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
 #pragma unroll
                 for (int t = 0; t < E; ++t) acc[j][t] = 0.f;
             for (int i = 0; i < p.n; ++i) {
-                issue(st_i);
+                issue((st + S - 1) & (S - 1));
                 cp_async_wait<S - 1>();  // this lane's copy of row i has landed
                 Frag<Tin, E> f;
-                if (e < p.d) f.a = ld_shared16(ring_w + 16u * 32u * st_c);
+                if (FULLW || e < p.d) f.a = ld_shared16(ring_w + 16u * 32u * st);
                 else f.zero();
-                st_c = (st_c + 1 == S) ? 0 : st_c + 1;
-                st_i = (st_i + 1 == S) ? 0 : st_i + 1;
+                st = (st + 1) & (S - 1);
                 float o[E], w[kPh1MaxSites];
                 f.get(o);
                 const float4 w0 = *reinterpret_cast<const float4 *>(aw + i * kPh1MaxSites);
@@ -309,13 +322,14 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
                     }
                 }
             }
-            if (e < p.d) {
+            if (FULLW || e < p.d) {
+                Tout *hp = h_pre + x * p.d + e;
 #pragma unroll
                 for (int j = 0; j < kPh1MaxSites; ++j) {
                     if (C8 || j < p.c) {
                         Frag<Tout, E> out;
                         out.set(acc[j]);
-                        out.store(h_pre + (int64_t)j * p.site_stride + x * p.d + e);
+                        out.store(hp + (int64_t)j * p.site_stride);
                     }
                 }
             }
@@ -325,7 +339,7 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
     cp_async_wait_all();
     if (KS && ch == 0)  // drain: the one phase per buffer a give-up may have left unconfirmed
         for (int b = 0; b < 2; ++b) {
-            const uint32_t iss = b ? issued1 : issued0, done = b ? seen1 : seen0;
+            const uint32_t iss = b ? issued1 : issued0, done = (uint32_t)conf[b];
             if (iss > done && !__all_sync(0xffffffffu, sm100::mbar_wait(kbar(b), (iss - 1u) & 1u, p.wait_cycles)) &&
                 lane == 0 && p.status)
                 atomicOr(p.status, LRAR_STATUS_WAIT_TIMEOUT);
@@ -344,14 +358,16 @@ struct Ph2Params {
 };
 
 // Phase 2: one warp per token merges h_pre with the partial-block summary.
+// Each lane reads its elements of h_pre (and lane 0 lse_pre) before it writes
+// the same elements of h (and lse), so h may be h_pre and lse may be lse_pre.
 template <typename Tin, typename Tp, typename Tout, int V>
 __global__ void __launch_bounds__(kThreads) block_phase2_kernel(const Ph2Params p) {
     constexpr int E = VecE<Tin>::value;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const Tin *__restrict__ part = static_cast<const Tin *>(p.partial);
     const Tin *__restrict__ pkeys = static_cast<const Tin *>(p.pkeys);
-    const Tp *__restrict__ h_pre = static_cast<const Tp *>(p.h_pre);
-    Tout *__restrict__ h = static_cast<Tout *>(p.h);
+    const Tp *h_pre = static_cast<const Tp *>(p.h_pre);  // may alias h: no __restrict__
+    Tout *h = static_cast<Tout *>(p.h);
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     for (int64_t x = (int64_t)blockIdx.x * kWarps + warp; x < p.T; x += nwarps) {
         // both rows first: their loads travel while the partial summary is scored
@@ -362,7 +378,7 @@ __global__ void __launch_bounds__(kThreads) block_phase2_kernel(const Ph2Params 
             const int e = (lane + 32 * v) * E;
             if (e < p.d) {
                 fb[v].load_nc(part + x * p.d + e);
-                fh[v].load_nc(h_pre + x * p.d + e);
+                fh[v].load(h_pre + x * p.d + e);  // coherent: h may be h_pre (in place)
             } else {
                 fb[v].zero();
                 fh[v].zero();
@@ -398,7 +414,7 @@ __global__ void __launch_bounds__(kThreads) block_phase2_kernel(const Ph2Params 
         ss = warp_sum(ss);
         qk = warp_sum(qk);
         const float sP = rsqrtf(fmaf(ss, p.inv_r, p.eps)) * qk;
-        const float lp = __ldg(p.lse_pre + x);
+        const float lp = p.lse_pre[x];  // coherent: lse may be lse_pre (in place)
         const float M = fmaxf(lp, sP);
         const float lse = M + logf(expf(lp - M) + expf(sP - M));
         const float w1 = expf(lp - lse), w2 = expf(sP - lse);
@@ -420,19 +436,23 @@ __global__ void __launch_bounds__(kThreads) block_phase2_kernel(const Ph2Params 
     }
 }
 
+
 // --------------------------------------------------------------- launch ----
 // Keys as whole 16-byte vectors (vector loads, and bulk copies when staged).
 template <typename Tin>
 static bool ph1_key_vec(const BlockPh1Args &a) {
     constexpr int esz = sizeof(Tin);
-    return (a.r * esz) % 16 == 0 && (a.variant == kSliced ? ((a.d - a.r) * esz) % 16 == 0
-                                                          : (reinterpret_cast<uintptr_t>(a.keys) & 15) == 0);
+    if ((a.r * esz) % 16) return false;
+    if (a.variant == kSliced) return ((a.d - a.r) * esz) % 16 == 0;
+    for (int i = 0; i < a.n; ++i)  // every key matrix (the API checks 16-byte alignment of the tables)
+        if (reinterpret_cast<uintptr_t>(a.keys[i]) & 15) return false;
+    return true;
 }
 
 // A token's keys are staged in shared memory when they are whole vectors and fit 4 KB.
 template <typename Tin>
 static bool ph1_stages_keys_t(const BlockPh1Args &a) {
-    const size_t kbuf_bytes = (size_t)round_up(a.n * (a.r * (int)sizeof(Tin) + 16), 16);
+    const size_t kbuf_bytes = (size_t)round_up(a.n * ph1_kstride<Tin>(a.r), 16);
     return ph1_key_vec<Tin>(a) && kbuf_bytes <= 4096;
 }
 
@@ -440,15 +460,32 @@ bool block_phase1_stages_keys(const BlockPh1Args &a) {
     return a.in_dtype == kBF16 ? ph1_stages_keys_t<bf16>(a) : ph1_stages_keys_t<float>(a);
 }
 
+// Dynamic shared memory of a phase-1 launch (layout of block_phase1_kernel).
+static size_t ph1_smem(int S, bool ks, int G, int n, int r, int kstride) {
+    const size_t kbuf = ks ? (size_t)round_up(n * kstride, 16) : 0;
+    return (size_t)kWarps * S * 32 * 16 + (size_t)G * 2 * kbuf + (ks ? (size_t)round_up(G * 2 * (8 + 4), 16) : 0) +
+           sizeof(float) * ((size_t)kPh1MaxSites * round_up(r, 4) + (size_t)G * 2 * kPh1MaxSites * n);
+}
+
+template <typename Tin, typename Tout, bool KS, bool FAST>
+static cudaError_t ph1_go(const Ph1Params &p, int grid, size_t smem, cudaStream_t s) {
+    constexpr int S = kPh1Stages;
+    block_phase1_kernel<Tin, Tout, S, KS, FAST, FAST><<<grid, kThreads, smem, s>>>(p);
+    return cudaGetLastError();
+}
+
 template <typename Tin, typename Tout>
 static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
     constexpr int E = VecE<Tin>::value;
+    constexpr int S = kPh1Stages;
     const int chunks_needed = (a.d + 32 * E - 1) / (32 * E);
     int chunks = 1;
     while (chunks < chunks_needed) chunks *= 2;  // 1, 2, 4 or 8 (validated: d <= 8 * 32 * E)
     Ph1Params p;
-    p.values = a.values;
-    p.keys = a.keys;
+    for (int i = 0; i < kMaxTab; ++i) {
+        p.vt.p[i] = i < a.n ? a.values[i] : nullptr;
+        p.kt.p[i] = (i < a.n && a.keys) ? a.keys[i] : nullptr;
+    }
     p.T = a.T;
     p.site_stride = a.T * (int64_t)a.d;
     p.n = a.n;
@@ -463,36 +500,29 @@ static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
     p.stall = a.stall ? 1 : 0;
     p.key_vec = ph1_key_vec<Tin>(a);
     const int G = kWarps / chunks;
-    constexpr int S = kPh1Stages;
-    const int kstride = a.r * (int)sizeof(Tin) + 16;
-    const size_t kbuf_bytes = (size_t)round_up(a.n * kstride, 16);
     const bool ks = ph1_stages_keys_t<Tin>(a);  // keys staged in shared memory
-    const size_t smem = (size_t)kWarps * S * 32 * 16 + (ks ? (size_t)G * 2 * (kbuf_bytes + 8) : 0) +
-                        sizeof(float) * ((size_t)kPh1MaxSites * round_up(a.r, 4) + (size_t)G * 2 * kPh1MaxSites * a.n);
-    const void *k = ks ? (const void *)block_phase1_kernel<Tin, Tout, S, true, true>
-                       : (const void *)block_phase1_kernel<Tin, Tout, S, false, true>;  // same resources for C8 or not
-    if (smem > 48 * 1024) {  // every variant this call may launch (8 sites, or the rest)
-        const void *ks_all[4] = {(const void *)block_phase1_kernel<Tin, Tout, S, true, true>,
-                                 (const void *)block_phase1_kernel<Tin, Tout, S, true, false>,
-                                 (const void *)block_phase1_kernel<Tin, Tout, S, false, true>,
-                                 (const void *)block_phase1_kernel<Tin, Tout, S, false, false>};
-        for (const void *kk : ks_all) {
+    const bool fullw = a.d == chunks * 32 * E;  // every lane's vector inside the row
+    const size_t smem = ph1_smem(S, ks, G, a.n, a.r, ph1_kstride<Tin>(a.r));
+    // every variant this call may launch: 8 sites on whole rows (fast), or the rest
+    const void *k_fast = ks ? (const void *)block_phase1_kernel<Tin, Tout, S, true, true, true>
+                            : (const void *)block_phase1_kernel<Tin, Tout, S, false, true, true>;
+    const void *k_gen = ks ? (const void *)block_phase1_kernel<Tin, Tout, S, true, false, false>
+                           : (const void *)block_phase1_kernel<Tin, Tout, S, false, false, false>;
+    if (smem > 48 * 1024)
+        for (const void *kk : {k_fast, k_gen}) {
             cudaError_t e = cudaFuncSetAttribute(kk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
             if (e != cudaSuccess) return e;
         }
-    }
-    const int grid = persistent_grid(k, kThreads, smem, (a.T + G - 1) / G, 1 << 30);
+    const int grid = persistent_grid(k_gen, kThreads, smem, (a.T + G - 1) / G, 1 << 30);
     for (int j0 = 0; j0 < a.c; j0 += kPh1MaxSites) {  // groups of at most 8 queries
         p.c = a.c - j0 < kPh1MaxSites ? a.c - j0 : kPh1MaxSites;
         p.queries = a.queries + (size_t)j0 * a.r;
         p.h_pre = static_cast<char *>(a.h_pre) + (size_t)j0 * p.site_stride * sizeof(Tout);
         p.lse_pre = a.lse_pre + (size_t)j0 * a.T;
-        const bool c8 = p.c == kPh1MaxSites;
-        if (ks && c8) block_phase1_kernel<Tin, Tout, S, true, true><<<grid, kThreads, smem, s>>>(p);
-        else if (ks) block_phase1_kernel<Tin, Tout, S, true, false><<<grid, kThreads, smem, s>>>(p);
-        else if (c8) block_phase1_kernel<Tin, Tout, S, false, true><<<grid, kThreads, smem, s>>>(p);
-        else block_phase1_kernel<Tin, Tout, S, false, false><<<grid, kThreads, smem, s>>>(p);
-        cudaError_t e = cudaGetLastError();
+        const bool fast = p.c == kPh1MaxSites && fullw;
+        cudaError_t e;
+        if (ks) e = fast ? ph1_go<Tin, Tout, true, true>(p, grid, smem, s) : ph1_go<Tin, Tout, true, false>(p, grid, smem, s);
+        else e = fast ? ph1_go<Tin, Tout, false, true>(p, grid, smem, s) : ph1_go<Tin, Tout, false, false>(p, grid, smem, s);
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;

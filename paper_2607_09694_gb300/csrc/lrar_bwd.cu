@@ -1055,6 +1055,244 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_slr_onepass_kernel(const __gr
     }
 }
 
+// Sliced keys, gradients accumulated, with the forward's lse: the one-pass
+// structure of bwd_slr_onepass_kernel sized for two CTAs per SM, so that
+// sixteen warps share each SM.  The ring carries the value row and the old
+// gradient row (3 stages); only each row's key vector is parked in the stash,
+// and the tables hold alpha_i and g_i alone: after the token's last row the
+// slice lanes recompute rho_i and s_i from the stashed key (the same fixed
+// butterfly as in the value pass, so bitwise the same values) and re-read the
+// old gradient of the slice, which the ring brought through L2 moments before.
+//
+// Shared memory: ring [kWarps][S][2][V][32] cells | q [rp] | dq [kWarps][rp] |
+// tables [kWarps][2][n4] (alpha, g) | per warp: stash [n][nv] cells and the
+// token's dh slice [nv] cells.
+inline size_t onepass_acc_smem(int S, int V, int n, int r, int nv) {
+    const int rp = round_up(r, 4), n4 = round_up(n, 4);
+    return (size_t)kWarps * S * 2 * V * 32 * 16 + sizeof(float) * (size_t)rp * (1 + kWarps) +
+           (size_t)kWarps * (sizeof(float) * 2 * n4 + (size_t)16 * nv * (n + 1));
+}
+
+template <typename T, int V, int S>
+__global__ void __launch_bounds__(kThreads, 2) bwd_slr_onepass_acc_kernel(const __grid_constant__ BwdParams p) {
+    constexpr int E = VecE<T>::value;
+    constexpr int P = 2;
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int rp = round_up(p.r, 4), n4 = round_up(p.n, 4);
+    const int nv = p.r / E;
+    float *q_s = reinterpret_cast<float *>(smem_raw + (size_t)kWarps * S * P * V * 32 * 16);
+    float *dq_all = q_s + rp;           // [kWarps][rp]
+    float *tab = dq_all + kWarps * rp;  // [kWarps][2][n4]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    float *a_s = tab + warp * 2 * n4;
+    float *g_s = a_s + n4;
+    const uint32_t stash_w = smem_u32(tab + kWarps * 2 * n4) + (uint32_t)(warp * nv * (p.n + 1) * 16);
+    const uint32_t dhs_w = stash_w + (uint32_t)(p.n * nv * 16);
+    const uint32_t ring_w = smem_u32(smem_raw) + (uint32_t)(warp * S * P * V * 32 * 16) + 16u * lane;
+    for (int j = threadIdx.x; j < p.r; j += kThreads) q_s[j] = p.query ? p.query[j] : 0.f;
+    __syncthreads();
+
+    const T *__restrict__ dh = static_cast<const T *>(p.dh);
+    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
+    const int tail0 = p.d - p.r;  // a whole number of vectors
+    const int tv0 = tail0 / E;    // first slice vector of a row
+    const int lead = tv0 % 32;    // lanes lead .. lead + nv - 1 hold the slice, all in register slot vk
+    const int vk = tv0 / 32;
+    const int kvi = lane - lead;
+    const bool has_key = kvi >= 0 && kvi < nv;
+    float qv[E];
+#pragma unroll
+    for (int t = 0; t < E; ++t) qv[t] = has_key ? q_s[kvi * E + t] : 0.f;
+    // slice pass: lane takes slice vector kp of sources lane / nv, lane / nv + kst, ...
+    const int kp = lane % nv, kst = 32 / nv, j0 = kp * E;
+    float qs[E];
+#pragma unroll
+    for (int t = 0; t < E; ++t) qs[t] = q_s[j0 + t];
+    float dq_r[E];
+#pragma unroll
+    for (int t = 0; t < E; ++t) dq_r[t] = 0.f;
+
+    const int64_t x0 = (int64_t)blockIdx.x * kWarps + warp;
+    int64_t ix = x0;  // next row to copy: source ii of token ix
+    int ii = 0;
+    auto cell = [&](int st, int plane, int v) -> uint32_t {
+        return ring_w + (uint32_t)((((st * P + plane) * V + v) * 32) * 16);
+    };
+    auto issue = [&](int st) {
+        if (ix < p.T) {
+            const T *row = src_row<T>(p.vt, ii, ix, p.d);
+            const T *old = dst_row<T>(p.dvt, ii, ix, p.d);
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) cp_async16(cell(st, 0, v), row + e);
+                if (e < tail0) cp_async16(cell(st, 1, v), old + e);  // the slice's old value is re-read later
+            }
+            if (++ii == p.n) {
+                ii = 0;
+                ix += nwarps;
+            }
+        }
+        cp_async_commit();
+    };
+#pragma unroll
+    for (int st = 0; st < S - 1; ++st) issue(st);
+    int st_c = 0, st_i = S - 1;
+
+    for (int64_t x = x0; x < p.T; x += nwarps) {
+        const int64_t row_off = x * p.d;
+        Frag<T, E> dhr[V];
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            const int e = (lane + 32 * v) * E;
+            if (e < p.d) dhr[v].load_nc(dh + row_off + e);
+            else dhr[v].zero();
+        }
+        const float lse = __ldg(p.lse + x);
+#pragma unroll
+        for (int v = 0; v < V; ++v)
+            if (v == vk && has_key) st_shared16(dhs_w + (uint32_t)(kvi * 16), dhr[v].a);
+
+        float asum = 0.f;
+        for (int i = 0; i < p.n; ++i) {
+            issue(st_i);
+            cp_async_wait<S - 1>();  // this lane's copies of row i have landed
+            Frag<T, E> f[V];
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) f[v].a = ld_shared16(cell(st_c, 0, v));
+                else f[v].zero();
+            }
+            float g0 = 0.f, g1 = 0.f, ss = 0.f, qk = 0.f;
+#pragma unroll
+            for (int v = 0; v < V; ++v) {  // vectors past d are zero
+                float o[E], dv[E];
+                f[v].get(o);
+                dhr[v].get(dv);
+#pragma unroll
+                for (int t = 0; t < E; t += 2) fma2(g0, g1, dv[t], dv[t + 1], o[t], o[t + 1]);
+                if (v == vk && has_key) {
+#pragma unroll
+                    for (int t = 0; t < E; ++t) {
+                        ss = fmaf(o[t], o[t], ss);
+                        qk = fmaf(qv[t], o[t], qk);
+                    }
+                    st_shared16(stash_w + (uint32_t)((i * nv + kvi) * 16), f[v].a);
+                }
+            }
+            for (int off = 1; off < nv; off <<= 1) {  // the slice group is aligned: partners stay inside
+                ss += __shfl_xor_sync(0xffffffffu, ss, off);
+                qk += __shfl_xor_sync(0xffffffffu, qk, off);
+            }
+            const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
+            const float s = __shfl_sync(0xffffffffu, rho * qk, lead);
+            const float a = expf(s - lse);
+            asum += a;
+            T *drow = dst_row<T>(p.dvt, i, x, p.d);
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < tail0) {
+                    Frag<T, E> of;
+                    of.a = ld_shared16(cell(st_c, 1, v));
+                    float dv[E], w[E];
+                    dhr[v].get(dv);
+                    of.get(w);
+#pragma unroll
+                    for (int t = 0; t < E; ++t) w[t] = fmaf(a, dv[t], w[t]);
+                    Frag<T, E> out;
+                    out.set(w);
+                    out.store(drow + e);
+                }
+            }
+            const float g = warp_sum(g0 + g1);
+            if (lane == lead) {
+                a_s[i] = a;
+                g_s[i] = g;
+            }
+            st_c = (st_c + 1 == S) ? 0 : st_c + 1;
+            st_i = (st_i + 1 == S) ? 0 : st_i + 1;
+        }
+        __syncwarp();  // stash, tables and the dh slice are visible to the whole warp
+        check_alpha_sum(p, asum, lane);
+
+        float part = 0.f;
+        for (int k = lane; k < p.n; k += 32) part = fmaf(a_s[k], g_s[k], part);
+        const float gbar = warp_sum(part);
+        float dhv[E];
+        {
+            Frag<T, E> hf;
+            hf.a = ld_shared16(dhs_w + (uint32_t)(kp * 16));
+            hf.get(dhv);
+        }
+        // sources k = lane / nv + m kst: the old slices of a batch are loaded together
+        constexpr int B = 4;
+        for (int kb = lane / nv; kb - (lane / nv) < p.n; kb += kst * B) {
+            Frag<T, E> of[B];
+#pragma unroll
+            for (int m = 0; m < B; ++m) {
+                const int k = kb + m * kst;
+                if (k < p.n) of[m].load(dst_row<T>(p.dvt, k, x, p.d) + tail0 + j0);
+                else of[m].zero();
+            }
+#pragma unroll
+            for (int m = 0; m < B; ++m) {
+                const int k = kb + m * kst;  // the nv lanes of source k are consecutive: an aligned group
+                Frag<T, E> kf;
+                if (k < p.n) kf.a = ld_shared16(stash_w + (uint32_t)((k * nv + kp) * 16));
+                else kf.zero();
+                float kv[E], w[E];
+                kf.get(kv);
+                of[m].get(w);
+                float ss = 0.f, qk = 0.f;
+#pragma unroll
+                for (int t = 0; t < E; ++t) {
+                    ss = fmaf(kv[t], kv[t], ss);
+                    qk = fmaf(qs[t], kv[t], qk);
+                }
+                for (int off = 1; off < nv; off <<= 1) {
+                    ss += __shfl_xor_sync(0xffffffffu, ss, off);
+                    qk += __shfl_xor_sync(0xffffffffu, qk, off);
+                }
+                if (k < p.n) {
+                    const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
+                    const float s = rho * qk;
+                    const float a = a_s[k];
+                    const float ds = a * (g_s[k] - gbar);
+                    const float c1 = ds * rho, c2 = s * p.inv_r;
+#pragma unroll
+                    for (int t = 0; t < E; ++t) {
+                        const float kbar = rho * kv[t];
+                        const float dk = c1 * (qs[t] - c2 * kbar);
+                        dq_r[t] = fmaf(ds, kbar, dq_r[t]);
+                        w[t] += fmaf(a, dhv[t], dk);
+                    }
+                    Frag<T, E> out;
+                    out.set(w);
+                    out.store(dst_row<T>(p.dvt, k, x, p.d) + tail0 + j0);
+                }
+            }
+        }
+        __syncwarp();  // the next token overwrites stash, tables and dh slice
+    }
+    cp_async_wait_all();
+    // lanes sharing a slice vector combine their dq parts with a fixed butterfly
+#pragma unroll
+    for (int t = 0; t < E; ++t)
+        for (int off = nv; off < 32; off <<= 1) dq_r[t] += __shfl_xor_sync(0xffffffffu, dq_r[t], off);
+    if (lane < nv)
+#pragma unroll
+        for (int t = 0; t < E; ++t) dq_all[warp * rp + j0 + t] = dq_r[t];
+    __syncthreads();
+    for (int j = threadIdx.x; j < p.r; j += kThreads) {
+        float acc = 0.f;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) acc += dq_all[w * rp + j];
+        p.partials[(int64_t)blockIdx.x * p.r + j] = acc;
+    }
+}
+
 // Full keys with gradients in another dtype than the inputs: rows loaded into
 // registers, U at a time.
 template <typename Tin, typename Tg, int V, int U>
@@ -1210,6 +1448,26 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     if constexpr (kPipe && V <= 4) {
         constexpr int OSN = OnePassStages<V, false>::value;
         const int nvk = a.r / E;
+        // accumulating: the one-pass kernel at two CTAs per SM when it fits
+        if (a.variant == kSliced && a.lse && a.accumulate && p.key_vec && nvk >= 1 && nvk <= 32 && 32 % nvk == 0 &&
+            a.d % a.r == 0) {
+            constexpr int OSA = 3;
+            const size_t smem2 = onepass_acc_smem(OSA, V, a.n, a.r, nvk);
+            const void *k2 = (const void *)bwd_slr_onepass_acc_kernel<Tin, V, OSA>;
+            int dev = 0, per_sm = 0;
+            cudaGetDevice(&dev);
+            cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
+            if (2 * (smem2 + 1024) <= (size_t)per_sm) {  // two CTAs per SM (1 KB reserved per CTA)
+                cudaError_t e = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
+                if (e != cudaSuccess) return e;
+                const int grid = persistent_grid(k2, kThreads, smem2, work, kMaxPartials);
+                bwd_slr_onepass_acc_kernel<Tin, V, OSA><<<grid, kThreads, smem2, s>>>(p);
+                e = cudaGetLastError();
+                if (e != cudaSuccess) return e;
+                dq_reduce_kernel<<<(a.r + 7) / 8, 256, 0, s>>>(a.partials, grid, a.r, a.dq, a.accumulate);
+                return cudaGetLastError();
+            }
+        }
         if (a.variant == kSliced && a.lse && !a.accumulate && p.key_vec && nvk >= 1 && nvk <= 32 &&
             32 % nvk == 0 && a.d % a.r == 0) {
             const size_t smem1 = onepass_smem(OSN, 1, V, a.n, a.r, nvk);

@@ -53,9 +53,9 @@ struct BwdArgs {
 
 struct BlockPh1Args {
     int variant, in_dtype, pre_dtype;
-    const void *values;   // completed sources [n, T, d]
-    const void *keys;     // P-LR keys [n, T, r]
-    const float *queries; // [c, r]
+    const void *const *values;  // host array of n pointers: completed sources, [T, d] each
+    const void *const *keys;    // host array of n P-LR key pointers ([T, r] each), or null
+    const float *queries;       // [c, r]
     int n, c;
     int64_t T;
     int d, r;

@@ -28,7 +28,7 @@ LIB_PATH = os.path.join(_PKG, "liblrar.so")
 EXPORTS = ("lrar_forward", "lrar_backward", "lrar_backward_workspace_size", "lrar_block_accumulate",
            "lrar_strerror", "lrar_last_error", "lrar_version", "lrar_backward_noalloc", "lrar_diagnostics",
            "lrar_diagnostics_workspace_size", "lrar_block_phase1", "lrar_block_phase2", "lrar_project",
-           "lrar_forward_ptrs", "lrar_backward_ptrs")
+           "lrar_forward_ptrs", "lrar_backward_ptrs", "lrar_block_phase1_ptrs")
 TEST_HOOKS = ("lrar_test_project_tile", "lrar_test_block_phase1_stalled")  # include/lrar_testing.h
 MAX_BLOCK_SITES = 64
 
@@ -63,6 +63,8 @@ def load(path: str | None = None):
         lib.lrar_backward_noalloc.restype = i
         lib.lrar_block_phase1.argtypes = [i, i, i, vp, vp, vp, i, i, i64, i, i, f32, vp, vp, vp, vp]
         lib.lrar_block_phase1.restype = i
+        lib.lrar_block_phase1_ptrs.argtypes = [i, i, i, vp, vp, vp, i, i, i64, i, i, f32, vp, vp, vp, vp]
+        lib.lrar_block_phase1_ptrs.restype = i
         lib.lrar_test_block_phase1_stalled.argtypes = [i, i, i, vp, vp, vp, i, i, i64, i, i, f32, vp, vp, vp,
                                                        ctypes.c_longlong, vp]
         lib.lrar_test_block_phase1_stalled.restype = i
@@ -246,6 +248,19 @@ def block_phase1(variant, values: torch.Tensor, keys: torch.Tensor | None, queri
     _check(load().lrar_block_phase1(variant, dtype_code(values), dtype_code(h_pre), _ptr(values), _ptr(keys),
                                     _ptr(queries), n, c, T, d, r, eps, _ptr(h_pre), _ptr(lse_pre), _ptr(status),
                                     _stream(stream)))
+
+
+def block_phase1_ptrs(variant, values, keys, queries: torch.Tensor, h_pre: torch.Tensor, lse_pre: torch.Tensor,
+                      eps: float = DEFAULT_EPS, status: torch.Tensor | None = None, stream=None) -> None:
+    """lrar_block_phase1_ptrs: block_phase1 with the completed sources as a list
+    of separate [T, d] tensors (and P-LR keys as a list of [T, r] tensors)."""
+    variant = _variant(variant)
+    n = len(values)
+    T, d = values[0].shape
+    c, r = queries.shape
+    _check(load().lrar_block_phase1_ptrs(variant, dtype_code(values[0]), dtype_code(h_pre), _table(values),
+                                         _table(keys), _ptr(queries), n, c, T, d, r, eps, _ptr(h_pre),
+                                         _ptr(lse_pre), _ptr(status), _stream(stream)))
 
 
 def block_phase2(variant, h_pre: torch.Tensor, lse_pre: torch.Tensor, partial: torch.Tensor,
