@@ -17,10 +17,10 @@
 // Phase 1 tiles a token's row over the warps of a group: warp (g, ch) of a CTA
 // owns the 32 x 16-byte chunk ch of token g's rows and keeps up to 8
 // accumulators per element, one per site, so every row read serves all the
-// block's sites.  The chunk warps split the c queries for scoring, each lane
-// working on one (source, key vector) pair, and score the group's next token
-// while its rows load; the weights pass through shared memory,
-// double-buffered, behind one named barrier per token.
+// block's sites.  Tokens go through a three-stage pipeline, one stage per pass
+// and one named barrier per pass: the chunk warps score token p + 2 (split by
+// source: each warp scores its sources against every query), take the softmax
+// of token p + 1 (split by query), and mix token p.
 #include "lrar.h"
 #include "lrar_device.cuh"
 #include "lrar_launch.h"
@@ -34,6 +34,7 @@ static_assert((kPh1Stages & (kPh1Stages - 1)) == 0, "the ring index wraps with a
 
 struct Ph1Params {
     SrcTab vt, kt;         // completed sources [T, d] each; P-LR keys [T, r] each
+    int qpl;               // queries per lane of the per-source scoring (1 or 2); 0: scoring split by query
     const float *queries;  // [c][r]
     void *h_pre;           // [c][T][d]
     float *lse_pre;        // [c][T]
@@ -45,6 +46,11 @@ struct Ph1Params {
     long long wait_cycles;  // bound of each key wait
     int stall;              // test hook: key waits go to a barrier that never completes
 };
+
+// Coordinate t of query j (zero past c and r), read from the caller's array.
+__device__ __forceinline__ float q_init(const Ph1Params &p, int j, int t) {
+    return (j < p.c && t < p.r) ? p.queries[j * p.r + t] : 0.f;
+}
 
 __device__ __forceinline__ void group_sync(int id, int threads) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
@@ -148,41 +154,129 @@ __device__ __forceinline__ void ph1_scores(const Ph1Params &p, const float *__re
     }
 }
 
-// Scores and softmax of token x for this warp's queries j = ch, ch + chunks,
-// ... < c (the chunk warps of a group share the queries): weights alpha_ij to
-// aw[i * kPh1MaxSites + j], lse_j to lse_pre.
+// Scores of token x split by query (keys that are not whole vectors, or too
+// many queries per lane for the per-source split): this warp's queries
+// j = ch, ch + chunks, ... < c against every source, into sc.
 template <typename Tin>
-__device__ __forceinline__ void ph1_score_warp(const Ph1Params &p, const float *__restrict__ q_s, int rp, int64_t x,
-                                               int ch, int lane, float *aw, const unsigned char *kb_s) {
+__device__ __forceinline__ void ph1_scores_by_query(const Ph1Params &p, const float *__restrict__ q_s, int rp,
+                                                    int64_t x, int ch, int lane, float *sc, const unsigned char *kb_s) {
     const int nq = ch < p.c ? (p.c - ch + p.chunks - 1) / p.chunks : 0;
     switch (nq) {  // queries of this warp: 8 / chunks when c = 8
         case 0: break;
-        case 1: ph1_scores<Tin, 1>(p, q_s, rp, x, lane, ch, p.chunks, aw, kb_s); break;
-        case 2: ph1_scores<Tin, 2>(p, q_s, rp, x, lane, ch, p.chunks, aw, kb_s); break;
-        case 3: ph1_scores<Tin, 3>(p, q_s, rp, x, lane, ch, p.chunks, aw, kb_s); break;
-        case 4: ph1_scores<Tin, 4>(p, q_s, rp, x, lane, ch, p.chunks, aw, kb_s); break;
-        default: ph1_scores<Tin, 8>(p, q_s, rp, x, lane, ch, p.chunks, aw, kb_s); break;  // 5..8: chunks == 1
+        case 1: ph1_scores<Tin, 1>(p, q_s, rp, x, lane, ch, p.chunks, sc, kb_s); break;
+        case 2: ph1_scores<Tin, 2>(p, q_s, rp, x, lane, ch, p.chunks, sc, kb_s); break;
+        case 3: ph1_scores<Tin, 3>(p, q_s, rp, x, lane, ch, p.chunks, sc, kb_s); break;
+        case 4: ph1_scores<Tin, 4>(p, q_s, rp, x, lane, ch, p.chunks, sc, kb_s); break;
+        default: ph1_scores<Tin, 8>(p, q_s, rp, x, lane, ch, p.chunks, sc, kb_s); break;  // 5..8: chunks == 1
     }
-    __syncwarp();
-    for (int j = ch; j < p.c; j += p.chunks) {
-        float m = -INFINITY;
-        for (int i = lane; i < p.n; i += 32) m = fmaxf(m, aw[i * kPh1MaxSites + j]);
-        m = warp_max(m);
-        float z = 0.f;
-        for (int i = lane; i < p.n; i += 32) z += expf(aw[i * kPh1MaxSites + j] - m);
-        z = warp_sum(z);
-        for (int i = lane; i < p.n; i += 32) aw[i * kPh1MaxSites + j] = expf(aw[i * kPh1MaxSites + j] - m) / z;
-        if (lane == 0) p.lse_pre[(int64_t)j * p.T + x] = m + logf(z);
-    }
-    __syncwarp();
 }
 
-// Phase 1 (§3.5): per token of a group, the group's warps mix its n rows into
-// c sites and score the group's next token, each warp its share of the queries.
+// Scores of token x split by source (keys that are whole 16-byte vectors, nv =
+// r / E of them dividing a warp): this warp scores sources i = chunks - 1 - ch,
+// 2 chunks - 1 - ch, ... against every query.  Lane l holds key vector v = l % nv and the queries
+// j = l / nv + u (32 / nv), u < QPL, whose vector v it reads from qv_s (float4
+// t of query slot u at qv_s[(u E / 4 + t) 32 + l], conflict-free);
+// the nv lanes of a source combine |k_i|^2 and the q_j . k_i parts with a fixed
+// butterfly, the same arithmetic in the same order as the split by query, and
+// lane v = 0 writes s_ij = rho_i (q_j . k_i) to sc[i * kPh1MaxSites + j].
+template <typename Tin, int QPL>
+__device__ __forceinline__ void ph1_scores_by_source(const Ph1Params &p, const float4 *__restrict__ qv_s, int64_t x,
+                                                     int ch, int lane, float *sc, const unsigned char *kb_s) {
+    constexpr int E = VecE<Tin>::value;
+    const int nv = p.r / E;
+    const int v = lane % nv, qg = lane / nv, gstep = 32 / nv;
+    // sources chunks - 1 - ch, 2 chunks - 1 - ch, ...: warp 0, which also stages the
+    // keys, is the last to take a second source
+    for (int i = p.chunks - 1 - ch; i < p.n; i += p.chunks) {  // warp-uniform
+        Frag<Tin, E> f;
+        if (kb_s) f.a = *reinterpret_cast<const uint4 *>(kb_s + i * ph1_kstride<Tin>(p.r) + v * 16);
+        else f.load_nc(ph1_key<Tin>(p, i, x) + v * E);
+        float k[E];
+        f.get(k);
+        float ss = 0.f, qk[QPL];
+#pragma unroll
+        for (int t = 0; t < E; ++t) ss = fmaf(k[t], k[t], ss);
+#pragma unroll
+        for (int u = 0; u < QPL; ++u) {
+            qk[u] = 0.f;
+#pragma unroll
+            for (int t = 0; t < E; t += 4) {
+                const float4 q4 = qv_s[(u * (E / 4) + t / 4) * 32 + lane];
+                qk[u] = fmaf(q4.x, k[t], qk[u]);
+                qk[u] = fmaf(q4.y, k[t + 1], qk[u]);
+                qk[u] = fmaf(q4.z, k[t + 2], qk[u]);
+                qk[u] = fmaf(q4.w, k[t + 3], qk[u]);
+            }
+        }
+        for (int off = 1; off < nv; off <<= 1) {  // the source's lanes form an aligned group
+            ss += __shfl_xor_sync(0xffffffffu, ss, off);
+#pragma unroll
+            for (int u = 0; u < QPL; ++u) qk[u] += __shfl_xor_sync(0xffffffffu, qk[u], off);
+        }
+        if (v == 0) {
+            const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
+#pragma unroll
+            for (int u = 0; u < QPL; ++u) {
+                const int j = qg + u * gstep;
+                if (j < p.c) sc[i * kPh1MaxSites + j] = rho * qk[u];
+            }
+        }
+    }
+}
+
+// Softmax of token x (Eq. 10) for the queries j = ch, ch + chunks, ... < c:
+// weights alpha_ij = exp(s_ij - lse_j) to aw[i * kPh1MaxSites + j], lse_j to
+// lse_pre, from the scores in sc.
+__device__ __forceinline__ void ph1_softmax(const Ph1Params &p, int64_t x, int ch, int lane, const float *sc,
+                                            float *aw) {
+    for (int j = ch; j < p.c; j += p.chunks) {
+        float m = -INFINITY;
+        for (int i = lane; i < p.n; i += 32) m = fmaxf(m, sc[i * kPh1MaxSites + j]);
+        m = warp_max(m);
+        float z = 0.f;
+        for (int i = lane; i < p.n; i += 32) z += expf(sc[i * kPh1MaxSites + j] - m);
+        z = warp_sum(z);
+        for (int i = lane; i < p.n; i += 32) aw[i * kPh1MaxSites + j] = expf(sc[i * kPh1MaxSites + j] - m) / z;
+        if (lane == 0) p.lse_pre[(int64_t)j * p.T + x] = m + logf(z);
+    }
+}
+
+// One row of phase 1's mix: acc_j (+)= alpha_ij o_i for the sites j < c, the
+// row in f and its weights at aw[j] (FIRST: acc_j = alpha_ij o_i, used with
+// all eight sites only).
+template <typename Tin, int E, bool C8, bool FIRST>
+__device__ __forceinline__ void ph1_row(float (&acc)[kPh1MaxSites][E], const Frag<Tin, E> &f,
+                                        const float *__restrict__ aw, int c) {
+    float o[E], w[kPh1MaxSites];
+    f.get(o);
+    const float4 w0 = *reinterpret_cast<const float4 *>(aw);
+    const float4 w1 = *reinterpret_cast<const float4 *>(aw + 4);
+    w[0] = w0.x, w[1] = w0.y, w[2] = w0.z, w[3] = w0.w, w[4] = w1.x, w[5] = w1.y, w[6] = w1.z, w[7] = w1.w;
+#pragma unroll
+    for (int j = 0; j < kPh1MaxSites; ++j) {
+        if (C8 || j < c) {
+#pragma unroll
+            for (int t = 0; t < E; t += 2) {
+                if (FIRST) {
+                    const float2 m = __fmul2_rn(make_float2(w[j], w[j]), make_float2(o[t], o[t + 1]));
+                    acc[j][t] = m.x;
+                    acc[j][t + 1] = m.y;
+                } else {
+                    fma2(acc[j][t], acc[j][t + 1], w[j], w[j], o[t], o[t + 1]);
+                }
+            }
+        }
+    }
+}
+
+// Phase 1 (§3.5): in pass p a token group's warps score the group's token
+// p + 2, take the softmax of token p + 1 and mix the n rows of token p into c
+// sites; scores and weights pass through shared memory (double-buffered by
+// token), and the pass ends at the group's named barrier.
 //   Rows stream through a per-lane cp.async ring (each lane copies and reads
 //   back its own 16-byte vector of every row), S - 1 rows ahead and across
 //   tokens, so the next token's rows travel while this one is mixed.
-//   KS: each group's keys are staged two tokens ahead in shared memory with
+//   KS: each group's keys are staged three tokens ahead in shared memory with
 //   bulk copies (double-buffered, one mbarrier per buffer) by the group's warp
 //   0, so scoring reads no global memory.  Each warp's wait for them is
 //   bounded (p.wait_cycles) and decided for the whole warp; one that runs out
@@ -210,6 +304,8 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
     float *q_s = reinterpret_cast<float *>(reinterpret_cast<unsigned char *>(kbar_all) +
                                            (KS ? round_up(G * 2 * (8 + 4), 16) : 0));  // [8][rp], zero past c and r
     float *a_all = q_s + kPh1MaxSites * rp;  // [G][2][n][8]: weights, double-buffered by token
+    float *s_all = a_all + (size_t)G * 2 * kPh1MaxSites * p.n;  // [G][2][n][8]: scores, double-buffered by token
+    float4 *qv_s = reinterpret_cast<float4 *>(s_all + (size_t)G * 2 * kPh1MaxSites * p.n);  // [2][E / 4][32]
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int g = warp / p.chunks, ch = warp % p.chunks;
     const int nthr = p.chunks * 32;  // threads of a token group (named barrier 1 + g)
@@ -219,6 +315,14 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
     for (int j = threadIdx.x; j < kPh1MaxSites * rp; j += kThreads) {
         const int jj = j / rp, t = j % rp;
         q_s[j] = (jj < p.c && t < p.r) ? p.queries[jj * p.r + t] : 0.f;
+    }
+    if (threadIdx.x < 2 * (E / 4) * 32) {  // per-lane query vectors of the per-source split
+        const int l = threadIdx.x % 32, ut = threadIdx.x / 32, u = ut / (E / 4), t4 = ut % (E / 4);
+        const int nvq = p.qpl ? p.r / E : 1;
+        const int j = l / nvq + u * (32 / nvq), t = (l % nvq) * E + 4 * t4;
+        const bool ok = u < p.qpl && j < kPh1MaxSites;
+        qv_s[threadIdx.x] = ok ? make_float4(q_init(p, j, t), q_init(p, j, t + 1), q_init(p, j, t + 2), q_init(p, j, t + 3))
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
     }
     if (KS && threadIdx.x < 2 * G) {
         sm100::mbar_init(smem_u32(kbar_all + threadIdx.x), 1);
@@ -237,6 +341,9 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
     Tout *__restrict__ h_pre = static_cast<Tout *>(p.h_pre);
     const int e = (ch * 32 + lane) * E;  // this lane's first element of the row
     float *aw0 = a_all + (size_t)g * 2 * kPh1MaxSites * p.n;
+    float *sc0 = s_all + (size_t)g * 2 * kPh1MaxSites * p.n;
+    auto awb = [&](int q) { return aw0 + (q & 1) * kPh1MaxSites * p.n; };  // weights of the group's token q
+    auto scb = [&](int q) { return sc0 + (q & 1) * kPh1MaxSites * p.n; };  // scores of the group's token q
     const int64_t stride = (int64_t)gridDim.x * G;
     const uint32_t ring_w = smem_u32(smem_raw) + (uint32_t)(warp * S * 32 * 16) + 16u * lane;
     unsigned char *kb0 = kb_all + (size_t)g * 2 * kbuf_bytes;
@@ -262,66 +369,96 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
         if (b) ++issued1;
         else ++issued0;
     };
-    auto score = [&](int q, int64_t xx, float *aw) {  // token q = xx of the group: this warp's queries
+    auto score = [&](int q, int64_t xx) {  // token q = xx of the group: this warp's share of the scores
         if (KS) kwait(q);
-        ph1_score_warp<Tin>(p, q_s, rp, xx, ch, lane, aw, KS ? kb0 + (q & 1) * kbuf_bytes : nullptr);
+        const unsigned char *kb = KS ? kb0 + (q & 1) * kbuf_bytes : nullptr;
+        if (p.qpl == 2) ph1_scores_by_source<Tin, 2>(p, qv_s, xx, ch, lane, scb(q), kb);
+        else if (p.qpl == 1) ph1_scores_by_source<Tin, 1>(p, qv_s, xx, ch, lane, scb(q), kb);
+        else ph1_scores_by_query<Tin>(p, q_s, rp, xx, ch, lane, scb(q), kb);
     };
 
     int64_t x = (int64_t)blockIdx.x * G + g;
-    // the ring: row ii of token ix is the next to copy
-    int64_t ix = x;
+    // the ring: this lane's next copy is its vector of source ii's row at element
+    // offset xoff (the group's token times d, plus e); rows_left copies remain
+    const bool cp_lane = FULLW || e < p.d;
+    const int64_t xstep = stride * p.d;
+    int64_t xoff = x * p.d + e;
     int ii = 0;
-    auto issue = [&](int st) {
-        if (ix < p.T) {
-            if (FULLW || e < p.d) cp_async16(ring_w + 16u * 32u * st, src_row<Tin>(p.vt, ii, ix, p.d) + e);
+    int rows_left = x < p.T ? (int)((p.T - x + stride - 1) / stride) * p.n : 0;  // warp-uniform
+    uint32_t wslot = ring_w;  // shared address the next copy goes to
+    const uint32_t ring_end = ring_w + 16u * 32u * S;
+    auto issue = [&]() {
+        if (rows_left > 0) {
+            if (cp_lane) cp_async16(wslot, static_cast<const Tin *>(p.vt.p[ii]) + xoff);
+            --rows_left;
             if (++ii == p.n) {
                 ii = 0;
-                ix += stride;
+                xoff += xstep;
             }
         }
         cp_async_commit();
+        wslot += 16u * 32u;
+        if (wslot == ring_end) wslot = ring_w;
     };
 #pragma unroll
-    for (int st = 0; st < S - 1; ++st) issue(st);
-    int st = 0;  // ring slot of the next row to mix; slot st - 1 (mod S) is refilled
+    for (int st = 0; st < S - 1; ++st) issue();
+    uint32_t rslot = ring_w;  // shared address of the next row to read
+    // Within a token each row is read from the ring one row ahead of its use:
+    // with K rows of the stream mixed before the token, K + S - 1 + i copies
+    // have been issued when row K + i is read, and the wait that leaves at most
+    // S - 2 of them pending means rows up to K + i have landed.  Each copy
+    // refills the slot of a row whose value a multiply-add has already used.
+    Frag<Tin, E> f;
+    auto read_row = [&]() {
+        if (cp_lane) f.a = ld_shared16(rslot);
+        else f.zero();
+        rslot += 16u * 32u;
+        if (rslot == ring_end) rslot = ring_w;
+    };
+    auto next_row = [&]() {
+        issue();
+        cp_async_wait<S - 2>();
+        read_row();
+    };
 
+    // prologue: token 0 scored; then token 1 scored and token 0's softmax
     if (KS && ch == 0) {
         if (x < p.T) stage(x, 0);
         if (x + stride < p.T) stage(x + stride, 1);
     }
-    if (x < p.T) score(0, x, aw0);
+    if (x < p.T) score(0, x);
+    group_sync(1 + g, nthr);
+    if (KS && ch == 0 && x + 2 * stride < p.T) stage(x + 2 * stride, 0);  // buffer 0 held token 0, scored above
+    if (x < p.T) ph1_softmax(p, x, ch, lane, scb(0), awb(0));
+    if (x + stride < p.T) score(1, x + stride);
     group_sync(1 + g, nthr);
     for (int pass = 0; (int64_t)blockIdx.x * G + pass * stride < p.T; ++pass, x += stride) {
-        const float *aw = aw0 + (pass & 1) * kPh1MaxSites * p.n;
-        // buffer pass % 2 held token `pass`, scored before the last barrier
-        if (KS && ch == 0 && x + 2 * stride < p.T) stage(x + 2 * stride, pass & 1);
-        if (x + stride < p.T) score(pass + 1, x + stride, aw0 + ((pass + 1) & 1) * kPh1MaxSites * p.n);
+        const float *aw = awb(pass);
+        // key buffer (pass + 1) % 2 held token pass + 1, scored before the last barrier
+        if (KS && ch == 0 && x + 3 * stride < p.T) stage(x + 3 * stride, (pass + 1) & 1);
+        if (x + stride < p.T) ph1_softmax(p, x + stride, ch, lane, scb(pass + 1), awb(pass + 1));
+        if (x + 2 * stride < p.T) score(pass + 2, x + 2 * stride);
         if (x < p.T) {
+            // the next row is read from the ring before this row's multiply-adds,
+            // so its shared-memory latency overlaps them; row 0 starts the
+            // accumulators with a product (the value of a multiply-add onto zero)
             float acc[kPh1MaxSites][E];
+            cp_async_wait<S - 2>();
+            read_row();
+            if (C8) {
+                ph1_row<Tin, E, C8, true>(acc, f, aw, p.c);
+            } else {  // fewer sites: zero, then every row as a multiply-add (fewer live values)
 #pragma unroll
-            for (int j = 0; j < kPh1MaxSites; ++j)
+                for (int j = 0; j < kPh1MaxSites; ++j)
 #pragma unroll
-                for (int t = 0; t < E; ++t) acc[j][t] = 0.f;
-            for (int i = 0; i < p.n; ++i) {
-                issue((st + S - 1) & (S - 1));
-                cp_async_wait<S - 1>();  // this lane's copy of row i has landed
-                Frag<Tin, E> f;
-                if (FULLW || e < p.d) f.a = ld_shared16(ring_w + 16u * 32u * st);
-                else f.zero();
-                st = (st + 1) & (S - 1);
-                float o[E], w[kPh1MaxSites];
-                f.get(o);
-                const float4 w0 = *reinterpret_cast<const float4 *>(aw + i * kPh1MaxSites);
-                const float4 w1 = *reinterpret_cast<const float4 *>(aw + i * kPh1MaxSites + 4);
-                w[0] = w0.x, w[1] = w0.y, w[2] = w0.z, w[3] = w0.w, w[4] = w1.x, w[5] = w1.y, w[6] = w1.z, w[7] = w1.w;
-#pragma unroll
-                for (int j = 0; j < kPh1MaxSites; ++j) {
-                    if (C8 || j < p.c) {
-#pragma unroll
-                        for (int t = 0; t < E; t += 2) fma2(acc[j][t], acc[j][t + 1], w[j], w[j], o[t], o[t + 1]);
-                    }
-                }
+                    for (int t = 0; t < E; ++t) acc[j][t] = 0.f;
+                ph1_row<Tin, E, C8, false>(acc, f, aw, p.c);
             }
+            for (int i = 1; i < p.n; ++i) {
+                next_row();
+                ph1_row<Tin, E, C8, false>(acc, f, aw + i * kPh1MaxSites, p.c);
+            }
+            issue();  // the stream stays S - 1 copies ahead of the next token's first row
             if (FULLW || e < p.d) {
                 Tout *hp = h_pre + x * p.d + e;
 #pragma unroll
@@ -334,7 +471,7 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
                 }
             }
         }
-        group_sync(1 + g, nthr);  // next weights complete; this pass's weights free for reuse
+        group_sync(1 + g, nthr);  // next weights and scores complete; this pass's weights free for reuse
     }
     cp_async_wait_all();
     if (KS && ch == 0)  // drain: the one phase per buffer a give-up may have left unconfirmed
@@ -464,7 +601,8 @@ bool block_phase1_stages_keys(const BlockPh1Args &a) {
 static size_t ph1_smem(int S, bool ks, int G, int n, int r, int kstride) {
     const size_t kbuf = ks ? (size_t)round_up(n * kstride, 16) : 0;
     return (size_t)kWarps * S * 32 * 16 + (size_t)G * 2 * kbuf + (ks ? (size_t)round_up(G * 2 * (8 + 4), 16) : 0) +
-           sizeof(float) * ((size_t)kPh1MaxSites * round_up(r, 4) + (size_t)G * 2 * kPh1MaxSites * n);
+           sizeof(float) * ((size_t)kPh1MaxSites * round_up(r, 4) + (size_t)G * 4 * kPh1MaxSites * n) +
+           2 * 2 * 32 * sizeof(float4);  // per-lane query vectors
 }
 
 template <typename Tin, typename Tout, bool KS, bool FAST>
@@ -499,6 +637,11 @@ static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
     p.wait_cycles = a.wait_cycles;
     p.stall = a.stall ? 1 : 0;
     p.key_vec = ph1_key_vec<Tin>(a);
+    {  // per-source scoring: keys as whole vectors, nv dividing a warp, at most 2 queries per lane
+        const int nv = a.r / E, c8 = a.c < kPh1MaxSites ? a.c : kPh1MaxSites;
+        const int qpl = (nv >= 1 && nv <= 32 && 32 % nv == 0) ? (c8 + 32 / nv - 1) / (32 / nv) : 99;
+        p.qpl = (p.key_vec && a.r % E == 0 && qpl <= 2) ? qpl : 0;
+    }
     const int G = kWarps / chunks;
     const bool ks = ph1_stages_keys_t<Tin>(a);  // keys staged in shared memory
     const bool fullw = a.d == chunks * 32 * E;  // every lane's vector inside the row

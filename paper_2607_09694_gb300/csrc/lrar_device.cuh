@@ -99,9 +99,18 @@ template <> struct Frag<bf16, 8> {
         f[0] = bf_lo(a.x); f[1] = bf_hi(a.x); f[2] = bf_lo(a.y); f[3] = bf_hi(a.y);
         f[4] = bf_lo(a.z); f[5] = bf_hi(a.z); f[6] = bf_lo(a.w); f[7] = bf_hi(a.w);
     }
+    // consecutive pairs, as the operands of packed fp32 arithmetic
+    __device__ __forceinline__ void get2(float2 *f) const {
+        f[0] = make_float2(bf_lo(a.x), bf_hi(a.x)); f[1] = make_float2(bf_lo(a.y), bf_hi(a.y));
+        f[2] = make_float2(bf_lo(a.z), bf_hi(a.z)); f[3] = make_float2(bf_lo(a.w), bf_hi(a.w));
+    }
     __device__ __forceinline__ void set(const float *f) {
         a.x = bf_pack(f[0], f[1]); a.y = bf_pack(f[2], f[3]);
         a.z = bf_pack(f[4], f[5]); a.w = bf_pack(f[6], f[7]);
+    }
+    __device__ __forceinline__ void set2(const float2 *f) {
+        a.x = bf_pack(f[0].x, f[0].y); a.y = bf_pack(f[1].x, f[1].y);
+        a.z = bf_pack(f[2].x, f[2].y); a.w = bf_pack(f[3].x, f[3].y);
     }
 };
 
@@ -115,6 +124,10 @@ template <> struct Frag<bf16, 4> {
         f[0] = bf_lo(a.x); f[1] = bf_hi(a.x); f[2] = bf_lo(a.y); f[3] = bf_hi(a.y);
     }
     __device__ __forceinline__ void set(const float *f) { a.x = bf_pack(f[0], f[1]); a.y = bf_pack(f[2], f[3]); }
+    __device__ __forceinline__ void get2(float2 *f) const {
+        f[0] = make_float2(bf_lo(a.x), bf_hi(a.x)); f[1] = make_float2(bf_lo(a.y), bf_hi(a.y));
+    }
+    __device__ __forceinline__ void set2(const float2 *f) { a.x = bf_pack(f[0].x, f[0].y); a.y = bf_pack(f[1].x, f[1].y); }
 };
 
 template <> struct Frag<float, 4> {
@@ -127,9 +140,17 @@ template <> struct Frag<float, 4> {
         f[0] = __uint_as_float(a.x); f[1] = __uint_as_float(a.y);
         f[2] = __uint_as_float(a.z); f[3] = __uint_as_float(a.w);
     }
+    __device__ __forceinline__ void get2(float2 *f) const {
+        f[0] = make_float2(__uint_as_float(a.x), __uint_as_float(a.y));
+        f[1] = make_float2(__uint_as_float(a.z), __uint_as_float(a.w));
+    }
     __device__ __forceinline__ void set(const float *f) {
         a.x = __float_as_uint(f[0]); a.y = __float_as_uint(f[1]);
         a.z = __float_as_uint(f[2]); a.w = __float_as_uint(f[3]);
+    }
+    __device__ __forceinline__ void set2(const float2 *f) {
+        a.x = __float_as_uint(f[0].x); a.y = __float_as_uint(f[0].y);
+        a.z = __float_as_uint(f[1].x); a.w = __float_as_uint(f[1].y);
     }
 };
 
@@ -141,6 +162,8 @@ template <> struct Frag<float, 8> {
     __device__ __forceinline__ void zero() { lo.zero(); hi.zero(); }
     __device__ __forceinline__ void get(float *f) const { lo.get(f); hi.get(f + 4); }
     __device__ __forceinline__ void set(const float *f) { lo.set(f); hi.set(f + 4); }
+    __device__ __forceinline__ void get2(float2 *f) const { lo.get2(f); hi.get2(f + 2); }
+    __device__ __forceinline__ void set2(const float2 *f) { lo.set2(f); hi.set2(f + 2); }
 };
 
 // ----------------------------------------------------------- reductions ---
@@ -197,10 +220,9 @@ __device__ __forceinline__ T *dst_row(const SrcTab &t, int i, int64_t x, int wid
 // Two fp32 fused multiply-adds in one packed instruction (d_k = a_k b_k + d_k,
 // each rounded to nearest even: the same results as two fmaf).
 __device__ __forceinline__ void fma2(float &d0, float &d1, float a0, float a1, float b0, float b1) {
-    asm("{\n\t.reg .b64 ra, rb, rc;\n\tmov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%0, %1};\n\t"
-        "fma.rn.f32x2 rc, ra, rb, rc;\n\tmov.b64 {%0, %1}, rc;\n\t}"
-        : "+f"(d0), "+f"(d1)
-        : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+    const float2 r = __ffma2_rn(make_float2(a0, a1), make_float2(b0, b1), make_float2(d0, d1));
+    d0 = r.x;
+    d1 = r.y;
 }
 
 }  // namespace lrar
