@@ -15,7 +15,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "liblrar.so")
-SOURCES = ["lrar_api.cu", "lrar_fwd.cu", "lrar_bwd.cu", "lrar_noalloc.cu", "lrar_block.cu", "lrar_proj.cu"]
+SOURCES = ["lrar_api.cu", "lrar_fwd.cu", "lrar_bwd.cu", "lrar_bwd_fixed.cu", "lrar_noalloc.cu", "lrar_block.cu",
+           "lrar_proj.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-fvisibility=hidden",
                      "-I", INCLUDE, "-I", CSRC]

@@ -29,31 +29,11 @@
 #include <type_traits>
 
 #include "lrar.h"
+#include "lrar_bwd.cuh"
 #include "lrar_device.cuh"
 #include "lrar_launch.h"
 
 namespace lrar {
-
-struct BwdParams {
-    SrcTab vt, kt, dvt, dkt;  // values, P-LR keys and their gradients, one matrix per source
-    const void *dh, *h;
-    const float *query, *lse;
-    float *partials;
-    int *status;  // optional: LRAR_STATUS_LSE_MISMATCH when a token's weights from lse do not sum to 1
-    int64_t T;
-    int n, d, r;
-    float eps, inv_r;
-    int sliced, key_vec, accumulate, h_bf16;
-};
-
-// Weights taken from a supplied lse sum to 1 up to fp32 rounding when the lse
-// belongs to the same values and query; a sum further than this from 1 marks
-// an lse of other inputs.
-constexpr float kLseSumTol = 1e-3f;
-
-__device__ __forceinline__ void check_alpha_sum(const BwdParams &p, float asum, int lane) {
-    if (lane == 0 && p.status && !(fabsf(asum - 1.f) <= kLseSumTol)) atomicOr(p.status, LRAR_STATUS_LSE_MISMATCH);
-}
 
 // Routing stage, identical arithmetic to the forward's (see lrar_fwd.cu).
 template <typename Tin>
@@ -1446,6 +1426,9 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     // pass + key pass kernel at n = 49 on GB300 (one CTA per SM against two),
     // so accumulating calls take bwd_lr_pipe_kernel.
     if constexpr (kPipe && V <= 4) {
+        bool launched = false;
+        cudaError_t ef = launch_bwd_fixed(p, a, launched, s);
+        if (ef != cudaSuccess || launched) return ef;
         constexpr int OSN = OnePassStages<V, false>::value;
         const int nvk = a.r / E;
         // accumulating: the one-pass kernel at two CTAs per SM when it fits
