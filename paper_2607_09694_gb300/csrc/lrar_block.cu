@@ -292,6 +292,7 @@ __device__ __forceinline__ void ph1_row(float (&acc)[kPh1MaxSites][E], const Fra
 //   FULLW: every lane's vector lies inside the row (d = chunks * 32 * E).
 template <typename Tin, typename Tout, int S, bool KS, bool C8, bool FULLW>
 __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_constant__ Ph1Params p) {
+    pdl_enter();
     constexpr int E = VecE<Tin>::value;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int rp = round_up(p.r, 4);
@@ -499,6 +500,7 @@ struct Ph2Params {
 // the same elements of h (and lse), so h may be h_pre and lse may be lse_pre.
 template <typename Tin, typename Tp, typename Tout, int V>
 __global__ void __launch_bounds__(kThreads) block_phase2_kernel(const Ph2Params p) {
+    pdl_enter();
     constexpr int E = VecE<Tin>::value;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const Tin *__restrict__ part = static_cast<const Tin *>(p.partial);
@@ -608,7 +610,7 @@ static size_t ph1_smem(int S, bool ks, int G, int n, int r, int kstride) {
 template <typename Tin, typename Tout, bool KS, bool FAST>
 static cudaError_t ph1_go(const Ph1Params &p, int grid, size_t smem, cudaStream_t s) {
     constexpr int S = kPh1Stages;
-    block_phase1_kernel<Tin, Tout, S, KS, FAST, FAST><<<grid, kThreads, smem, s>>>(p);
+    launch_pdl(block_phase1_kernel<Tin, Tout, S, KS, FAST, FAST>, grid, kThreads, smem, s, p);
     return cudaGetLastError();
 }
 
@@ -695,7 +697,7 @@ static cudaError_t launch_ph2_t(const BlockPh2Args &a, cudaStream_t s) {
     p.sliced = a.variant == kSliced;
     const void *k = (const void *)block_phase2_kernel<Tin, Tp, Tout, V>;
     const int grid = persistent_grid(k, kThreads, 0, (a.T + kWarps - 1) / kWarps, 1 << 30);
-    block_phase2_kernel<Tin, Tp, Tout, V><<<grid, kThreads, 0, s>>>(p);
+    launch_pdl(block_phase2_kernel<Tin, Tp, Tout, V>, grid, kThreads, 0, s, p);
     return cudaGetLastError();
 }
 

@@ -146,6 +146,7 @@ __device__ __forceinline__ float lr_bwd_row(const Frag<Tin, VecE<Tin>::value> *f
 
 template <typename Tin, typename Tg, int V, int U, bool ACC>
 __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) bwd_lr_kernel(const __grid_constant__ BwdParams p) {
+    pdl_enter();
     constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
     const int rp = round_up(p.r, 4);
@@ -455,6 +456,7 @@ __device__ __forceinline__ void key_pass(const BwdParams &p, const T *__restrict
 
 template <typename T, int V, int S, bool ACC, bool VK>
 __global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_lr_pipe_kernel(const __grid_constant__ BwdParams p) {
+    pdl_enter();
     constexpr int E = VecE<T>::value;
     constexpr int P = ACC ? 2 : 1;  // planes per stage: o, old gradient
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -712,6 +714,7 @@ __host__ __device__ inline size_t full_ring_bytes(int cells, int d) {
 // bytes in flight for eight warps.
 template <typename T, int V, int S, bool ACC>
 __global__ void __launch_bounds__(kThreads, 1) bwd_full_pipe_kernel(const __grid_constant__ BwdParams p) {
+    pdl_enter();
     constexpr int E = VecE<T>::value;
     constexpr int P = ACC ? 2 : 1;
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -832,6 +835,7 @@ inline size_t onepass_smem(int S, int P, int V, int n, int r, int nv) {
 
 template <typename T, int V, int S, bool ACC>
 __global__ void __launch_bounds__(kThreads, 1) bwd_slr_onepass_kernel(const __grid_constant__ BwdParams p) {
+    pdl_enter();
     constexpr int E = VecE<T>::value;
     constexpr int P = ACC ? 2 : 1;
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -1055,6 +1059,7 @@ inline size_t onepass_acc_smem(int S, int V, int n, int r, int nv) {
 
 template <typename T, int V, int S>
 __global__ void __launch_bounds__(kThreads, 2) bwd_slr_onepass_acc_kernel(const __grid_constant__ BwdParams p) {
+    pdl_enter();
     constexpr int E = VecE<T>::value;
     constexpr int P = 2;
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -1277,6 +1282,7 @@ __global__ void __launch_bounds__(kThreads, 2) bwd_slr_onepass_acc_kernel(const 
 // registers, U at a time.
 template <typename Tin, typename Tg, int V, int U>
 __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(const __grid_constant__ BwdParams p) {
+    pdl_enter();
     constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
     float *q_s = smem;                    // [32 V E] (q_slot), zero past d
@@ -1346,6 +1352,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 2 ? 2 : 1)) bwd_full_kernel(co
 // warp per coordinate, lane l sums partials l, l+32, ... and a fixed butterfly
 // combines the lanes, so the result depends only on the number of partials.
 __global__ void dq_reduce_kernel(const float *__restrict__ partials, int nparts, int rq, float *dq, int accumulate) {
+    pdl_enter();
     const int j = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
     const int lane = threadIdx.x & 31;
     if (j >= rq) return;  // whole warps leave together (blockDim is a multiple of 32)
@@ -1357,7 +1364,7 @@ __global__ void dq_reduce_kernel(const float *__restrict__ partials, int nparts,
 
 cudaError_t launch_partial_sum(const float *partials, int nparts, int width, float *out, int accumulate,
                                cudaStream_t s) {
-    dq_reduce_kernel<<<(width + 7) / 8, 256, 0, s>>>(partials, nparts, width, out, accumulate);
+    launch_pdl(dq_reduce_kernel, (width + 7) / 8, 256, 0, s, partials, nparts, width, out, accumulate);
     return cudaGetLastError();
 }
 
@@ -1444,10 +1451,10 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
                 cudaError_t e = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
                 if (e != cudaSuccess) return e;
                 const int grid = persistent_grid(k2, kThreads, smem2, work, kMaxPartials);
-                bwd_slr_onepass_acc_kernel<Tin, V, OSA><<<grid, kThreads, smem2, s>>>(p);
+                launch_pdl(bwd_slr_onepass_acc_kernel<Tin, V, OSA>, grid, kThreads, smem2, s, p);
                 e = cudaGetLastError();
                 if (e != cudaSuccess) return e;
-                dq_reduce_kernel<<<(a.r + 7) / 8, 256, 0, s>>>(a.partials, grid, a.r, a.dq, a.accumulate);
+                launch_pdl(dq_reduce_kernel, (a.r + 7) / 8, 256, 0, s, a.partials, grid, a.r, a.dq, a.accumulate);
                 return cudaGetLastError();
             }
         }
@@ -1462,10 +1469,10 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
                 cudaError_t e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
                 if (e != cudaSuccess) return e;
                 const int grid = persistent_grid(k1, kThreads, smem1, work, kMaxPartials);
-                bwd_slr_onepass_kernel<Tin, V, OSN, false><<<grid, kThreads, smem1, s>>>(p);
+                launch_pdl(bwd_slr_onepass_kernel<Tin, V, OSN, false>, grid, kThreads, smem1, s, p);
                 e = cudaGetLastError();
                 if (e != cudaSuccess) return e;
-                dq_reduce_kernel<<<(a.r + 7) / 8, 256, 0, s>>>(a.partials, grid, a.r, a.dq, a.accumulate);
+                launch_pdl(dq_reduce_kernel, (a.r + 7) / 8, 256, 0, s, a.partials, grid, a.r, a.dq, a.accumulate);
                 return cudaGetLastError();
             }
         }
@@ -1507,26 +1514,26 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     }
     const int grid = persistent_grid(k, kThreads, smem, work, kMaxPartials);
     if (a.variant == kFull && kPipe && a.accumulate)
-        bwd_full_pipe_kernel<Tin, V, FSA, true><<<grid, kThreads, smem, s>>>(p);
+        launch_pdl(bwd_full_pipe_kernel<Tin, V, FSA, true>, grid, kThreads, smem, s, p);
     else if (a.variant == kFull && kPipe)
-        bwd_full_pipe_kernel<Tin, V, FSN, false><<<grid, kThreads, smem, s>>>(p);
+        launch_pdl(bwd_full_pipe_kernel<Tin, V, FSN, false>, grid, kThreads, smem, s, p);
     else if (a.variant == kFull)
-        bwd_full_kernel<Tin, Tg, V, U><<<grid, kThreads, smem, s>>>(p);
+        launch_pdl(bwd_full_kernel<Tin, Tg, V, U>, grid, kThreads, smem, s, p);
     else if (kPipe && a.accumulate && vk)
-        bwd_lr_pipe_kernel<Tin, V, SA, true, true><<<grid, kThreads, smem, s>>>(p);
+        launch_pdl(bwd_lr_pipe_kernel<Tin, V, SA, true, true>, grid, kThreads, smem, s, p);
     else if (kPipe && a.accumulate)
-        bwd_lr_pipe_kernel<Tin, V, SA, true, false><<<grid, kThreads, smem, s>>>(p);
+        launch_pdl(bwd_lr_pipe_kernel<Tin, V, SA, true, false>, grid, kThreads, smem, s, p);
     else if (kPipe && vk)
-        bwd_lr_pipe_kernel<Tin, V, SN, false, true><<<grid, kThreads, smem, s>>>(p);
+        launch_pdl(bwd_lr_pipe_kernel<Tin, V, SN, false, true>, grid, kThreads, smem, s, p);
     else if (kPipe)
-        bwd_lr_pipe_kernel<Tin, V, SN, false, false><<<grid, kThreads, smem, s>>>(p);
+        launch_pdl(bwd_lr_pipe_kernel<Tin, V, SN, false, false>, grid, kThreads, smem, s, p);
     else if (a.accumulate)
-        bwd_lr_kernel<Tin, Tg, V, UA, true><<<grid, kThreads, smem, s>>>(p);
+        launch_pdl(bwd_lr_kernel<Tin, Tg, V, UA, true>, grid, kThreads, smem, s, p);
     else
-        bwd_lr_kernel<Tin, Tg, V, BwdRows<V, false>::value, false><<<grid, kThreads, smem, s>>>(p);
+        launch_pdl(bwd_lr_kernel<Tin, Tg, V, BwdRows<V, false>::value, false>, grid, kThreads, smem, s, p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    dq_reduce_kernel<<<(rq + 7) / 8, 256, 0, s>>>(a.partials, grid, rq, a.dq, a.accumulate);
+    launch_pdl(dq_reduce_kernel, (rq + 7) / 8, 256, 0, s, a.partials, grid, rq, a.dq, a.accumulate);
     return cudaGetLastError();
 }
 
@@ -1551,6 +1558,7 @@ cudaError_t launch_backward(const BwdArgs &a, cudaStream_t s) {
 template <typename Td, typename Ts>
 __global__ void block_acc_kernel(Td *__restrict__ dst, const Ts *__restrict__ src, int64_t count, float alpha,
                                  float beta, int vec) {
+    pdl_enter();
     const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t nthreads = (int64_t)gridDim.x * blockDim.x;
     const int64_t groups = vec ? count / 8 : 0;
@@ -1588,7 +1596,7 @@ static cudaError_t launch_acc_t(void *dst, const void *src, int64_t count, float
     const int64_t groups = vec ? count / 8 : count;
     const int grid = persistent_grid((const void *)block_acc_kernel<Td, Ts>, threads, 0,
                                      (groups + threads - 1) / threads, 1 << 30);
-    block_acc_kernel<Td, Ts><<<grid, threads, 0, s>>>(static_cast<Td *>(dst), static_cast<const Ts *>(src), count,
+    launch_pdl(block_acc_kernel<Td, Ts>, grid, threads, 0, s, static_cast<Td *>(dst), static_cast<const Ts *>(src), count,
                                                        alpha, beta, vec);
     return cudaGetLastError();
 }

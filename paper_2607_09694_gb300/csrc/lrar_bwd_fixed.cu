@@ -53,6 +53,7 @@ template <int D, int R, int S, bool ACC> struct FixedShape {
 
 template <int D, int R, int S, bool ACC>
 __global__ void __launch_bounds__(kThreads, 2) bwd_slr_fixed_kernel(const __grid_constant__ BwdParams p) {
+    pdl_enter();
     using Sh = FixedShape<D, R, S, ACC>;
     constexpr int E = Sh::E, V = Sh::V, NV = Sh::NV, LEAD = Sh::LEAD, KST = Sh::KST, P = Sh::P;
     constexpr int TAIL0 = D - R;
@@ -283,7 +284,7 @@ cudaError_t go_fixed(const BwdParams &p, const BwdArgs &a, bool &launched, cudaS
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int grid = persistent_grid(k, kThreads, smem, (a.T + kWarps - 1) / kWarps, kMaxPartials);
-    bwd_slr_fixed_kernel<D, R, S, ACC><<<grid, kThreads, smem, s>>>(p);
+    launch_pdl(bwd_slr_fixed_kernel<D, R, S, ACC>, grid, kThreads, smem, s, p);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     launched = true;

@@ -166,6 +166,19 @@ template <> struct Frag<float, 8> {
     __device__ __forceinline__ void set2(const float2 *f) { lo.set2(f); hi.set2(f + 2); }
 };
 
+// ---------------------------------------------------- dependent launch ---
+// Every kernel of the library is launched with programmatic stream
+// serialization (launch_pdl): it may be scheduled while the kernel before it
+// in the stream is still running, and waits here, before its first access to
+// global memory, until that kernel has completed and its writes are visible;
+// it then lets the next kernel be scheduled in turn.  Only the launch and the
+// CTAs' set-up overlap; in a kernel launched without the attribute both
+// instructions return at once.
+__device__ __forceinline__ void pdl_enter() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ----------------------------------------------------------- reductions ---
 // xor butterflies leave the identical bit pattern in every lane.
 __device__ __forceinline__ float warp_sum(float v) {

@@ -170,6 +170,7 @@ constexpr int kPrefetchRows = 8;
 
 template <typename Tin, typename Tout, int V, int U, bool KS>
 __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(const __grid_constant__ FwdParams p) {
+    pdl_enter();
     constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
     float *q_s = smem;                                         // [r]
@@ -310,6 +311,7 @@ __device__ __forceinline__ void full_row_step(const Frag<Tin, VecE<Tin>::value> 
 template <typename Tin, typename Tout, int V, int S>
 __global__ void __launch_bounds__(kThreads, (V * VecE<Tin>::value <= 32 ? 2 : 1))
     fwd_full_kernel(const __grid_constant__ FwdParams p) {
+    pdl_enter();
     constexpr int E = VecE<Tin>::value;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     float *q_s = reinterpret_cast<float *>(smem_raw + (size_t)kWarps * S * V * 32 * 16);  // [32 V E] (q_slot), zero past d
@@ -413,7 +415,7 @@ static cudaError_t launch_fwd_t(const FwdArgs &a, cudaStream_t s, int chunks = 1
             if (e != cudaSuccess) return e;
         }
         const int grid = persistent_grid(k, kThreads, smem, work, 1 << 30);
-        fwd_full_kernel<Tin, Tout, V, S><<<grid, kThreads, smem, s>>>(p);
+        launch_pdl(fwd_full_kernel<Tin, Tout, V, S>, grid, kThreads, smem, s, p);
     } else {
         // Keys staged in shared memory when rows are split over warps (each warp
         // routes its token, so routing weighs twice as much), the keys are whole
@@ -429,8 +431,8 @@ static cudaError_t launch_fwd_t(const FwdArgs &a, cudaStream_t s, int chunks = 1
             if (e != cudaSuccess) return e;
         }
         const int grid = persistent_grid(k, kThreads, smem, work, 1 << 30);
-        if (ks) fwd_lr_kernel<Tin, Tout, V, U, true><<<grid, kThreads, smem, s>>>(p);
-        else fwd_lr_kernel<Tin, Tout, V, U, false><<<grid, kThreads, smem, s>>>(p);
+        if (ks) launch_pdl(fwd_lr_kernel<Tin, Tout, V, U, true>, grid, kThreads, smem, s, p);
+        else launch_pdl(fwd_lr_kernel<Tin, Tout, V, U, false>, grid, kThreads, smem, s, p);
     }
     return cudaGetLastError();
 }
@@ -455,6 +457,7 @@ static cudaError_t launch_fwd_w(const FwdArgs &a, cudaStream_t s) {
 template <typename Tin, int V>
 __global__ void __launch_bounds__(kThreads)
     diag_kernel(const __grid_constant__ FwdParams p, float *neff, float *partials, int full) {
+    pdl_enter();
     constexpr int E = VecE<Tin>::value;
     extern __shared__ float smem[];
     float *q_s = smem;                                    // [r]
@@ -554,7 +557,7 @@ static cudaError_t launch_diag_t(const FwdArgs &a, float *neff, float *mean_alph
         if (e != cudaSuccess) return e;
     }
     const int grid = persistent_grid(k, kThreads, smem, (a.T + kWarps - 1) / kWarps, kMaxPartials);
-    diag_kernel<Tin, V><<<grid, kThreads, smem, s>>>(p, neff, mean_alpha ? partials : nullptr, a.variant == kFull);
+    launch_pdl(diag_kernel<Tin, V>, grid, kThreads, smem, s, p, neff, mean_alpha ? partials : nullptr, a.variant == kFull);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess || !mean_alpha) return e;
     return launch_partial_sum(partials, grid, a.n, mean_alpha, 0, s);

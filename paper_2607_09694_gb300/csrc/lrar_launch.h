@@ -128,4 +128,23 @@ cudaError_t launch_block_accumulate(int dst_dtype, void *dst, int src_dtype, con
 // capped by `cap`.
 int persistent_grid(const void *kernel, int threads, size_t smem, int64_t work_ctas, int cap);
 
+// Launches kernel with programmatic stream serialization, so that it can be
+// scheduled while the previous kernel in the stream finishes (every kernel of
+// the library waits for its predecessor with griddepcontrol.wait before it
+// touches global memory).  Errors are returned and kept for cudaGetLastError.
+template <typename... K, typename... A>
+inline cudaError_t launch_pdl(void (*kernel)(K...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, A &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<A &&>(args)...);
+}
+
 }  // namespace lrar

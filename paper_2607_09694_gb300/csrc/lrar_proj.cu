@@ -72,6 +72,7 @@ template <int kPN>
 __global__ void __launch_bounds__(kPThreads, 1)
     proj_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_w,
                 const ProjParams p) {
+    pdl_enter();
     constexpr int kStageBytes = ProjTile<kPN>::kStageBytes;
     constexpr int kPStages = ProjTile<kPN>::kStages;
     extern __shared__ unsigned char smem_raw[];
@@ -278,7 +279,7 @@ int launch_project_t(const CUtensorMap &map_a, const void *w, int64_t T, int m, 
     const int64_t tiles = (T + kPM - 1) / kPM * ((d + r + BN - 1) / BN);
     const int grid = persistent_grid((const void *)proj_kernel<BN>, kPThreads, smem, tiles, 1 << 30);
     if (grid < 1) return record_error(LRAR_ERR_CUDA, "no SM can hold the projection kernel");
-    proj_kernel<BN><<<grid, kPThreads, smem, s>>>(map_a, map_w, p);
+    launch_pdl(proj_kernel<BN>, grid, kPThreads, smem, s, map_a, map_w, p);
     e = cudaGetLastError();
     if (e != cudaSuccess) return record_error(LRAR_ERR_CUDA, cudaGetErrorString(e));
     return LRAR_OK;
