@@ -17,9 +17,12 @@ extern "C" {
 #endif
 
 /*
- * lrar_project with the tile width forced instead of chosen from the shape:
- * tile is one of the compiled widths 160, 176, 192, 224, 240, 256
- * (LRAR_ERR_INVALID_ARG otherwise), so that a test covers every width.
+ * lrar_project with the tile form and width forced instead of chosen from the
+ * shape: tile is one of the compiled widths 160, 176, 192, 224, 240, 256 for
+ * the single-CTA form (128-row tiles), or 2000 plus one of them for the
+ * CTA-pair form (256-row tiles over a cluster of two CTAs on two SMs,
+ * tcgen05.mma.cta_group::2); anything else is LRAR_ERR_INVALID_ARG.  So a test
+ * covers every width of both forms.
  */
 int lrar_test_project_tile(int tile, int in_dtype, const void *a, const void *w, int64_t T, int m, int d, int r,
                            void *o, void *keys, int *status, void *stream);

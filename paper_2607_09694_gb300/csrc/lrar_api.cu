@@ -545,7 +545,8 @@ int project_impl(int tile, int in_dtype, const void *a, const void *w, int64_t T
         return fail(LRAR_ERR_ALIGNMENT, "a, w, o and keys must be 16-byte aligned");
     if (status && !aligned4(status)) return fail(LRAR_ERR_ALIGNMENT, "status must be 4-byte aligned");
     if (tile != 0 && !lrar::project_tile_ok(tile))
-        return fail(LRAR_ERR_INVALID_ARG, "tile must be 160, 176, 192, 224, 240 or 256 (got %d)", tile);
+        return fail(LRAR_ERR_INVALID_ARG,
+                    "tile must be 160, 176, 192, 224, 240 or 256, or 2000 plus one of them (got %d)", tile);
     if (T == 0) return LRAR_OK;
     return lrar::launch_project(a, w, T, m, d, r, o, keys, status, tile, static_cast<cudaStream_t>(stream));
 }
@@ -559,7 +560,8 @@ LRAR_API int lrar_project(int in_dtype, const void *a, const void *w, int64_t T,
 
 LRAR_API int lrar_test_project_tile(int tile, int in_dtype, const void *a, const void *w, int64_t T, int m, int d,
                                     int r, void *o, void *keys, int *status, void *stream) {
-    if (tile == 0) return fail(LRAR_ERR_INVALID_ARG, "tile must be 160, 176, 192, 224, 240 or 256 (got 0)");
+    if (tile == 0)
+        return fail(LRAR_ERR_INVALID_ARG, "tile must be 160, 176, 192, 224, 240 or 256, or 2000 plus one of them (got 0)");
     return project_impl(tile, in_dtype, a, w, T, m, d, r, o, keys, status, stream);
 }
 

@@ -227,6 +227,215 @@ __global__ void __launch_bounds__(kPThreads, 1)
     }
 }
 
+// The CTA-pair (two-SM) form: a cluster of two CTAs computes a 256 x kPN tile
+// with tcgen05.mma.cta_group::2 (M = 256, N = kPN), each CTA holding 128 rows of
+// A and kPN / 2 rows of W per stage, so each SM's shared memory feeds half the
+// B operand of the single-CTA form per multiply-add.  The leader (rank 0) issues
+// every MMA; both CTAs' TMA loads complete on the leader's full barriers (the
+// leader announces both CTAs' bytes), each MMA block's commit frees the stage in
+// both CTAs, a finished tile is announced to both CTAs' epilogues, and each
+// CTA's epilogue writes its own 128 rows (its half of D sits in its own TMEM)
+// and then arrives on the leader's accumulator barrier.  TMEM is allocated and
+// freed by one warp of each CTA for the pair.  Every barrier wait is bounded; a
+// wait that runs out sets *status and the abort flag of both CTAs; the leader
+// waits (bounded) for the copies of the stages it issued, the other CTA idles
+// 2^22 cycles before it leaves (its copies complete on the leader's barriers,
+// which it cannot wait on), and both meet at a cluster barrier before TMEM is
+// freed.
+template <int kPN> struct ProjPairTile {
+    static constexpr int kHalf = kPN / 2;  // rows of W per CTA and stage
+    static constexpr int kBBytes = kHalf * kPK * 2;
+    static constexpr int kStageBytes = kABytes + kBBytes;
+    static constexpr int kFit = (227 * 1024 - 1024 - 256) / kStageBytes;
+    static constexpr int kStages = kFit > 12 ? 12 : kFit;
+    static constexpr size_t kSmem = (size_t)kStages * kStageBytes + 1024 /* alignment slack */ + 256 /* barriers */;
+    static_assert(kStageBytes % 1024 == 0, "stage tiles must keep 1024-byte alignment");
+    static_assert(kPN % 16 == 0 && kPN <= (int)kAccCols, "M = 256 MMA needs N a multiple of 16 within an accumulator");
+};
+
+template <int kPN>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPThreads, 1)
+    proj_pair_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_w,
+                     const ProjParams p) {
+    pdl_enter();
+    constexpr int kStageBytes = ProjPairTile<kPN>::kStageBytes;
+    constexpr int kPStages = ProjPairTile<kPN>::kStages;
+    constexpr int kHalf = ProjPairTile<kPN>::kHalf;
+    extern __shared__ unsigned char smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;  // the same offset in both CTAs
+    const uint32_t bars = base + kPStages * kStageBytes;
+    auto full = [&](int s) { return bars + 8u * s; };                      // leader: both CTAs' bytes of stage s landed
+    auto empty = [&](int s) { return bars + 8u * (kPStages + s); };         // the MMAs reading stage s are done
+    auto acc_full = [&](int b) { return bars + 8u * (2 * kPStages + b); };  // accumulator b holds a tile
+    auto acc_empty = [&](int b) { return bars + 8u * (2 * kPStages + 2 + b); };  // leader: both halves of b read
+    const uint32_t done_bar = bars + 8u * (2 * kPStages + 4);              // leader: every MMA has completed
+    const uint32_t tmem_slot = done_bar + 8u;
+    const uint32_t abort_a = tmem_slot + 4u;
+    volatile int *abort = reinterpret_cast<volatile int *>(smem_raw + (abort_a - raw));
+    auto stage_a = [&](int s) { return base + (uint32_t)(s * kStageBytes); };
+    auto stage_b = [&](int s) { return base + (uint32_t)(s * kStageBytes + kABytes); };
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_rank();
+    const bool leader = rank == 0;
+    const int N = p.d + p.r;
+    const int nkb = (p.m + kPK - 1) / kPK;
+    const int n_nt = (N + kPN - 1) / kPN;
+    const int64_t n_tiles = (p.T + 2 * kPM - 1) / (2 * kPM) * n_nt;  // tile t: rows (t / n_nt) * 256, columns (t % n_nt) * kPN
+    const int64_t pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kPStages; ++s) {
+            mbar_init(full(s), 1);
+            mbar_init(empty(s), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(acc_full(b), 1);
+            mbar_init(acc_empty(b), 8);  // four epilogue warps in each CTA
+        }
+        mbar_init(done_bar, 1);
+        *abort = 0;
+        mbar_fence_init();
+    }
+    if (warp == 4 && lane == 0) {
+        tma_prefetch_map(&map_a);
+        tma_prefetch_map(&map_w);
+    }
+    cluster_sync();  // both CTAs' barriers exist before any copy or arrival reaches them
+    if (warp == 5) {
+        tmem_alloc_pair(tmem_slot, kTmemCols);
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(smem_raw + (tmem_slot - raw));
+    auto give_up = [&]() {
+        *abort = 1;
+        st_cluster_u32(cluster_addr(abort_a, rank ^ 1u), 1u);
+        if (p.status) atomicOr(p.status, LRAR_STATUS_WAIT_TIMEOUT);
+    };
+
+    int64_t issued = 0;  // K-blocks whose loads this CTA issued (producer lane)
+    if (warp == 4 && lane == 0) {
+        int64_t g = 0;
+        bool ok = true;
+        for (int64_t t = pair; t < n_tiles && ok && !*abort; t += npairs) {
+            const int m0 = (int)(t / n_nt) * 2 * kPM + (int)rank * kPM;
+            const int n0 = (int)(t % n_nt) * kPN + (int)rank * kHalf;
+            for (int kb = 0; kb < nkb; ++kb, ++g) {
+                const int s = (int)(g % kPStages);
+                const uint32_t round = (uint32_t)(g / kPStages);
+                if (round > 0 && !mbar_wait_cluster(empty(s), (round - 1) & 1u, kWaitLimit, abort)) {
+                    give_up();
+                    ok = false;
+                    break;
+                }
+                if (leader) mbar_arrive_expect_tx(full(s), 2u * (uint32_t)kStageBytes);  // both CTAs' loads
+                const uint32_t fb = cluster_addr(full(s), 0);
+                tma_load_2d_pair(stage_a(s), &map_a, fb, kb * kPK, m0);
+                tma_load_2d_pair(stage_b(s), &map_w, fb, kb * kPK, n0);
+                issued = g + 1;
+            }
+        }
+    } else if (warp == 5 && lane == 0 && leader) {
+        constexpr uint32_t idesc = idesc_bf16_f32(2 * kPM, kPN);
+        int64_t g = 0;
+        int it = 0;
+        for (int64_t t = pair; t < n_tiles && !*abort; t += npairs, ++it) {
+            const int b = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1);
+            if (use > 0 && !mbar_wait_cluster(acc_empty(b), (use - 1) & 1u, kWaitLimit, abort)) {
+                give_up();
+                break;
+            }
+            tc_fence_after();
+            const uint32_t acc = tmem + b * kAccCols;
+            bool ok = true;
+            for (int kb = 0; kb < nkb; ++kb, ++g) {
+                const int s = (int)(g % kPStages);
+                if (!mbar_wait_cluster(full(s), (uint32_t)(g / kPStages) & 1u, kWaitLimit, abort)) {
+                    give_up();
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint64_t ad = sw128_kmajor_desc(stage_a(s)), bd = sw128_kmajor_desc(stage_b(s));
+#pragma unroll
+                for (int k = 0; k < kPK / 16; ++k)  // +32 bytes along K per step: +2 in the address field
+                    tc_mma_f16_pair(acc, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0);
+                tc_commit_pair_both(empty(s));
+            }
+            if (!ok) break;
+            tc_commit_pair_both(acc_full(b));
+        }
+        tc_commit_pair(done_bar);  // arrives once every MMA issued above has completed
+        if (!mbar_wait(done_bar, 0, kWaitLimit)) give_up();
+    } else if (warp < 4) {
+        const uint32_t acc_empty_leader0 = cluster_addr(acc_empty(0), 0), acc_empty_leader1 = cluster_addr(acc_empty(1), 0);
+        int it = 0;
+        for (int64_t t = pair; t < n_tiles; t += npairs, ++it) {
+            const int b = it & 1;
+            // warp-uniform decision: tcgen05.ld below needs all 32 lanes
+            if (!__all_sync(0xffffffffu, mbar_wait_cluster(acc_full(b), (uint32_t)(it >> 1) & 1u, kWaitLimit, abort))) {
+                if (lane == 0) give_up();
+                break;
+            }
+            tc_fence_after();
+            const int64_t row = (t / n_nt) * 2 * kPM + rank * kPM + warp * 32 + lane;
+            const int n0 = (int)(t % n_nt) * kPN;
+            const uint32_t trow = tmem + b * kAccCols + ((uint32_t)(warp * 32) << 16);
+#pragma unroll 1
+            for (int c0 = 0; c0 < kPN; c0 += 16) {
+                if (n0 + c0 >= N) break;  // warp-uniform
+                uint32_t v[16];
+                tc_ld16(trow + (uint32_t)c0, v);
+                tc_wait_ld();
+                if (row >= p.T) continue;
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int col = n0 + c0 + 8 * h;  // 8 columns = one 16-byte store
+                    if (col >= N) break;
+                    float f[8];
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) f[q] = __uint_as_float(v[8 * h + q]);
+                    Frag<bf16, 8> out;
+                    out.set(f);
+                    if (col < p.d) out.store(p.o + row * p.d + col);
+                    else out.store(p.keys + row * p.r + (col - p.d));
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(b ? acc_empty_leader1 : acc_empty_leader0);  // this half of b is read
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 4 && lane == 0) {
+        if (leader) {
+            // Normally every load was consumed; after a give-up, wait (bounded) for
+            // the stages still in flight before shared memory goes away.
+            for (int64_t g = issued - kPStages > 0 ? issued - kPStages : 0; g < issued; ++g)
+                if (!mbar_wait_cluster(full((int)(g % kPStages)), (uint32_t)(g / kPStages) & 1u, kWaitLimit, nullptr)) {
+                    if (p.status) atomicOr(p.status, LRAR_STATUS_WAIT_TIMEOUT);
+                }
+        } else if (*abort) {
+            const long long t0 = clock64();  // this CTA's own copies complete on the leader's barriers
+            while (clock64() - t0 < (1LL << 22)) {
+            }
+        }
+    }
+    __syncthreads();
+    cluster_sync();  // no MMA, copy or arrival of either CTA is pending past this point
+    if (warp == 5) {
+        tc_fence_after();
+        tmem_dealloc_pair(tmem, kTmemCols);
+    }
+}
+
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -285,23 +494,70 @@ int launch_project_t(const CUtensorMap &map_a, const void *w, int64_t T, int m, 
     return LRAR_OK;
 }
 
-// Relative rate of useful work with tile width BN: the share of SM time in
-// whole waves of one tile per SM, times the share of computed columns kept,
-// times the multiply-adds per operand byte of a 128 x BN tile (the shared-memory
-// feed per SM bounds the tensor pipe: measured rates follow BN / (128 + BN)).
-double tile_efficiency(int64_t T, int N, int BN, int sms) {
-    const int64_t nt = (N + BN - 1) / BN, tiles = (T + kPM - 1) / kPM * nt;
-    const double waves = (double)tiles / sms;
-    return waves / std::ceil(waves) * (double)N / (double)(nt * BN) * (double)BN / (double)(kPM + BN);
+template <int BN>
+int launch_project_pair_t(const CUtensorMap &map_a, const void *w, int64_t T, int m, int d, int r, void *o, void *keys,
+                          int *status, cudaStream_t s) {
+    CUtensorMap map_w;
+    if (!make_map(&map_w, w, d + r, m, BN / 2))
+        return record_error(LRAR_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point or arguments)");
+    constexpr size_t smem = ProjPairTile<BN>::kSmem;
+    const void *k = (const void *)proj_pair_kernel<BN>;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return record_error(LRAR_ERR_CUDA, cudaGetErrorString(e));
+    ProjParams p;
+    p.o = static_cast<bf16 *>(o);
+    p.keys = static_cast<bf16 *>(keys);
+    p.T = T;
+    p.m = m;
+    p.d = d;
+    p.r = r;
+    p.status = status;
+    const int64_t tiles = (T + 2 * kPM - 1) / (2 * kPM) * ((d + r + BN - 1) / BN);
+    // one cluster per pair of SMs that can hold it at once (persistent)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2, 1, 1);
+    cfg.blockDim = dim3(kPThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int clusters = 0;
+    e = cudaOccupancyMaxActiveClusters(&clusters, k, &cfg);
+    if (e != cudaSuccess) return record_error(LRAR_ERR_CUDA, cudaGetErrorString(e));
+    if (clusters < 1) return record_error(LRAR_ERR_CUDA, "no pair of SMs can hold the projection kernel");
+    const int grid = 2 * (int)(tiles < clusters ? tiles : clusters);
+    launch_pdl(proj_pair_kernel<BN>, grid, kPThreads, smem, s, map_a, map_w, p);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return record_error(LRAR_ERR_CUDA, cudaGetErrorString(e));
+    return LRAR_OK;
+}
+
+// Relative rate of useful work of a form and tile width: the share of SM time
+// in whole waves (one tile per SM, or per pair of SMs), times the share of
+// computed columns kept, times the rate the form reaches per busy SM at that
+// width (kRate, TFLOP/s measured on GB300 at m = 2816 and m = 2048, where the
+// main loop dominates; the pair form feeds each SM half of B per multiply-add).
+double tile_efficiency(int64_t T, int N, int BN, bool pair, int sms) {
+    const int rows = pair ? 2 * kPM : kPM, units = pair ? sms / 2 : sms;
+    const int64_t nt = (N + BN - 1) / BN, tiles = (T + rows - 1) / rows * nt;
+    const double waves = (double)tiles / units;
+    return waves / std::ceil(waves) * (double)N / (double)(nt * BN);
 }
 
 constexpr int kTileWidths[] = {160, 176, 192, 224, 240, 256};
+constexpr double kRate[2][6] = {{1300, 1400, 1480, 1615, 1620, 1700},   // single CTA
+                                {1340, 1470, 1560, 1650, 1740, 1840}};  // CTA pair
+constexpr int kPairTile = 2000;  // the test hook's code of the CTA-pair form: kPairTile + width
 
 }  // namespace
 
 bool project_tile_ok(int tile) {
     for (int c : kTileWidths)
-        if (c == tile) return true;
+        if (c == tile || c + kPairTile == tile) return true;
     return false;
 }
 
@@ -315,15 +571,23 @@ int launch_project(const void *a, const void *w, int64_t T, int m, int d, int r,
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     int bn = 0;
     double best = -1.0;
-    for (int c : kTileWidths) {  // the wider tile wins ties (fewer bytes per multiply-add)
-        const double e = tile_efficiency(T, d + r, c, sms);
-        if (e >= best * 1.001) {
-            best = e;
-            bn = c;
+    for (int form = 0; form < 2; ++form)
+        for (int i = 0; i < 6; ++i) {  // later candidates (wider, pair) win ties
+            const int c = kTileWidths[i];
+            const double e = tile_efficiency(T, d + r, c, form == 1, sms) * kRate[form][i];
+            if (e >= best * 1.001) {
+                best = e;
+                bn = form ? kPairTile + c : c;
+            }
         }
-    }
     if (tile != 0) bn = tile;  // forced by the test hook (checked by the caller)
     switch (bn) {
+        case kPairTile + 160: return launch_project_pair_t<160>(map_a, w, T, m, d, r, o, keys, status, s);
+        case kPairTile + 176: return launch_project_pair_t<176>(map_a, w, T, m, d, r, o, keys, status, s);
+        case kPairTile + 192: return launch_project_pair_t<192>(map_a, w, T, m, d, r, o, keys, status, s);
+        case kPairTile + 224: return launch_project_pair_t<224>(map_a, w, T, m, d, r, o, keys, status, s);
+        case kPairTile + 240: return launch_project_pair_t<240>(map_a, w, T, m, d, r, o, keys, status, s);
+        case kPairTile + 256: return launch_project_pair_t<256>(map_a, w, T, m, d, r, o, keys, status, s);
         case 160: return launch_project_t<160>(map_a, w, T, m, d, r, o, keys, status, s);
         case 176: return launch_project_t<176>(map_a, w, T, m, d, r, o, keys, status, s);
         case 192: return launch_project_t<192>(map_a, w, T, m, d, r, o, keys, status, s);

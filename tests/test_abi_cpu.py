@@ -312,6 +312,8 @@ def test_test_hooks_reject(lib):
     assert t(0, 1, FAKE, FAKE, 8, 64, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_INVALID_ARG
     assert t(200, 1, FAKE, FAKE, 8, 64, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_INVALID_ARG
     assert t(160, 1, FAKE, FAKE, 0, 64, 64, 16, FAKE, FAKE, None, None) == lrar.OK  # T == 0
+    assert t(2176, 1, FAKE, FAKE, 0, 64, 64, 16, FAKE, FAKE, None, None) == lrar.OK  # CTA-pair form, T == 0
+    assert t(2200, 1, FAKE, FAKE, 8, 64, 64, 16, FAKE, FAKE, None, None) == lrar.ERR_INVALID_ARG
     s = lib.lrar_test_block_phase1_stalled
     args = [1, 1, 1, FAKE, None, FAKE, 4, 8, 16, 64, 8, EPS, FAKE, FAKE]
     assert s(*args, None, 1000, None) == lrar.ERR_INVALID_ARG      # status required

@@ -60,7 +60,8 @@ def _compare(T, m, d, r, seed=3, tokens=None, tile=0):
 
 
 def test_whole_tiles():
-    """T = 256 (two 128-row tiles), m = d = 1024, r = 32: N = 1056 = 6 tiles of 176."""
+    """T = 256 (one 256-row tile of the CTA-pair form, two 128-row tiles of the
+    single-CTA form), m = d = 1024, r = 32 (N = 1056)."""
     _compare(256, 1024, 1024, 32)
 
 
@@ -75,6 +76,14 @@ def test_every_tile_width(width):
     """Each compiled tile width (forced through the lrar_test_project_tile hook)
     on ragged T, m and N, the value/key split falling inside a tile."""
     _compare(300, 1000, 1024, 16, seed=4, tile=width)
+
+
+@pytest.mark.parametrize("width", [160, 176, 192, 224, 240, 256])
+def test_every_pair_tile_width(width):
+    """The CTA-pair (two-SM, tcgen05.mma.cta_group::2) form at each width
+    (hook code 2000 + width): 256-row tiles split over the two CTAs of a
+    cluster, on ragged T, m and N."""
+    _compare(300, 1000, 1024, 16, seed=4, tile=2000 + width)
 
 
 def test_swiglu_output_projection():
@@ -101,8 +110,8 @@ def test_full_size_sampled_tokens():
 
 
 def test_large_decoder_sampled_tokens():
-    """The d = 2048 decoder (m = d = 2048, r = 64, T = 32768): d + r = 2112 is
-    twelve 176-wide tiles, the other tile width of the kernel."""
+    """The d = 2048 decoder (m = d = 2048, r = 64, T = 32768): d + r = 2112
+    columns in 240-wide tiles of the CTA-pair form, the last one partly outside."""
     g = np.random.default_rng(10)
     tokens = np.sort(np.concatenate([g.choice(32768, 24, replace=False), [0, 32767]]))
     _compare(32768, 2048, 2048, 64, seed=10, tokens=tokens)
