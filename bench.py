@@ -514,11 +514,16 @@ def run_profile_proj(args):
     w = (synth.randn((d + r, m), 1, "proj_w", device=dev) / m ** 0.5).to(torch.bfloat16)
     o = torch.empty(T, d, dtype=torch.bfloat16, device=dev) if d else None
     k = torch.empty(T, r, dtype=torch.bfloat16, device=dev)
+    if args.proj_tile:  # form and width forced through the test hook (2000 + width: CTA pair)
+        call = lambda: lrar.test_project_tile(args.proj_tile, a, w, o, k)  # noqa: E731
+    else:
+        call = lambda: lrar.project(a, w, o, k)  # noqa: E731
     for _ in range(args.warmup):
-        lrar.project(a, w, o, k)
-    ms = _median_ms(torch, lambda: lrar.project(a, w, o, k), args.steps)
+        call()
+    ms = _median_ms(torch, call, args.steps)
     flops = 2.0 * T * m * (d + r)
-    print(json.dumps({"profile_proj": m, "T": T, "d": d, "r": r, "ms": ms, "tflops": flops / ms / 1e9}), flush=True)
+    print(json.dumps({"profile_proj": m, "T": T, "d": d, "r": r, "tile": args.proj_tile or "chosen", "ms": ms,
+                      "tflops": flops / ms / 1e9}), flush=True)
 
 
 def _median_ms(torch, fn, reps):
@@ -924,6 +929,8 @@ def main():
                     help="time the Block two-phase path on this many tokens (profiling)")
     ap.add_argument("--profile-proj", type=int, default=0,
                     help="time the fused projection with this input width m (profiling; --tokens, --site-d, --site-r)")
+    ap.add_argument("--proj-tile", type=int, default=0,
+                    help="--profile-proj: force the tile width (160..256, or 2000 + width for the CTA-pair form)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
