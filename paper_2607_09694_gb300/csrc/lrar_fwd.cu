@@ -200,6 +200,18 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
             cp_async_wait_all();
             __syncwarp();  // every lane's pieces are visible to the warp
         }
+        // the token's first rows do not depend on the weights: their loads go out
+        // before the routing, so the two latencies overlap
+        const int pre = p.n < U ? p.n : U;
+        Frag<Tin, E> f0[U][V];
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (u < pre && e < dc) f0[u][v].load_nc(src_row<Tin>(p.vt, u, x, p.d) + e0 + e);
+                else f0[u][v].zero();
+            }
         const float lse = lr_route<Tin>(p.vt, p.kt, p.n, p.d, p.r, p.eps, p.inv_r, p.sliced, p.key_vec, x,
                                         lane, q_s, a_s, nullptr, nullptr, KS ? kb_s : nullptr);
         if (lane == 0 && p.lse && e0 == 0) p.lse[x] = lse;
@@ -214,7 +226,20 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
         float acc[V * E];
 #pragma unroll
         for (int t = 0; t < V * E; ++t) acc[t] = 0.f;
-        int i = 0;
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            if (u < pre) {
+                const float a = a_s[u];
+#pragma unroll
+                for (int v = 0; v < V; ++v) {
+                    float o[E];
+                    f0[u][v].get(o);
+#pragma unroll
+                    for (int t = 0; t < E; ++t) acc[v * E + t] = fmaf(a, o[t], acc[v * E + t]);
+                }
+            }
+        }
+        int i = pre;
         for (; i + U <= p.n; i += U) {
             if (!staged && i == pf_at) stage_next();
             Frag<Tin, E> f[U][V];
