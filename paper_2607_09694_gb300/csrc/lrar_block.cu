@@ -21,6 +21,9 @@
 // and one named barrier per pass: the chunk warps score token p + 2 (split by
 // source: each warp scores its sources against every query), take the softmax
 // of token p + 1 (split by query), and mix token p.
+#include <algorithm>
+#include <type_traits>
+
 #include "lrar.h"
 #include "lrar_device.cuh"
 #include "lrar_launch.h"
@@ -45,6 +48,7 @@ struct Ph1Params {
     int *status;            // optional: LRAR_STATUS_WAIT_TIMEOUT when a key wait gives up
     long long wait_cycles;  // bound of each key wait
     int stall;              // test hook: key waits go to a barrier that never completes
+    int tw;                 // weights kernel on the tensor cores: tokens per warp chunk
 };
 
 // Coordinate t of query j (zero past c and r), read from the caller's array.
@@ -484,6 +488,398 @@ __global__ void __launch_bounds__(kThreads, 2) block_phase1_kernel(const __grid_
         }
 }
 
+// ----------------------------------------------------- split phase 1 ----
+// Phase 1 in two kernels, for shapes whose weights fit one row of h_pre:
+//   block_weights_kernel (bf16 keys of depth 16..64: block_weights_mma_kernel,
+//       the scores on the tensor cores)  computes s_ij (Eq. 8-9) for every
+//       completed source i and site j, the softmax over i (Eq. 10) and lse_j,
+//       writes lse_j to lse_pre and alpha_ij as fp32 at float i * 8 + j of the
+//       token's row of the last site's h_pre, which serves as scratch;
+//   block_mix_kernel  the mix of phase 1 with those weights: in pass p a token
+//       group copies token p + 1's weights from that row into shared memory and
+//       mixes token p, whose row the last site then overwrites with its h_pre.
+//       Its first source rows stream in while the weights kernel finishes.
+// The mix carries no scoring, so its instructions go to the row stream and
+// the multiply-adds.
+
+// The fp32 weight row of token x: the start of the last site's h_pre row.
+template <typename Tout>
+__device__ __forceinline__ float *ph1_weight_row(const Ph1Params &p, int64_t x) {
+    return reinterpret_cast<float *>(static_cast<Tout *>(p.h_pre) + (int64_t)(p.c - 1) * p.site_stride + x * p.d);
+}
+
+// Scores of kWTok tokens at once (keys that are whole 16-byte vectors whose
+// nv = r / E vectors divide a warp): lane (source i0 + l / nv, vector l % nv)
+// loads its key vector of every round and token before any arithmetic, so the
+// loads of all of them are in flight together; then, round by round, |k|^2 and
+// the eight q_j . k products (a fixed butterfly over the nv lanes, the
+// arithmetic of ph1_scores) give s_ij = rho_i (q_j . k_i) in sc[t][i][j].
+constexpr int kWTok = 2;     // tokens per warp and iteration of the weights kernel
+constexpr int kWRounds = 4;  // source rounds whose key vectors are held at once
+template <typename Tin>
+__device__ __forceinline__ void ph1_scores_batch(const Ph1Params &p, const float *__restrict__ q_s, int rp,
+                                                 const int64_t (&xs)[kWTok], int lane, float *sc) {
+    constexpr int E = VecE<Tin>::value;
+    const int nv = p.r / E, per = 32 / nv, v = lane % nv, so = lane / nv;
+    for (int i0 = 0; i0 < p.n; i0 += kWRounds * per) {
+        Frag<Tin, E> k[kWTok][kWRounds];
+#pragma unroll
+        for (int t = 0; t < kWTok; ++t)
+#pragma unroll
+            for (int rr = 0; rr < kWRounds; ++rr) {
+                const int i = i0 + rr * per + so;
+                if (xs[t] < p.T && i < p.n) k[t][rr].load_nc(ph1_key<Tin>(p, i, xs[t]) + v * E);
+                else k[t][rr].zero();
+            }
+#pragma unroll
+        for (int t = 0; t < kWTok; ++t)
+#pragma unroll
+            for (int rr = 0; rr < kWRounds; ++rr) {
+                const int i = i0 + rr * per + so;
+                if (i0 + rr * per >= p.n) break;  // warp-uniform
+                float kv[E];
+                k[t][rr].get(kv);
+                float ss = 0.f, qk[kPh1MaxSites];
+#pragma unroll
+                for (int e = 0; e < E; ++e) ss = fmaf(kv[e], kv[e], ss);
+#pragma unroll
+                for (int j = 0; j < kPh1MaxSites; ++j) {
+                    qk[j] = 0.f;
+                    const float *qj = q_s + j * rp + v * E;
+#pragma unroll
+                    for (int e = 0; e < E; e += 4) {
+                        const float4 q4 = *reinterpret_cast<const float4 *>(qj + e);
+                        qk[j] = fmaf(q4.x, kv[e], qk[j]);
+                        qk[j] = fmaf(q4.y, kv[e + 1], qk[j]);
+                        qk[j] = fmaf(q4.z, kv[e + 2], qk[j]);
+                        qk[j] = fmaf(q4.w, kv[e + 3], qk[j]);
+                    }
+                }
+                for (int off = 1; off < nv; off <<= 1) {  // the source's lanes form an aligned group
+                    ss += __shfl_xor_sync(0xffffffffu, ss, off);
+#pragma unroll
+                    for (int j = 0; j < kPh1MaxSites; ++j) qk[j] += __shfl_xor_sync(0xffffffffu, qk[j], off);
+                }
+                if (v == 0 && i < p.n) {
+                    const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
+#pragma unroll
+                    for (int j = 0; j < kPh1MaxSites; ++j) sc[(t * p.n + i) * kPh1MaxSites + j] = rho * qk[j];
+                }
+            }
+    }
+}
+
+template <typename Tin, typename Tout>
+__global__ void __launch_bounds__(kThreads) block_weights_kernel(const __grid_constant__ Ph1Params p) {
+    pdl_enter();
+    extern __shared__ __align__(16) float wsm[];
+    const int rp = round_up(p.r, 4);
+    float *q_s = wsm;                                       // [8][rp], zero past c and r
+    float *sc_all = q_s + kPh1MaxSites * rp;                // [kWarps][kWTok][n][8]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int j = threadIdx.x; j < kPh1MaxSites * rp; j += kThreads) {
+        const int jj = j / rp, t = j % rp;
+        q_s[j] = (jj < p.c && t < p.r) ? p.queries[jj * p.r + t] : 0.f;
+    }
+    __syncthreads();
+    float *sc = sc_all + (size_t)warp * kWTok * kPh1MaxSites * p.n;
+    const int nv = p.key_vec ? p.r / VecE<Tin>::value : 0;
+    const bool batch = nv >= 1 && nv <= 32 && 32 % nv == 0;
+    const int j = lane >> 2, slot = lane & 3;  // softmax: lane (j, slot) takes sources slot, slot + 4, ...
+    const int64_t wstride = (int64_t)gridDim.x * kWarps;
+    for (int64_t x0 = ((int64_t)blockIdx.x * kWarps + warp) * kWTok; x0 < p.T; x0 += wstride * kWTok) {
+        int64_t xs[kWTok];
+#pragma unroll
+        for (int t = 0; t < kWTok; ++t) xs[t] = x0 + t;
+        if (batch) {
+            ph1_scores_batch<Tin>(p, q_s, rp, xs, lane, sc);
+        } else {
+            for (int t = 0; t < kWTok; ++t)
+                if (xs[t] < p.T) ph1_scores<Tin, kPh1MaxSites>(p, q_s, rp, xs[t], lane, 0, 1, sc + t * p.n * kPh1MaxSites, nullptr);
+        }
+        __syncwarp();
+#pragma unroll
+        for (int t = 0; t < kWTok; ++t) {
+            if (xs[t] >= p.T) break;  // warp-uniform
+            const float *st = sc + t * p.n * kPh1MaxSites;
+            float m = -INFINITY;
+            for (int i = slot; i < p.n; i += 4) m = fmaxf(m, st[i * kPh1MaxSites + j]);
+            m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
+            m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
+            float z = 0.f;
+            for (int i = slot; i < p.n; i += 4) z += expf(st[i * kPh1MaxSites + j] - m);
+            z += __shfl_xor_sync(0xffffffffu, z, 1);
+            z += __shfl_xor_sync(0xffffffffu, z, 2);
+            float *wrow = ph1_weight_row<Tout>(p, xs[t]);
+            if (j < p.c) {
+                for (int i = slot; i < p.n; i += 4) wrow[i * kPh1MaxSites + j] = expf(st[i * kPh1MaxSites + j] - m) / z;
+                if (slot == 0) p.lse_pre[(int64_t)j * p.T + xs[t]] = m + logf(z);
+            }
+        }
+        __syncwarp();  // the scores are rewritten for the next tokens
+    }
+}
+
+// ---------------------------------------------- weights on the tensor cores ----
+// With bf16 keys of depth r = 16 KS the scores of a chunk of tokens are one
+// small contraction: rows are the chunk's (token, source) pairs, columns the
+// c <= 8 queries.  It runs as m16n8k16 MMAs.  Each fp32 query coordinate is
+// split exactly into three bf16 parts q = q1 + q2 + q3 (each part the bf16
+// rounding of what the previous ones leave, so that together they carry q's
+// 24-bit significand); every bf16 product q_u k is exact and the MMA sums in
+// fp32, so s_ij = rho_i (q_j . k_i) comes out with fp32 accuracy.  The depth
+// index is permuted so that lane t of a quad holds one contiguous quarter of a
+// key row (depth 4 KS t ... 4 KS t + 4 KS - 1): depth 4 KS t + 4 s + {0, 1} is
+// column {2t, 2t + 1} of k-step s and 4 KS t + 4 s + {2, 3} column
+// {2t + 8, 2t + 9}; the queries take the same permutation, which leaves the
+// contraction unchanged.  |k_i|^2 comes from the same registers (mixed-precision
+// multiply-adds, then the quad's four lanes).
+__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                               uint32_t b0, uint32_t b1) {
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// ss += lo^2 + hi^2 of a bf16 pair (exact products, fp32 sums).
+__device__ __forceinline__ void sumsq_bf16x2(float &ss, uint32_t w) {
+    asm("{\n\t.reg .b16 l, h;\n\tmov.b32 {l, h}, %1;\n\t"
+        "fma.rn.f32.bf16 %0, l, l, %0;\n\tfma.rn.f32.bf16 %0, h, h, %0;\n\t}"
+        : "+f"(ss)
+        : "r"(w));
+}
+
+// The three bf16 parts of x (x = u0 + u1 + u2 up to 2^-27 |x|).
+__device__ __forceinline__ void split3_bf16(float x, bf16 (&u)[3]) {
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+        u[k] = __float2bfloat16_rn(x);
+        x -= __bfloat162float(u[k]);  // exact: the rounding error of a bf16 rounding is an fp32 number
+    }
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(bf16 lo, bf16 hi) {
+    return (uint32_t)__bfloat16_as_ushort(lo) | ((uint32_t)__bfloat16_as_ushort(hi) << 16);
+}
+
+template <typename Tout, int KS>
+__global__ void __launch_bounds__(kThreads, 2) block_weights_mma_kernel(const __grid_constant__ Ph1Params p) {
+    pdl_enter();
+    constexpr int W = 2 * KS;                  // bf16 pairs of a key row per lane
+    constexpr int G = KS >= 3 ? 4 : 8 / KS;    // tiles of 16 pairs whose rows are loaded together
+    extern __shared__ __align__(16) float wsm[];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int g = lane >> 2, t4 = lane & 3;
+    const int tw = p.tw, n = p.n;
+    float *sc = wsm + (size_t)warp * tw * n * kPh1MaxSites;  // [tw * n][8] scores of the warp's chunk
+    // B fragments: query g's depth quarter t4, three parts each
+    uint32_t qb[3][KS][2];
+#pragma unroll
+    for (int s = 0; s < KS; ++s)
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int e = 4 * KS * t4 + 4 * s + 2 * h;
+            bf16 u0[3], u1[3];
+            split3_bf16(g < p.c ? p.queries[g * p.r + e] : 0.f, u0);
+            split3_bf16(g < p.c ? p.queries[g * p.r + e + 1] : 0.f, u1);
+#pragma unroll
+            for (int k = 0; k < 3; ++k) qb[k][s][h] = pack_bf16(u0[k], u1[k]);
+        }
+    const uint64_t magic = 0xFFFFFFFFull / (uint32_t)n + 1;  // P / n = (P * magic) >> 32 for P < 2^32 / n
+    const int64_t nchunks = (p.T + tw - 1) / tw;
+    for (int64_t ch = (int64_t)blockIdx.x * kWarps + warp; ch < nchunks; ch += (int64_t)gridDim.x * kWarps) {
+        const int64_t x0 = ch * tw;
+        const int tcount = (int)(p.T - x0 < tw ? p.T - x0 : tw);
+        const int np = tcount * n;  // pairs (token u, source i) at u * n + i
+        for (int tile0 = 0; tile0 * 16 < np; tile0 += G) {
+            uint32_t w[G][2][W];  // rows g and g + 8 of each tile
+#pragma unroll
+            for (int gi = 0; gi < G; ++gi)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int P = (tile0 + gi) * 16 + g + 8 * h;
+                    if (P < np) {
+                        const int u = (int)(((uint64_t)P * magic) >> 32), i = P - u * n;
+                        const bf16 *kr = ph1_key<bf16>(p, i, x0 + u) + 4 * KS * t4;
+                        if constexpr (KS % 2 == 0) {
+#pragma unroll
+                            for (int v = 0; v < KS / 2; ++v) {
+                                const uint4 q4 = ld_nc16(kr + 8 * v);
+                                w[gi][h][4 * v] = q4.x; w[gi][h][4 * v + 1] = q4.y;
+                                w[gi][h][4 * v + 2] = q4.z; w[gi][h][4 * v + 3] = q4.w;
+                            }
+                        } else {
+#pragma unroll
+                            for (int v = 0; v < KS; ++v) {
+                                const uint2 q2 = ld_nc8(kr + 4 * v);
+                                w[gi][h][2 * v] = q2.x; w[gi][h][2 * v + 1] = q2.y;
+                            }
+                        }
+                    } else {
+#pragma unroll
+                        for (int v = 0; v < W; ++v) w[gi][h][v] = 0u;
+                    }
+                }
+#pragma unroll
+            for (int gi = 0; gi < G; ++gi) {
+                const int P0 = (tile0 + gi) * 16 + g;
+                if ((tile0 + gi) * 16 >= np) break;  // warp-uniform
+                float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                for (int k = 2; k >= 0; --k)  // smallest parts first
+#pragma unroll
+                    for (int s = 0; s < KS; ++s)
+                        mma_bf16_16816(acc, w[gi][0][2 * s], w[gi][1][2 * s], w[gi][0][2 * s + 1], w[gi][1][2 * s + 1],
+                                       qb[k][s][0], qb[k][s][1]);
+                float ss0 = 0.f, ss1 = 0.f;
+#pragma unroll
+                for (int v = 0; v < W; ++v) {
+                    sumsq_bf16x2(ss0, w[gi][0][v]);
+                    sumsq_bf16x2(ss1, w[gi][1][v]);
+                }
+                ss0 += __shfl_xor_sync(0xffffffffu, ss0, 1);
+                ss1 += __shfl_xor_sync(0xffffffffu, ss1, 1);
+                ss0 += __shfl_xor_sync(0xffffffffu, ss0, 2);
+                ss1 += __shfl_xor_sync(0xffffffffu, ss1, 2);
+                const float rho0 = rsqrtf(fmaf(ss0, p.inv_r, p.eps)), rho1 = rsqrtf(fmaf(ss1, p.inv_r, p.eps));
+                if (P0 < np)
+                    *reinterpret_cast<float2 *>(sc + P0 * kPh1MaxSites + 2 * t4) = make_float2(rho0 * acc[0], rho0 * acc[1]);
+                if (P0 + 8 < np)
+                    *reinterpret_cast<float2 *>(sc + (P0 + 8) * kPh1MaxSites + 2 * t4) =
+                        make_float2(rho1 * acc[2], rho1 * acc[3]);
+            }
+        }
+        __syncwarp();
+        // softmax over the sources: lane (u0, j) takes tokens u0, u0 + 4, ... of the chunk for query j
+        const int j = lane & 7;
+        for (int u = lane >> 3; u < tcount; u += 4) {
+            float *st = sc + u * n * kPh1MaxSites + j;
+            float m = -INFINITY;
+            for (int i = 0; i < n; ++i) m = fmaxf(m, st[i * kPh1MaxSites]);
+            float z = 0.f;
+            for (int i = 0; i < n; ++i) {
+                const float e = expf(st[i * kPh1MaxSites] - m);
+                st[i * kPh1MaxSites] = e;
+                z += e;
+            }
+            if (j < p.c) {
+                float *wrow = ph1_weight_row<Tout>(p, x0 + u);
+                for (int i = 0; i < n; ++i) wrow[i * kPh1MaxSites + j] = st[i * kPh1MaxSites] / z;
+                p.lse_pre[(int64_t)j * p.T + x0 + u] = m + logf(z);
+            }
+        }
+        __syncwarp();  // the scores are rewritten for the next chunk
+    }
+}
+
+template <typename Tin, typename Tout, int S, bool C8, bool FULLW>
+__global__ void __launch_bounds__(kThreads, 2) block_mix_kernel(const __grid_constant__ Ph1Params p) {
+    constexpr int E = VecE<Tin>::value;
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int G = kWarps / p.chunks;  // token groups per CTA
+    float *a_all = reinterpret_cast<float *>(smem_raw + (size_t)kWarps * S * 32 * 16);  // [G][2][n][8]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int g = warp / p.chunks, ch = warp % p.chunks;
+    const int nthr = p.chunks * 32;
+    const int gt = ch * 32 + lane;  // thread index within the group
+    Tout *__restrict__ h_pre = static_cast<Tout *>(p.h_pre);
+    const int e = (ch * 32 + lane) * E;
+    float *aw0 = a_all + (size_t)g * 2 * kPh1MaxSites * p.n;
+    auto awb = [&](int q) { return aw0 + (q & 1) * kPh1MaxSites * p.n; };
+    const int n4 = p.n * kPh1MaxSites / 4;  // 16-byte pieces of a token's weights
+    auto fetch = [&](int q, int64_t xx) {   // token q = xx of the group: its weights into shared memory
+        const float4 *src = reinterpret_cast<const float4 *>(ph1_weight_row<Tout>(p, xx));
+        float4 *dst = reinterpret_cast<float4 *>(awb(q));
+        for (int t = gt; t < n4; t += nthr) dst[t] = src[t];
+    };
+    const int64_t stride = (int64_t)gridDim.x * G;
+    const uint32_t ring_w = smem_u32(smem_raw) + (uint32_t)(warp * S * 32 * 16) + 16u * lane;
+
+    int64_t x = (int64_t)blockIdx.x * G + g;
+    const bool cp_lane = FULLW || e < p.d;
+    const int64_t xstep = stride * p.d;
+    int64_t xoff = x * p.d + e;
+    int ii = 0;
+    int rows_left = x < p.T ? (int)((p.T - x + stride - 1) / stride) * p.n : 0;  // warp-uniform
+    uint32_t wslot = ring_w;
+    const uint32_t ring_end = ring_w + 16u * 32u * S;
+    auto issue = [&]() {
+        if (rows_left > 0) {
+            if (cp_lane) cp_async16(wslot, static_cast<const Tin *>(p.vt.p[ii]) + xoff);
+            --rows_left;
+            if (++ii == p.n) {
+                ii = 0;
+                xoff += xstep;
+            }
+        }
+        cp_async_commit();
+        wslot += 16u * 32u;
+        if (wslot == ring_end) wslot = ring_w;
+    };
+#pragma unroll
+    for (int st = 0; st < S - 1; ++st) issue();
+    // The first rows stream in before the wait: they are completed sources,
+    // written before the weights kernel that precedes this grid began, and that
+    // kernel lets this grid start only after its own wait on its predecessors.
+    // The weights, that kernel's output, are read after the wait.
+    pdl_wait();
+    pdl_launch_dependents();
+    uint32_t rslot = ring_w;
+    Frag<Tin, E> f;
+    auto read_row = [&]() {
+        if (cp_lane) f.a = ld_shared16(rslot);
+        else f.zero();
+        rslot += 16u * 32u;
+        if (rslot == ring_end) rslot = ring_w;
+    };
+    auto next_row = [&]() {
+        issue();
+        cp_async_wait<S - 2>();
+        read_row();
+    };
+
+    if (x < p.T) fetch(0, x);
+    group_sync(1 + g, nthr);
+    for (int pass = 0; (int64_t)blockIdx.x * G + pass * stride < p.T; ++pass, x += stride) {
+        const float *aw = awb(pass);
+        // token pass + 1's weights: its h_pre rows are written only in the next pass
+        if (x + stride < p.T) fetch(pass + 1, x + stride);
+        if (x < p.T) {
+            float acc[kPh1MaxSites][E];
+            cp_async_wait<S - 2>();
+            read_row();
+            if (C8) {
+                ph1_row<Tin, E, C8, true>(acc, f, aw, p.c);
+            } else {
+#pragma unroll
+                for (int j = 0; j < kPh1MaxSites; ++j)
+#pragma unroll
+                    for (int t = 0; t < E; ++t) acc[j][t] = 0.f;
+                ph1_row<Tin, E, C8, false>(acc, f, aw, p.c);
+            }
+            for (int i = 1; i < p.n; ++i) {
+                next_row();
+                ph1_row<Tin, E, C8, false>(acc, f, aw + i * kPh1MaxSites, p.c);
+            }
+            issue();  // the stream stays S - 1 copies ahead of the next token's first row
+            if (FULLW || e < p.d) {
+                Tout *hp = h_pre + x * p.d + e;
+#pragma unroll
+                for (int j = 0; j < kPh1MaxSites; ++j) {
+                    if (C8 || j < p.c) {
+                        Frag<Tout, E> out;
+                        out.set(acc[j]);
+                        out.store(hp + (int64_t)j * p.site_stride);
+                    }
+                }
+            }
+        }
+        group_sync(1 + g, nthr);  // next weights copied; this token's weight row is overwritten
+    }
+    cp_async_wait_all();
+}
+
 struct Ph2Params {
     const void *h_pre, *partial, *pkeys;
     const float *lse_pre, *query;
@@ -622,6 +1018,7 @@ static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
     int chunks = 1;
     while (chunks < chunks_needed) chunks *= 2;  // 1, 2, 4 or 8 (validated: d <= 8 * 32 * E)
     Ph1Params p;
+    p.tw = 1;
     for (int i = 0; i < kMaxTab; ++i) {
         p.vt.p[i] = i < a.n ? a.values[i] : nullptr;
         p.kt.p[i] = (i < a.n && a.keys) ? a.keys[i] : nullptr;
@@ -659,6 +1056,42 @@ static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
             if (e != cudaSuccess) return e;
         }
     const int grid = persistent_grid(k_gen, kThreads, smem, (a.T + G - 1) / G, 1 << 30);
+    // split phase 1 (weights kernel, then the mix) when a token's weights fit the
+    // last site's row of h_pre; the stall test hook keeps the key-staging kernel
+    const bool split = !a.stall && (size_t)a.n * kPh1MaxSites * sizeof(float) <= (size_t)a.d * sizeof(Tout);
+    size_t smem_w =
+        sizeof(float) * ((size_t)kPh1MaxSites * round_up(a.r, 4) + (size_t)kWarps * kWTok * kPh1MaxSites * a.n);
+    const size_t smem_m = (size_t)kWarps * S * 32 * 16 + sizeof(float) * (size_t)G * 2 * kPh1MaxSites * a.n;
+    // bf16 keys of depth 16, 32, 48 or 64 as whole vectors: scores on the tensor cores
+    const int kst = (a.r % 16 == 0 && a.r <= 64) ? a.r / 16 : 0;  // k-steps of the MMA
+    const bool mma = std::is_same<Tin, bf16>::value && p.key_vec && kst > 0;
+    const void *kw = !mma ? (const void *)block_weights_kernel<Tin, Tout>
+                   : kst == 1 ? (const void *)block_weights_mma_kernel<Tout, 1>
+                   : kst == 2 ? (const void *)block_weights_mma_kernel<Tout, 2>
+                   : kst == 3 ? (const void *)block_weights_mma_kernel<Tout, 3>
+                             : (const void *)block_weights_mma_kernel<Tout, 4>;
+    // tokens per warp chunk: enough chunks for every resident warp, at most 16, scores within 8 KB a warp
+    const int tw_max = std::max(1, std::min(16, 256 / a.n));
+    if (mma) smem_w = sizeof(float) * (size_t)kWarps * tw_max * kPh1MaxSites * a.n;
+    const void *km_fast = (const void *)block_mix_kernel<Tin, Tout, S, true, true>;
+    const void *km_gen = (const void *)block_mix_kernel<Tin, Tout, S, false, false>;
+    int grid_w = 0, grid_m = 0;
+    if (split) {
+        for (const void *kk : {kw, km_fast, km_gen}) {
+            const size_t sm = kk == kw ? smem_w : smem_m;
+            cudaError_t e = cudaFuncSetAttribute(kk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+            if (e != cudaSuccess) return e;
+        }
+        if (mma) {
+            const int64_t slots = (int64_t)persistent_grid(kw, kThreads, smem_w, 1 << 30, 1 << 30) * kWarps;
+            p.tw = (int)std::max<int64_t>(1, std::min<int64_t>(tw_max, (a.T + slots - 1) / slots));
+            const int64_t nchunks = (a.T + p.tw - 1) / p.tw;
+            grid_w = (int)std::min<int64_t>(slots / kWarps, (nchunks + kWarps - 1) / kWarps);
+        } else {
+            grid_w = persistent_grid(kw, kThreads, smem_w, (a.T + kWarps * kWTok - 1) / (kWarps * kWTok), 1 << 30);
+        }
+        grid_m = persistent_grid(km_gen, kThreads, smem_m, (a.T + G - 1) / G, 1 << 30);
+    }
     for (int j0 = 0; j0 < a.c; j0 += kPh1MaxSites) {  // groups of at most 8 queries
         p.c = a.c - j0 < kPh1MaxSites ? a.c - j0 : kPh1MaxSites;
         p.queries = a.queries + (size_t)j0 * a.r;
@@ -666,6 +1099,18 @@ static cudaError_t launch_ph1_t(const BlockPh1Args &a, cudaStream_t s) {
         p.lse_pre = a.lse_pre + (size_t)j0 * a.T;
         const bool fast = p.c == kPh1MaxSites && fullw;
         cudaError_t e;
+        if (split) {
+            if (!mma) launch_pdl(block_weights_kernel<Tin, Tout>, grid_w, kThreads, smem_w, s, p);
+            else if (kst == 1) launch_pdl(block_weights_mma_kernel<Tout, 1>, grid_w, kThreads, smem_w, s, p);
+            else if (kst == 2) launch_pdl(block_weights_mma_kernel<Tout, 2>, grid_w, kThreads, smem_w, s, p);
+            else if (kst == 3) launch_pdl(block_weights_mma_kernel<Tout, 3>, grid_w, kThreads, smem_w, s, p);
+            else launch_pdl(block_weights_mma_kernel<Tout, 4>, grid_w, kThreads, smem_w, s, p);
+            if ((e = cudaGetLastError()) != cudaSuccess) return e;
+            if (fast) launch_pdl(block_mix_kernel<Tin, Tout, S, true, true>, grid_m, kThreads, smem_m, s, p);
+            else launch_pdl(block_mix_kernel<Tin, Tout, S, false, false>, grid_m, kThreads, smem_m, s, p);
+            if ((e = cudaGetLastError()) != cudaSuccess) return e;
+            continue;
+        }
         if (ks) e = fast ? ph1_go<Tin, Tout, true, true>(p, grid, smem, s) : ph1_go<Tin, Tout, true, false>(p, grid, smem, s);
         else e = fast ? ph1_go<Tin, Tout, false, true>(p, grid, smem, s) : ph1_go<Tin, Tout, false, false>(p, grid, smem, s);
         if (e != cudaSuccess) return e;

@@ -179,6 +179,14 @@ __device__ __forceinline__ void pdl_enter() {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
+// The same two steps apart, for a kernel that starts reading inputs written
+// before its predecessor began (never its predecessor's own outputs) ahead of
+// the wait.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ----------------------------------------------------------- reductions ---
 // xor butterflies leave the identical bit pattern in every lane.
 __device__ __forceinline__ float warp_sum(float v) {

@@ -109,6 +109,21 @@ def test_bf16_members_d2048(b):
         H.assert_abs(f"lse[site {j}]", lse, ref["lse"], 1e-4)
 
 
+@pytest.mark.parametrize("variant,r,c,b,T", [("sliced", 32, 8, 1, 333), ("sliced", 48, 5, 2, 333),
+                                               ("projected", 32, 8, 2, 333), ("projected", 16, 3, 4, 333),
+                                               ("sliced", 64, 8, 15, 333), ("sliced", 32, 8, 3, 20011)])
+def test_bf16_key_depths(variant, r, c, b, T):
+    """bf16 sources with keys of depth 16, 32, 48 and 64 (the phase-1 scores on the
+    tensor cores, one to four k-steps), up to 16 completed sources, fewer than 8
+    sites, and a token count that leaves several tokens per warp and a ragged
+    last chunk (T = 20011).  Both sides mix the same bf16 sources, so h is held
+    to the fp32 bar."""
+    for j, (h, lse), ref, _ in _run(variant, c=c, b=b, T=T, d=256, r=r, store="bf16", stack="bf16", pre="f32",
+                                    seed=19 + r + b):
+        H.assert_abs(f"h[site {j}]", h, ref["h"])
+        H.assert_abs(f"lse[site {j}]", lse, ref["lse"], 1e-4)
+
+
 def test_bf16_phase1_outputs_within_one_rounding():
     """With a bf16 h_pre, phase 2 sees the completed-source mix rounded once; its
     weight is at most 1, so h moves by at most half a bf16 spacing of that mix
