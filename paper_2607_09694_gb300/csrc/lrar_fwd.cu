@@ -240,6 +240,7 @@ __global__ void __launch_bounds__(kThreads, (V <= 4 ? 2 : 1)) fwd_lr_kernel(cons
             }
         }
         int i = pre;
+        if (!staged && pf_at < i) stage_next();  // the staging point falls among the preloaded rows
         for (; i + U <= p.n; i += U) {
             if (!staged && i == pf_at) stage_next();
             Frag<Tin, E> f[U][V];
