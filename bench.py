@@ -665,11 +665,7 @@ def run_suite(args):
                 for j in range(1, ns):
                     lrar.block_phase2("sliced", h_pre[j], lse_pre[j], stack[1 + b], None, qs[t0 - 1 + j], h, lse)
 
-        tp_bytes = 0
-        for b in range(M // c + 1):
-            ns = c if b < M // c else 1
-            tp_bytes += T * ((1 + b) * d * 2 + ns * (d * pb + 4))
-            tp_bytes += (ns - 1) * T * (d * pb + 4 + d * 2 + d * 2 + 4 + 2 * r)
+        tp_bytes = sites.block_two_phase_forward_bytes(T, d, r, c, M, pre_bytes=pb)
         tn = _median_ms(torch, naive, max(3, reps // 2))
         tt = _median_ms(torch, two_phase, max(3, reps // 2))
         emit({"suite": "Block S-LR forward sweep, 65 sites, d2048 r64 c8 T32768", "h_pre_bytes": pb,
@@ -685,7 +681,8 @@ def run_block_step(emit, dev, reps: int):
     """The Block AttnRes training step of the 32-layer, d = 2048 decoder
     (M = 64 sub-layer outputs, c = 8, S-LR r = 64, T = 32768, bf16 outputs, h
     and gradients) through sweep.BlockSweep: per step the assembly after each
-    sub-layer and the mix at each of the 65 sites (forward), then the backward
+    sub-layer and the two-phase mix of the 65 sites (forward: phase 1 per block,
+    phase 2 at each site after a block's first), then the backward
     at each site in reverse and the fan-out of the summary gradients to the
     members.  The outputs are written afresh before every step (untimed), as
     the sub-layers would; bytes of the mix and of the assembly / fan-out (a9)
@@ -703,7 +700,7 @@ def run_block_step(emit, dev, reps: int):
     h = torch.empty(M + 1, T, d, dtype=torch.bfloat16, device=dev)
     lse = torch.empty(M + 1, T, device=dev)
     douts = [torch.empty(T, d, dtype=torch.bfloat16, device=dev) for _ in range(M + 1)]
-    sw = BlockSweep("sliced", outs, qs, [dh[t] for t in range(M + 1)], h, lse, douts, c, r=r)
+    sw = BlockSweep("sliced", outs, qs, [dh[t] for t in range(M + 1)], h, lse, douts, c, r=r, two_phase=True)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
            torch.cuda.Event(enable_timing=True)) for _ in range(reps + 1)]
     for a, b, e in ev:
@@ -718,14 +715,14 @@ def run_block_step(emit, dev, reps: int):
     torch.cuda.synchronize()
     fwd = statistics.median(a.elapsed_time(b) for a, b, _ in ev[1:])
     bwd = statistics.median(b.elapsed_time(e) for _, b, e in ev[1:])
-    mix_f = mix_b = 0
+    mix_f = sites.block_two_phase_forward_bytes(T, d, r, c, M)  # bf16 h serves as h_pre
+    mix_b = 0
     for t in range(1, M + 2):
         shp = sites.SiteShape("sliced", sites.block_num_sources(t, c), T, d, r, accumulate=int(t != M + 1))
-        mix_f += sites.forward_bytes(shp)
         mix_b += sites.backward_bytes(shp)
     asm = sum(sites.block_accumulate_bytes(T, d, 2, True) for i in range(1, M + 1) if not sites.block_opens_slot(i, c))
     fan = (M + 1) * sites.block_accumulate_bytes(T, d, 2, False)
-    emit({"suite": "Block S-LR training step, 65 sites, d2048 r64 c8 T32768 (site by site)",
+    emit({"suite": "Block S-LR training step, 65 sites, d2048 r64 c8 T32768 (two-phase forward)",
           "fwd_ms": fwd, "bwd_ms": bwd, "step_ms": fwd + bwd, "mix_fwd_bytes": mix_f, "assembly_bytes": asm,
           "mix_bwd_bytes": mix_b, "fanout_bytes": fan, "fwd_gbs": (mix_f + asm) / fwd / 1e6,
           "bwd_gbs": (mix_b + fan) / bwd / 1e6, "step_gbs": (mix_f + asm + mix_b + fan) / (fwd + bwd) / 1e6,

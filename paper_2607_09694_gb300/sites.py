@@ -106,6 +106,22 @@ def backward_bytes(s: SiteShape) -> int:
     return s.T * per_tok
 
 
+def block_two_phase_forward_bytes(T: int, d: int, r: int, c: int, M: int, variant: str = "sliced",
+                                  in_bytes: int = 2, pre_bytes: int = 2, out_bytes: int = 2) -> int:
+    """Two-phase Block forward (§3.5) over sites t = 1..M+1 in blocks of c sites:
+    per block b, phase 1 reads the 1 + b completed sources (+ their P-LR keys)
+    and writes h_pre and lse_pre of each of the block's ns sites; phase 2, at
+    every site of the block after the first, reads h_pre, lse_pre and the
+    partial summary (+ its key) and writes h and lse."""
+    rp = r if variant == "projected" else 0
+    total = 0
+    for b in range(M // c + 1):
+        ns = min(c, M + 1 - b * c)
+        total += T * ((1 + b) * (d + rp) * in_bytes + ns * (d * pre_bytes + 4))
+        total += (ns - 1) * T * (d * pre_bytes + 4 + (d + rp) * in_bytes + d * out_bytes + 4)
+    return total
+
+
 def block_accumulate_bytes(T: int, width: int, elem_bytes: int, beta_nonzero: bool) -> int:
     """dst = beta*dst + alpha*src: read src (+ dst when beta != 0), write dst."""
     return T * width * elem_bytes * (3 if beta_nonzero else 2)

@@ -99,3 +99,30 @@ def test_byte_model_headline():
     s = sites.SiteShape("sliced", 49, 16384, 1024, 16)
     assert abs(sites.forward_bytes(s) / 1e9 - 1.678) < 1e-3
     assert abs(sites.backward_bytes(s) / 1e9 - 4.966) < 1e-3
+
+
+@pytest.mark.parametrize("variant,pre", [("sliced", 2), ("sliced", 4), ("projected", 2)])
+def test_two_phase_bytes_with_one_site_per_block(variant, pre):
+    """With c = 1 every block holds one site and has no phase 2: the two-phase
+    forward moves exactly the bytes of the per-site forwards over the same
+    source counts (h_pre is then the site's h)."""
+    T, d, r, M = 64, 256, 16, 7
+    per_site = sum(sites.forward_bytes(sites.SiteShape(variant, sites.block_num_sources(t, 1), T, d, r,
+                                                       out_bytes=pre)) for t in range(1, M + 2))
+    assert sites.block_two_phase_forward_bytes(T, d, r, 1, M, variant, pre_bytes=pre) == per_site
+
+
+def test_two_phase_bytes_of_the_large_decoder():
+    """The d = 2048 decoder (M = 64, c = 8, r = 64, T = 32768, bf16 h_pre): 8
+    blocks of 8 sites and the final read site alone.  Phase 1 reads sum(1 + b)
+    source rows per token over the 9 blocks and writes 65 h_pre rows; phase 2 runs
+    at 56 sites, each reading an h_pre row and a partial summary and writing h."""
+    T, d = 32768, 2048
+    row = d * 2
+    ph1 = T * (sum(1 + b for b in range(9)) * row + 65 * (row + 4))
+    ph2 = 56 * T * (row + 4 + row + row + 4)
+    assert sites.block_two_phase_forward_bytes(T, d, 64, 8, 64) == ph1 + ph2
+    # against the site-by-site forward of the same sites: 56.1 GB
+    naive = sum(sites.forward_bytes(sites.SiteShape("sliced", sites.block_num_sources(t, 8), T, d, 64))
+                for t in range(1, 66))
+    assert abs(naive / 1e9 - 56.11) < 0.01 and abs((ph1 + ph2) / 1e9 - 37.34) < 0.01
