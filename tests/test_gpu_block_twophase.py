@@ -109,18 +109,29 @@ def test_bf16_members_d2048(b):
         H.assert_abs(f"lse[site {j}]", lse, ref["lse"], 1e-4)
 
 
-@pytest.mark.parametrize("variant,r,c,b,T", [("sliced", 32, 8, 1, 333), ("sliced", 48, 5, 2, 333),
-                                               ("projected", 32, 8, 2, 333), ("projected", 16, 3, 4, 333),
-                                               ("sliced", 64, 8, 15, 333), ("sliced", 32, 8, 3, 20011)])
-def test_bf16_key_depths(variant, r, c, b, T):
+@pytest.mark.parametrize("variant,r,c,b,T,d", [("sliced", 32, 8, 1, 333, 256), ("sliced", 48, 5, 2, 333, 256),
+                                                 ("projected", 32, 8, 2, 333, 256), ("projected", 16, 3, 4, 333, 256),
+                                                 ("sliced", 64, 8, 15, 333, 256), ("sliced", 32, 8, 3, 20011, 256),
+                                                 ("projected", 48, 2, 30, 3001, 384)])
+def test_bf16_key_depths(variant, r, c, b, T, d):
     """bf16 sources with keys of depth 16, 32, 48 and 64 (the phase-1 scores on the
-    tensor cores, one to four k-steps), up to 16 completed sources, fewer than 8
-    sites, and a token count that leaves several tokens per warp and a ragged
-    last chunk (T = 20011).  Both sides mix the same bf16 sources, so h is held
-    to the fp32 bar."""
-    for j, (h, lse), ref, _ in _run(variant, c=c, b=b, T=T, d=256, r=r, store="bf16", stack="bf16", pre="f32",
+    tensor cores, one to four k-steps), up to 31 completed sources, fewer than 8
+    sites, and token counts that leave several tokens per warp and a ragged last
+    chunk (T = 20011; T = 3001 with 31 sources).  Both sides mix the same bf16
+    sources, so h is held to the fp32 bar."""
+    for j, (h, lse), ref, _ in _run(variant, c=c, b=b, T=T, d=d, r=r, store="bf16", stack="bf16", pre="f32",
                                     seed=19 + r + b):
         H.assert_abs(f"h[site {j}]", h, ref["h"])
+        H.assert_abs(f"lse[site {j}]", lse, ref["lse"], 1e-4)
+
+
+def test_weights_wider_than_an_h_pre_row():
+    """21 completed sources with a bf16 h_pre of d = 256: a token's 21 x 8 fp32
+    weights do not fit one h_pre row, so phase 1 runs as the single fused kernel."""
+    for j, (h, lse), ref, pre_ref in _run("sliced", c=4, b=20, T=333, d=256, r=16, store="bf16", stack="bf16",
+                                          pre="bf16", seed=23):
+        bound = 0.5 * H.bf16_ulp(pre_ref["h"]) + 1e-5 * H.rms(ref["h"])
+        assert np.all(np.abs(h - ref["h"]) <= bound), j
         H.assert_abs(f"lse[site {j}]", lse, ref["lse"], 1e-4)
 
 
