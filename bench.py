@@ -684,9 +684,10 @@ def run_block_step(emit, dev, reps: int):
     sub-layer and the two-phase mix of the 65 sites (forward: phase 1 per block,
     phase 2 at each site after a block's first), then the backward
     at each site in reverse and the fan-out of the summary gradients to the
-    members.  The outputs are written afresh before every step (untimed), as
-    the sub-layers would; bytes of the mix and of the assembly / fan-out (a9)
-    are reported separately."""
+    members, as copies into per-member tensors or handed over as views of the
+    slot accumulators (one line each).  The outputs are written afresh before
+    every step (untimed), as the sub-layers would; bytes of the mix and of the
+    assembly / fan-out (a9) are reported separately."""
     import torch
 
     from paper_2607_09694_gb300 import sites, synth
@@ -701,32 +702,34 @@ def run_block_step(emit, dev, reps: int):
     lse = torch.empty(M + 1, T, device=dev)
     douts = [torch.empty(T, d, dtype=torch.bfloat16, device=dev) for _ in range(M + 1)]
     sw = BlockSweep("sliced", outs, qs, [dh[t] for t in range(M + 1)], h, lse, douts, c, r=r, two_phase=True)
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
-           torch.cuda.Event(enable_timing=True)) for _ in range(reps + 1)]
-    for a, b, e in ev:
-        for i in range(M + 1):
-            outs[i].copy_(fresh[i])
-        sw.rearm()
-        a.record()
-        sw.forward()
-        b.record()
-        sw.backward()
-        e.record()
-    torch.cuda.synchronize()
-    fwd = statistics.median(a.elapsed_time(b) for a, b, _ in ev[1:])
-    bwd = statistics.median(b.elapsed_time(e) for _, b, e in ev[1:])
     mix_f = sites.block_two_phase_forward_bytes(T, d, r, c, M)  # bf16 h serves as h_pre
     mix_b = 0
     for t in range(1, M + 2):
         shp = sites.SiteShape("sliced", sites.block_num_sources(t, c), T, d, r, accumulate=int(t != M + 1))
         mix_b += sites.backward_bytes(shp)
     asm = sum(sites.block_accumulate_bytes(T, d, 2, True) for i in range(1, M + 1) if not sites.block_opens_slot(i, c))
-    fan = (M + 1) * sites.block_accumulate_bytes(T, d, 2, False)
-    emit({"suite": "Block S-LR training step, 65 sites, d2048 r64 c8 T32768 (two-phase forward)",
-          "fwd_ms": fwd, "bwd_ms": bwd, "step_ms": fwd + bwd, "mix_fwd_bytes": mix_f, "assembly_bytes": asm,
-          "mix_bwd_bytes": mix_b, "fanout_bytes": fan, "fwd_gbs": (mix_f + asm) / fwd / 1e6,
-          "bwd_gbs": (mix_b + fan) / bwd / 1e6, "step_gbs": (mix_f + asm + mix_b + fan) / (fwd + bwd) / 1e6,
-          "tokens_per_s_per_site": T * (M + 1) / ((fwd + bwd) / 1e3)})
+    # the fan-out as copies into doutputs, or handed over as views (member_grad)
+    for mode, hand_over in (("fan-out copies", None), ("member gradients handed over", lambda i, g, gk: None)):
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+               torch.cuda.Event(enable_timing=True)) for _ in range(reps + 1)]
+        for a, b, e in ev:
+            for i in range(M + 1):
+                outs[i].copy_(fresh[i])
+            sw.rearm()
+            a.record()
+            sw.forward()
+            b.record()
+            sw.backward(member_grad=hand_over)
+            e.record()
+        torch.cuda.synchronize()
+        fwd = statistics.median(a.elapsed_time(b) for a, b, _ in ev[1:])
+        bwd = statistics.median(b.elapsed_time(e) for _, b, e in ev[1:])
+        fan = 0 if hand_over else (M + 1) * sites.block_accumulate_bytes(T, d, 2, False)
+        emit({"suite": f"Block S-LR training step, 65 sites, d2048 r64 c8 T32768 (two-phase forward, {mode})",
+              "fwd_ms": fwd, "bwd_ms": bwd, "step_ms": fwd + bwd, "mix_fwd_bytes": mix_f, "assembly_bytes": asm,
+              "mix_bwd_bytes": mix_b, "fanout_bytes": fan, "fwd_gbs": (mix_f + asm) / fwd / 1e6,
+              "bwd_gbs": (mix_b + fan) / bwd / 1e6, "step_gbs": (mix_f + asm + mix_b + fan) / (fwd + bwd) / 1e6,
+              "tokens_per_s_per_site": T * (M + 1) / ((fwd + bwd) / 1e3)})
     del fresh, outs, dh, h, douts, sw
     torch.cuda.empty_cache()
 

@@ -225,12 +225,22 @@ class BlockSweep:
                                   stream=s.cuda_stream)
 
     # backward ----------------------------------------------------------------
-    def backward(self, stream: torch.cuda.Stream | None = None) -> None:
+    def backward(self, stream: torch.cuda.Stream | None = None, member_grad=None) -> None:
         """Sites in reverse: site t adds the gradients of its sources into the
         accumulators of their slots (site M+1 writes them); right after site
         i+1, the accumulator of o_i's slot holds the whole gradient of o_i
         (every later site reads o_i through that slot), so it is copied to
-        doutputs[i] -- the fan-out of the summary gradients to the members."""
+        doutputs[i] -- the fan-out of the summary gradients to the members.
+
+        member_grad: optional callable(i, dout, dkey), the fan-out as a
+        hand-over instead of copies.  It is called as soon as o_i's gradient is
+        complete, with views of the slot accumulators that hold it (dkey: the
+        key gradient with P-LR keys, else None), and inside the stream's
+        context.  The views keep d o_i until the next site's backward, which is
+        enqueued after the call returns, so work that the callable enqueues on
+        the stream reads them in time: in a training step, the backward of the
+        sub-layer that wrote o_i.  doutputs and dkeys are then left untouched,
+        and the step moves no fan-out bytes."""
         s = stream or torch.cuda.current_stream()
         with torch.cuda.stream(s):
             self.dq.zero_()
@@ -247,6 +257,10 @@ class BlockSweep:
                                stream=s.cuda_stream)
             i = t - 1  # o_{t-1} is read by sites t..M+1 only: its gradient is complete
             b = self._slot(i)
+            if member_grad is not None:
+                with torch.cuda.stream(s):
+                    member_grad(i, self.grads[b], self.dkgrads[b] if self.keys is not None else None)
+                continue
             lrar.block_accumulate(self.doutputs[i], self.grads[b], 1.0, 0.0, stream=s.cuda_stream)
             if self.keys is not None:
                 lrar.block_accumulate(self.dkeys[i], self.dkgrads[b], 1.0, 0.0, stream=s.cuda_stream)
@@ -256,6 +270,6 @@ class BlockSweep:
         output tensors: the next forward assembles them again."""
         self.assembled = False
 
-    def step(self, stream: torch.cuda.Stream | None = None) -> None:
+    def step(self, stream: torch.cuda.Stream | None = None, member_grad=None) -> None:
         self.forward(stream)
-        self.backward(stream)
+        self.backward(stream, member_grad)

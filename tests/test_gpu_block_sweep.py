@@ -138,6 +138,42 @@ def test_block_step_bf16_decoder_shape():
         H.assert_rms(f"doutputs[{i}]", got[i], douts[i])
 
 
+@pytest.mark.parametrize("variant", ["sliced", "projected"])
+def test_member_gradients_handed_over(variant):
+    """The fan-out as a hand-over: the views passed to member_grad as each
+    output's gradient completes, copied there on the stream, equal bit for bit
+    the doutputs (and dkeys) that the copying fan-out writes; doutputs stay
+    untouched."""
+    M, c, T, d, r = 13, 4, 96, 128, 8
+    outs, keys, queries, dh = _inputs(variant, M, T, d, r, "f32", seed=64)
+    ref = _run(variant, outs, keys, queries, dh, c, r)
+    dev = torch.device("cuda")
+    o = [outs[i].to(dev).clone() for i in range(M + 1)]
+    k = [keys[i].to(dev).clone() for i in range(M + 1)] if keys is not None else None
+    h = torch.empty(M + 1, T, d, device=dev)
+    lse = torch.empty(M + 1, T, device=dev)
+    do = [torch.full((T, d), float("nan"), device=dev) for _ in range(M + 1)]
+    dk = [torch.full((T, r), float("nan"), device=dev) for _ in range(M + 1)] if k is not None else None
+    sw = BlockSweep(variant, o, queries.to(dev), [dh[t].to(dev) for t in range(M + 1)], h, lse, do, c, keys=k,
+                    dkeys=dk, r=r)
+    got, got_k, order = {}, {}, []
+
+    def take(i, g, gk):
+        order.append(i)
+        got[i] = g.clone()
+        if gk is not None:
+            got_k[i] = gk.clone()
+
+    sw.step(member_grad=take)
+    torch.cuda.synchronize()
+    assert order == list(range(M, -1, -1))
+    for i in range(M + 1):
+        assert torch.equal(got[i], ref.doutputs[i]), i
+        assert torch.isnan(do[i]).all(), i
+        if keys is not None:
+            assert torch.equal(got_k[i], ref.dkeys[i]), i
+
+
 def test_forward_runs_once_per_set_of_outputs():
     outs, _, queries, dh = _inputs("sliced", 4, 16, 64, 4, "f32", seed=63)
     sw = _run("sliced", outs, None, queries, dh, 2, 4)
