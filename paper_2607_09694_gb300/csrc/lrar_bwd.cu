@@ -956,7 +956,8 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_slr_onepass_kernel(const __gr
             }
             const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
             const float s = __shfl_sync(0xffffffffu, rho * qk, lead);
-            const float a = expf(s - lse);
+            // one source weighs exactly 1 (a softmax over one score), however s rounds against lse
+            const float a = p.n == 1 ? 1.f : expf(s - lse);
             asum += a;
             T *drow = dst_row<T>(p.dvt, i, x, p.d);
 #pragma unroll
@@ -1058,7 +1059,7 @@ inline size_t onepass_acc_smem(int S, int V, int n, int r, int nv) {
 }
 
 template <typename T, int V, int S>
-__global__ void __launch_bounds__(kThreads, 2) bwd_slr_onepass_acc_kernel(const __grid_constant__ BwdParams p) {
+__global__ void __launch_bounds__(kThreads, V >= 8 ? 1 : 2) bwd_slr_onepass_acc_kernel(const __grid_constant__ BwdParams p) {
     pdl_enter();
     constexpr int E = VecE<T>::value;
     constexpr int P = 2;
@@ -1172,7 +1173,8 @@ __global__ void __launch_bounds__(kThreads, 2) bwd_slr_onepass_acc_kernel(const 
             }
             const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
             const float s = __shfl_sync(0xffffffffu, rho * qk, lead);
-            const float a = expf(s - lse);
+            // one source weighs exactly 1 (a softmax over one score), however s rounds against lse
+            const float a = p.n == 1 ? 1.f : expf(s - lse);
             asum += a;
             T *drow = dst_row<T>(p.dvt, i, x, p.d);
 #pragma unroll
@@ -1425,29 +1427,36 @@ static cudaError_t launch_bwd_t(const BwdArgs &a, cudaStream_t s) {
     size_t smem;
     int rq;
     constexpr bool kPipe = LRAR_BWD_PIPE && std::is_same<Tin, Tg>::value;
-    // Sliced keys with the forward's lse, gradients written (not accumulated):
-    // one pass over the values when the slice is whole vectors forming an
-    // aligned lane group (r / E divides 32, r divides d) and the per-warp stash
-    // fits in shared memory.  The accumulating form of the same kernel
-    // (ACC = true, equally exact) measured 2-3 % slower than the routing + value
-    // pass + key pass kernel at n = 49 on GB300 (one CTA per SM against two),
-    // so accumulating calls take bwd_lr_pipe_kernel.
-    if constexpr (kPipe && V <= 4) {
+    // Sliced keys with the forward's lse: one pass over the values when the
+    // slice is whole vectors forming an aligned lane group (r / E divides 32,
+    // r divides d) and the per-warp stash fits in shared memory -- the
+    // fixed-shape kernel at (d, r) = (1024, 16), else bwd_slr_onepass_acc_kernel
+    // (accumulating) or bwd_slr_onepass_kernel (writing).  Other calls take the
+    // routing + value pass + key pass kernel (bwd_lr_pipe_kernel).
+    if constexpr (kPipe) {
         bool launched = false;
         cudaError_t ef = launch_bwd_fixed(p, a, launched, s);
         if (ef != cudaSuccess || launched) return ef;
         constexpr int OSN = OnePassStages<V, false>::value;
         const int nvk = a.r / E;
-        // accumulating: the one-pass kernel at two CTAs per SM when it fits
+        // accumulating: the one-pass kernel when it fits two CTAs per SM (one at
+        // eight vectors per lane, where the other kernels run one CTA per SM too).
+        // At eight vectors per lane (d = 2048) it wins at few sources and loses
+        // at many (fraction of the copy peak, one-pass against routing + value
+        // pass + key pass: n = 2: 0.82 / 0.65, n = 5: 0.94 / 0.84, n = 9: 0.97 /
+        // 0.96, n = 17: 0.96 / 0.99), so there it serves n <= 9.
+        constexpr int kAccMaxSources = V >= 8 ? 9 : kMaxSources;
         if (a.variant == kSliced && a.lse && a.accumulate && p.key_vec && nvk >= 1 && nvk <= 32 && 32 % nvk == 0 &&
-            a.d % a.r == 0) {
+            a.d % a.r == 0 && a.n <= kAccMaxSources) {
             constexpr int OSA = 3;
             const size_t smem2 = onepass_acc_smem(OSA, V, a.n, a.r, nvk);
             const void *k2 = (const void *)bwd_slr_onepass_acc_kernel<Tin, V, OSA>;
-            int dev = 0, per_sm = 0;
+            int dev = 0, per_sm = 0, optin = 0;
             cudaGetDevice(&dev);
             cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
-            if (2 * (smem2 + 1024) <= (size_t)per_sm) {  // two CTAs per SM (1 KB reserved per CTA)
+            cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+            constexpr int kCtas = V >= 8 ? 1 : 2;  // CTAs per SM (1 KB reserved per CTA)
+            if (kCtas * (smem2 + 1024) <= (size_t)per_sm && smem2 <= (size_t)optin) {
                 cudaError_t e = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
                 if (e != cudaSuccess) return e;
                 const int grid = persistent_grid(k2, kThreads, smem2, work, kMaxPartials);

@@ -162,7 +162,8 @@ __global__ void __launch_bounds__(kThreads, 2) bwd_slr_fixed_kernel(const __grid
             }
             const float rho = rsqrtf(fmaf(ss, p.inv_r, p.eps));
             const float s = __shfl_sync(0xffffffffu, rho * qk, LEAD);
-            const float a = expf(s - lse);
+            // one source weighs exactly 1 (a softmax over one score), however s rounds against lse
+            const float a = p.n == 1 ? 1.f : expf(s - lse);
             asum += a;
             bf16 *drow = static_cast<bf16 *>(const_cast<void *>(p.dvt.p[i])) + x * D + lane * E;
 #pragma unroll

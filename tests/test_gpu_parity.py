@@ -199,6 +199,19 @@ def test_sliced_one_pass_shapes(n, d, r):
     _check(si, H.run_gpu(si, "bf16", "bf16"), H.run_oracle(si), si.n, "ulp")
 
 
+@pytest.mark.parametrize("n,d", [(1, 2048), (2, 2048), (5, 2048), (9, 2048), (10, 2048), (4, 1536)])
+@pytest.mark.parametrize("accumulate", [False, True])
+def test_sliced_one_pass_eight_vectors(n, d, accumulate):
+    """The one-pass sliced backward at eight vectors per lane (r = 64 at
+    d = 2048, the Block decoder's shape, and d = 1536, whose rows leave lanes'
+    vectors empty), one CTA per SM: accumulating up to 9 sources (10 take the
+    routing + value pass + key pass kernel), writing wherever the stash fits."""
+    si = synth.site("slr", n=n, T=150, d=d, r=64)
+    init = _init(si, dtype=torch.bfloat16) if accumulate else None
+    got = H.run_gpu(si, "bf16", "bf16", accumulate=accumulate, init=init)
+    _check(si, got, H.run_oracle(si), si.n, "ulp", init=init)
+
+
 @pytest.mark.parametrize("r", [1, 4, 8, 16, 64])
 def test_projected_key_widths(r):
     si = synth.site("plr", n=12, T=260, r=r)
