@@ -708,6 +708,8 @@ def run_block_step(emit, dev, reps: int):
         shp = sites.SiteShape("sliced", sites.block_num_sources(t, c), T, d, r, accumulate=int(t != M + 1))
         mix_b += sites.backward_bytes(shp)
     asm = sum(sites.block_accumulate_bytes(T, d, 2, True) for i in range(1, M + 1) if not sites.block_opens_slot(i, c))
+    # where a member joins its running sum inside phase 2, the partial summary is not read a second time
+    asm -= sites.block_phase2_assembled_sites(M, c) * T * d * 2
     # the fan-out as copies into doutputs, or handed over as views (member_grad)
     for mode, hand_over in (("fan-out copies", None), ("member gradients handed over", lambda i, g, gk: None)):
         ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),

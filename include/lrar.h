@@ -252,6 +252,27 @@ int lrar_block_phase1_ptrs(int variant, int in_dtype, int pre_dtype, const void 
 int lrar_block_phase2(int variant, int in_dtype, int pre_dtype, int out_dtype, const void *h_pre,
                       const float *lse_pre, const void *partial, const void *partial_key, const float *query,
                       int64_t T, int d, int r, float eps, void *h, float *lse, void *stream);
+/* Phase 2 that also assembles the partial summary it reads (Eq. 6): with the
+ * open block's running sum through the previous member, prev_partial, and the
+ * newest member's output, member, the partial summary is b = prev_partial +
+ * member (float32 sum rounded once to in_dtype, bit for bit the result of
+ * lrar_block_accumulate(member, prev_partial, alpha = beta = 1)).  b is written
+ * over member, and the site's h and lse are those of lrar_block_phase2 with
+ * partial = b.  For LRAR_PROJECTED, member_key is likewise replaced by
+ * prev_partial_key + member_key.  The accumulate + phase-2 pair it replaces
+ * reads b twice; this call reads its two terms once.
+ *   prev_partial      [T, d] in_dtype, read
+ *   member            [T, d] in_dtype, read and overwritten with b
+ *   prev_partial_key  [T, r] in_dtype (LRAR_PROJECTED), read; else ignored
+ *   member_key        [T, r] in_dtype (LRAR_PROJECTED), read and overwritten; else ignored
+ * member (and member_key) must not overlap prev_partial, h_pre or h.
+ * Everything else, and the errors, as lrar_block_phase2; prev_partial (and,
+ * for LRAR_PROJECTED, prev_partial_key) NULL with T > 0 is LRAR_ERR_INVALID_ARG.
+ */
+int lrar_block_phase2_assemble(int variant, int in_dtype, int pre_dtype, int out_dtype, const void *h_pre,
+                               const float *lse_pre, const void *prev_partial, void *member,
+                               const void *prev_partial_key, void *member_key, const float *query, int64_t T,
+                               int d, int r, float eps, void *h, float *lse, void *stream);
 
 /*
  * Routing diagnostics of one site (§4.5-4.6): the effective number of sources

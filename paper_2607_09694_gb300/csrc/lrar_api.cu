@@ -489,10 +489,47 @@ LRAR_API int lrar_test_block_phase1_stalled(int variant, int in_dtype, int pre_d
                              r, eps, h_pre, lse_pre, status, wait_cycles, true, stream);
 }
 
+namespace {
+
+int block_phase2_impl(int variant, int in_dtype, int pre_dtype, int out_dtype, const void *h_pre,
+                      const float *lse_pre, const void *prev, const void *partial, const void *prev_key,
+                      const void *partial_key, const float *query, int64_t T, int d, int r, float eps, void *h,
+                      float *lse, void *stream, const char *name);
+
+}  // namespace
+
 LRAR_API int lrar_block_phase2(int variant, int in_dtype, int pre_dtype, int out_dtype, const void *h_pre,
                                const float *lse_pre, const void *partial, const void *partial_key,
                                const float *query, int64_t T, int d, int r, float eps, void *h, float *lse,
                                void *stream) {
+    return block_phase2_impl(variant, in_dtype, pre_dtype, out_dtype, h_pre, lse_pre, nullptr, partial, nullptr,
+                             partial_key, query, T, d, r, eps, h, lse, stream, "lrar_block_phase2");
+}
+
+LRAR_API int lrar_block_phase2_assemble(int variant, int in_dtype, int pre_dtype, int out_dtype, const void *h_pre,
+                                        const float *lse_pre, const void *prev_partial, void *member,
+                                        const void *prev_partial_key, void *member_key, const float *query,
+                                        int64_t T, int d, int r, float eps, void *h, float *lse, void *stream) {
+    if (variant == LRAR_FULL)
+        return fail(LRAR_ERR_UNSUPPORTED, "the two-phase block path serves low-rank keys (sliced, projected)");
+    if (T > 0 && !prev_partial) return fail(LRAR_ERR_INVALID_ARG, "prev_partial is required");
+    if (T > 0 && variant == LRAR_PROJECTED && !prev_partial_key)
+        return fail(LRAR_ERR_INVALID_ARG, "the previous partial summary's projected key is required");
+    if (prev_partial && !aligned16(prev_partial))
+        return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (lse, query and keys 4-byte)");
+    if (variant == LRAR_PROJECTED && prev_partial_key && !aligned4(prev_partial_key))
+        return fail(LRAR_ERR_ALIGNMENT, "tensors must be 16-byte aligned (lse, query and keys 4-byte)");
+    return block_phase2_impl(variant, in_dtype, pre_dtype, out_dtype, h_pre, lse_pre, prev_partial, member,
+                             variant == LRAR_PROJECTED ? prev_partial_key : nullptr, member_key, query, T, d, r,
+                             eps, h, lse, stream, "lrar_block_phase2_assemble");
+}
+
+namespace {
+
+int block_phase2_impl(int variant, int in_dtype, int pre_dtype, int out_dtype, const void *h_pre,
+                      const float *lse_pre, const void *prev, const void *partial, const void *prev_key,
+                      const void *partial_key, const float *query, int64_t T, int d, int r, float eps, void *h,
+                      float *lse, void *stream, const char *name) {
     if (variant == LRAR_FULL)
         return fail(LRAR_ERR_UNSUPPORTED, "the two-phase block path serves low-rank keys (sliced, projected)");
     int rc = check_shape(variant, in_dtype, 1, T, d, r, eps);
@@ -515,6 +552,8 @@ LRAR_API int lrar_block_phase2(int variant, int in_dtype, int pre_dtype, int out
     a.lse_pre = lse_pre;
     a.partial = partial;
     a.pkeys = variant == LRAR_PROJECTED ? partial_key : nullptr;
+    a.prev = prev;
+    a.prev_keys = variant == LRAR_PROJECTED ? prev_key : nullptr;
     a.query = query;
     a.T = T;
     a.d = d;
@@ -523,9 +562,11 @@ LRAR_API int lrar_block_phase2(int variant, int in_dtype, int pre_dtype, int out
     a.h = h;
     a.lse = lse;
     cudaError_t e = lrar::launch_block_phase2(a, static_cast<cudaStream_t>(stream));
-    if (e != cudaSuccess) return cuda_fail(e, "lrar_block_phase2");
+    if (e != cudaSuccess) return cuda_fail(e, name);
     return LRAR_OK;
 }
+
+}  // namespace
 
 namespace {
 

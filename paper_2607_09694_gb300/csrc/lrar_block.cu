@@ -882,6 +882,8 @@ __global__ void __launch_bounds__(kThreads, 2) block_mix_kernel(const __grid_con
 
 struct Ph2Params {
     const void *h_pre, *partial, *pkeys;
+    const void *prev, *prev_keys;  // assembling: the running sum before the member (then partial / pkeys are
+                                   // the member's output / key, replaced by the sum)
     const float *lse_pre, *query;
     void *h;
     float *lse;
@@ -894,6 +896,10 @@ struct Ph2Params {
 // Phase 2: one warp per token merges h_pre with the partial-block summary.
 // Each lane reads its elements of h_pre (and lane 0 lse_pre) before it writes
 // the same elements of h (and lse), so h may be h_pre and lse may be lse_pre.
+// Assembling (p.prev set), the partial summary is first formed from the
+// running sum before the newest member and that member's output (Eq. 6): the
+// fp32 sum rounded once to the stack type, as lrar_block_accumulate forms it,
+// written over the member and used as read back.
 template <typename Tin, typename Tp, typename Tout, int V>
 __global__ void __launch_bounds__(kThreads) block_phase2_kernel(const Ph2Params p) {
     pdl_enter();
@@ -908,15 +914,45 @@ __global__ void __launch_bounds__(kThreads) block_phase2_kernel(const Ph2Params 
         // both rows first: their loads travel while the partial summary is scored
         Frag<Tin, E> fb[V];
         Frag<Tp, E> fh[V];
+        if (p.prev) {
+            Frag<Tin, E> fp[V];
 #pragma unroll
-        for (int v = 0; v < V; ++v) {
-            const int e = (lane + 32 * v) * E;
-            if (e < p.d) {
-                fb[v].load_nc(part + x * p.d + e);
-                fh[v].load(h_pre + x * p.d + e);  // coherent: h may be h_pre (in place)
-            } else {
-                fb[v].zero();
-                fh[v].zero();
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) {
+                    fb[v].load(part + x * p.d + e);  // coherent: the member row is rewritten below
+                    fp[v].load_nc(static_cast<const Tin *>(p.prev) + x * p.d + e);
+                    fh[v].load(h_pre + x * p.d + e);
+                } else {
+                    fb[v].zero();
+                    fp[v].zero();
+                    fh[v].zero();
+                }
+            }
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) {
+                    float m[E], b[E];
+                    fb[v].get(m);
+                    fp[v].get(b);
+#pragma unroll
+                    for (int t = 0; t < E; ++t) b[t] += m[t];
+                    fb[v].set(b);  // rounded once: the partial summary as stored
+                    fb[v].store(const_cast<Tin *>(part) + x * p.d + e);
+                }
+            }
+        } else {
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                const int e = (lane + 32 * v) * E;
+                if (e < p.d) {
+                    fb[v].load_nc(part + x * p.d + e);
+                    fh[v].load(h_pre + x * p.d + e);  // coherent: h may be h_pre (in place)
+                } else {
+                    fb[v].zero();
+                    fh[v].zero();
+                }
             }
         }
         // score of the partial summary, Eq. (8)-(9); an S-LR key is the tail of
@@ -937,6 +973,16 @@ __global__ void __launch_bounds__(kThreads) block_phase2_kernel(const Ph2Params 
                             qk = fmaf(__ldg(p.query + (e + t - k0)), b[t], qk);
                         }
                 }
+            }
+        } else if (p.prev_keys) {
+            Tin *kp = const_cast<Tin *>(pkeys) + x * p.r;
+            const Tin *pp = static_cast<const Tin *>(p.prev_keys) + x * p.r;
+            for (int j = lane; j < p.r; j += 32) {
+                const Tin kr = from_f<Tin>(to_f(pp[j]) + to_f(kp[j]));
+                kp[j] = kr;
+                const float k = to_f(kr);
+                ss = fmaf(k, k, ss);
+                qk = fmaf(__ldg(p.query + j), k, qk);
             }
         } else {
             const Tin *kp = pkeys + x * p.r;
@@ -1130,6 +1176,8 @@ static cudaError_t launch_ph2_t(const BlockPh2Args &a, cudaStream_t s) {
     p.h_pre = a.h_pre;
     p.partial = a.partial;
     p.pkeys = a.pkeys;
+    p.prev = a.prev;
+    p.prev_keys = a.prev_keys;
     p.lse_pre = a.lse_pre;
     p.query = a.query;
     p.h = a.h;

@@ -79,8 +79,10 @@ struct BlockPh2Args {
     int variant, in_dtype, pre_dtype, out_dtype;
     const void *h_pre;     // [T, d] of one site
     const float *lse_pre;  // [T]
-    const void *partial;   // partial-block summary [T, d]
-    const void *pkeys;     // its P-LR key [T, r]
+    const void *partial;   // partial-block summary [T, d] (assembling: the newest member's output, replaced by it)
+    const void *pkeys;     // its P-LR key [T, r] (likewise)
+    const void *prev = nullptr;       // assembling: the running sum before the member [T, d], else null
+    const void *prev_keys = nullptr;  // and its P-LR key [T, r]
     const float *query;    // [r]
     int64_t T;
     int d, r;

@@ -28,7 +28,7 @@ LIB_PATH = os.path.join(_PKG, "liblrar.so")
 EXPORTS = ("lrar_forward", "lrar_backward", "lrar_backward_workspace_size", "lrar_block_accumulate",
            "lrar_strerror", "lrar_last_error", "lrar_version", "lrar_backward_noalloc", "lrar_diagnostics",
            "lrar_diagnostics_workspace_size", "lrar_block_phase1", "lrar_block_phase2", "lrar_project",
-           "lrar_forward_ptrs", "lrar_backward_ptrs", "lrar_block_phase1_ptrs")
+           "lrar_forward_ptrs", "lrar_backward_ptrs", "lrar_block_phase1_ptrs", "lrar_block_phase2_assemble")
 TEST_HOOKS = ("lrar_test_project_tile", "lrar_test_block_phase1_stalled")  # include/lrar_testing.h
 MAX_BLOCK_SITES = 64
 
@@ -72,6 +72,9 @@ def load(path: str | None = None):
         lib.lrar_test_project_tile.restype = i
         lib.lrar_block_phase2.argtypes = [i, i, i, i, vp, vp, vp, vp, vp, i64, i, i, f32, vp, vp, vp]
         lib.lrar_block_phase2.restype = i
+        lib.lrar_block_phase2_assemble.argtypes = [i, i, i, i, vp, vp, vp, vp, vp, vp, vp, i64, i, i, f32, vp, vp,
+                                                   vp]
+        lib.lrar_block_phase2_assemble.restype = i
         lib.lrar_diagnostics.argtypes = [i, i, vp, vp, vp, i, i64, i, i, f32, vp, vp, vp, sz, vp]
         lib.lrar_diagnostics.restype = i
         lib.lrar_diagnostics_workspace_size.argtypes = [i]
@@ -273,6 +276,21 @@ def block_phase2(variant, h_pre: torch.Tensor, lse_pre: torch.Tensor, partial: t
     _check(load().lrar_block_phase2(variant, dtype_code(partial), dtype_code(h_pre), dtype_code(h), _ptr(h_pre),
                                     _ptr(lse_pre), _ptr(partial), _ptr(partial_key), _ptr(query), T, d, r, eps,
                                     _ptr(h), _ptr(lse), _stream(stream)))
+
+
+def block_phase2_assemble(variant, h_pre: torch.Tensor, lse_pre: torch.Tensor, prev_partial: torch.Tensor,
+                          member: torch.Tensor, prev_partial_key: torch.Tensor | None, member_key: torch.Tensor | None,
+                          query: torch.Tensor, h: torch.Tensor, lse: torch.Tensor | None = None,
+                          eps: float = DEFAULT_EPS, stream=None) -> None:
+    """lrar_block_phase2_assemble: member := prev_partial + member (the partial
+    summary, Eq. 6; keys likewise for P-LR), then the site's mix as block_phase2."""
+    variant = _variant(variant)
+    T, d = member.shape
+    r = query.numel()
+    _check(load().lrar_block_phase2_assemble(variant, dtype_code(member), dtype_code(h_pre), dtype_code(h),
+                                             _ptr(h_pre), _ptr(lse_pre), _ptr(prev_partial), _ptr(member),
+                                             _ptr(prev_partial_key), _ptr(member_key), _ptr(query), T, d, r, eps,
+                                             _ptr(h), _ptr(lse), _stream(stream)))
 
 
 def diagnostics(variant, values: torch.Tensor, keys: torch.Tensor | None, query: torch.Tensor | None,

@@ -122,6 +122,13 @@ def block_two_phase_forward_bytes(T: int, d: int, r: int, c: int, M: int, varian
     return total
 
 
+def block_phase2_assembled_sites(M: int, c: int) -> int:
+    """Sites of the two-phase forward whose partial summary is assembled inside
+    phase 2 (lrar_block_phase2_assemble): every site of a block after its second,
+    where the newest member joins a running sum of at least one member."""
+    return sum(max(0, min(c, M + 1 - b * c) - 2) for b in range(M // c + 1))
+
+
 def block_accumulate_bytes(T: int, width: int, elem_bytes: int, beta_nonzero: bool) -> int:
     """dst = beta*dst + alpha*src: read src (+ dst when beta != 0), write dst."""
     return T * width * elem_bytes * (3 if beta_nonzero else 2)

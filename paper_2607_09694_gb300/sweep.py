@@ -218,11 +218,17 @@ class BlockSweep:
                                    self.lse[t0 - 1:t0 - 1 + ns], eps=self.eps, stream=s.cuda_stream)
             for j in range(1, ns):
                 t = t0 + j
-                self._assemble(t - 1, s)  # the partial summary through o_{t-1}
-                pk = self.keys[t - 1] if self.keys is not None else None
-                lrar.block_phase2(self.variant, self.h[t - 1], self.lse[t - 1], self.outputs[t - 1], pk,
-                                  self.queries[t - 1], self.h[t - 1], self.lse[t - 1], eps=self.eps,
-                                  stream=s.cuda_stream)
+                i = t - 1  # the partial summary runs through o_i
+                pk = self.keys[i] if self.keys is not None else None
+                if sites.block_opens_slot(i, c):  # o_i alone
+                    lrar.block_phase2(self.variant, self.h[t - 1], self.lse[t - 1], self.outputs[i], pk,
+                                      self.queries[t - 1], self.h[t - 1], self.lse[t - 1], eps=self.eps,
+                                      stream=s.cuda_stream)
+                else:  # o_i joins its block's running sum inside phase 2 (no separate assembly pass)
+                    ppk = self.keys[i - 1] if self.keys is not None else None
+                    lrar.block_phase2_assemble(self.variant, self.h[t - 1], self.lse[t - 1], self.outputs[i - 1],
+                                               self.outputs[i], ppk, pk, self.queries[t - 1], self.h[t - 1],
+                                               self.lse[t - 1], eps=self.eps, stream=s.cuda_stream)
 
     # backward ----------------------------------------------------------------
     def backward(self, stream: torch.cuda.Stream | None = None, member_grad=None) -> None:

@@ -319,3 +319,40 @@ def test_test_hooks_reject(lib):
     assert s(*args, None, 1000, None) == lrar.ERR_INVALID_ARG      # status required
     assert s(*args, FAKE, 0, None) == lrar.ERR_INVALID_ARG         # wait bound
     assert s(*args[:9], 64, 7, EPS, FAKE, FAKE, FAKE, 1000, None) == lrar.ERR_UNSUPPORTED  # r = 7: no staging
+
+
+def test_block_phase2_rejects(lib):
+    """Both phase-2 entries check their arguments before any device work."""
+    p2 = lib.lrar_block_phase2
+    args = [1, 1, 1, 1, FAKE, FAKE, FAKE, None, FAKE, 16, 64, 8, EPS, FAKE, FAKE]
+    assert p2(0, *args[1:], None) == lrar.ERR_UNSUPPORTED                         # full keys
+    bad = list(args)
+    bad[6] = None
+    assert p2(*bad, None) == lrar.ERR_INVALID_ARG                                 # partial
+    bad = list(args)
+    bad[6] = FAKE + 4
+    assert p2(*bad, None) == lrar.ERR_ALIGNMENT                                   # partial alignment
+    bad = list(args)
+    bad[9] = 0
+    bad[6] = None
+    assert p2(*bad, None) == lrar.OK                                              # T == 0
+    pa = lib.lrar_block_phase2_assemble
+    args = [1, 1, 1, 1, FAKE, FAKE, FAKE, FAKE, None, None, FAKE, 16, 64, 8, EPS, FAKE, FAKE]
+    assert pa(0, *args[1:], None) == lrar.ERR_UNSUPPORTED                         # full keys
+    bad = list(args)
+    bad[6] = None
+    assert pa(*bad, None) == lrar.ERR_INVALID_ARG                                 # prev_partial
+    assert b"prev_partial" in lib.lrar_last_error()
+    bad = list(args)
+    bad[6] = FAKE + 4
+    assert pa(*bad, None) == lrar.ERR_ALIGNMENT                                   # prev_partial alignment
+    bad = list(args)
+    bad[7] = None
+    assert pa(*bad, None) == lrar.ERR_INVALID_ARG                                 # member
+    proj = [2] + args[1:]
+    proj[9] = FAKE
+    assert pa(*proj, None) == lrar.ERR_INVALID_ARG                                # projected: prev key
+    bad = list(args)
+    bad[11] = 0
+    bad[6] = bad[7] = None
+    assert pa(*bad, None) == lrar.OK                                              # T == 0

@@ -126,3 +126,18 @@ def test_two_phase_bytes_of_the_large_decoder():
     naive = sum(sites.forward_bytes(sites.SiteShape("sliced", sites.block_num_sources(t, 8), T, d, 64))
                 for t in range(1, 66))
     assert abs(naive / 1e9 - 56.11) < 0.01 and abs((ph1 + ph2) / 1e9 - 37.34) < 0.01
+
+
+@pytest.mark.parametrize("M,c,expect", [(64, 8, 48), (13, 4, 6), (7, 1, 0), (12, 4, 6), (5, 8, 4)])
+def test_sites_assembled_inside_phase2(M, c, expect):
+    """Blocks of ns sites fold the assembly of members 2..ns-1 of the open block
+    into phase 2: M = 64, c = 8 has eight full blocks of 8 sites (6 each) and a
+    final block of one; M = 5, c = 8 one block of 6 sites."""
+    assert sites.block_phase2_assembled_sites(M, c) == expect
+    brute = 0
+    for b in range(M // c + 1):
+        t0 = b * c + 1
+        for t in range(t0 + 1, min(t0 + c, M + 2)):
+            i = t - 1
+            brute += int(not sites.block_opens_slot(i, c))
+    assert brute == expect

@@ -196,3 +196,39 @@ def test_phase1_status_stays_clear():
                       status=status)
     torch.cuda.synchronize()
     assert status.item() == 0x100
+
+
+@pytest.mark.parametrize("variant,dtype,pre,d,r", [("sliced", "bf16", "bf16", 1024, 16), ("sliced", "f32", "f32", 200, 8),
+                                                   ("projected", "bf16", "f32", 512, 32)])
+def test_phase2_assemble_equals_accumulate_then_phase2(variant, dtype, pre, d, r):
+    """lrar_block_phase2_assemble forms the partial summary (running sum plus
+    the newest member) inside phase 2: the summary it writes over the member,
+    and h and lse, equal bit for bit lrar_block_accumulate followed by
+    lrar_block_phase2 on the same inputs (in place: h is h_pre)."""
+    dev = torch.device("cuda")
+    T = 333
+    sdt, pdt = H.TORCH_DTYPE[dtype], H.TORCH_DTYPE[pre]
+    prev = synth.randn((T, d), 31, "values").to(sdt).to(dev)
+    member = synth.randn((T, d), 32, "values").to(sdt).to(dev)
+    h_pre = synth.randn((T, d), 33, "values").to(pdt).to(dev)
+    lse_pre = (synth.randn((T,), 34, "scale") + 2.0).to(dev)
+    query = synth.queries(1, r, 35, std=0.5)[0].to(dev)
+    pkey = synth.randn((T, r), 36, "keys").to(sdt).to(dev) if variant == "projected" else None
+    mkey = synth.randn((T, r), 37, "keys").to(sdt).to(dev) if variant == "projected" else None
+
+    m_a, h_a, l_a = member.clone(), h_pre.clone(), lse_pre.clone()
+    k_a = mkey.clone() if mkey is not None else None
+    lrar.block_accumulate(m_a, prev, 1.0, 1.0)
+    if k_a is not None:
+        lrar.block_accumulate(k_a, pkey, 1.0, 1.0)
+    lrar.block_phase2(variant, h_a, l_a, m_a, k_a, query, h_a, l_a)
+
+    m_b, h_b, l_b = member.clone(), h_pre.clone(), lse_pre.clone()
+    k_b = mkey.clone() if mkey is not None else None
+    lrar.block_phase2_assemble(variant, h_b, l_b, prev, m_b, pkey, k_b, query, h_b, l_b)
+    torch.cuda.synchronize()
+    assert torch.equal(m_a, m_b)
+    assert torch.equal(h_a, h_b)
+    assert torch.equal(l_a, l_b)
+    if k_a is not None:
+        assert torch.equal(k_a, k_b)
