@@ -254,6 +254,17 @@ def test_fp32_widths(d, variant):
     _check(si, H.run_gpu(si, "f32", "f32"), H.run_oracle(si), si.n, "f32")
 
 
+@pytest.mark.parametrize("n,accumulate", [(1, True), (6, True), (6, False), (12, True)])
+def test_fp32_one_pass_eight_vectors(n, accumulate):
+    """float32 rows of 1024 (eight 16-byte vectors per lane) with the forward's
+    lse: the one-pass sliced kernels at one CTA per SM (accumulating up to 9
+    sources; 12 take the three-stage kernel), held to the float32 bar."""
+    si = synth.site("tiny", variant="sliced", n=n, T=70, d=1024, r=8)
+    init = _init(si) if accumulate else None
+    got = H.run_gpu(si, "f32", "f32", accumulate=accumulate, init=init)
+    _check(si, got, H.run_oracle(si), si.n, "f32", init=init)
+
+
 def test_single_source_is_exact_identity():
     """n = 1 with no query: h = o_0 and dvalues = dh exactly, dq = 0."""
     si = synth.site("slr", n=1, T=100)
