@@ -64,9 +64,9 @@ def test_peaks_measured_or_fallback(tmp_path, monkeypatch):
 
 def test_step_bytes_match_the_per_site_counts():
     """One step: 49 forwards and 49 backwards, the first backward (site 49)
-    writing the gradients and the others accumulating.  The headline site's
-    counts are the survey's: F = 1.678 GB, B = 3.322 GB written / 4.966 GB
-    accumulated (T = 16384, d = 1024, bf16)."""
+    writing the gradients and the others accumulating.  The headline site
+    (n = 49, T = 16384, d = 1024, bf16) moves F = 1.678 GB forward and
+    B = 3.322 GB backward with the gradients written, 4.966 GB accumulated."""
     fwd, bwd = bench.site_bytes()
     assert len(fwd) == len(bwd) == 49
     assert fwd[48] == pytest.approx(1.678e9, rel=1e-3)
