@@ -139,3 +139,32 @@ def test_backward_flags_slots_and_member_hand_over(fake, M, c):
     assert [i for i, _ in order] == list(range(M, -1, -1))
     assert all(gid == id(sw.grads[sites.block_slot(i, c)]) for i, gid in order)
     assert not any(cl[0] == "acc" for cl in fake.calls)  # no fan-out copies when handed over
+
+
+@pytest.mark.parametrize("variant", ["sliced", "projected"])
+def test_depth_sweep_order_sources_and_flags(fake, variant):
+    """sweep.DepthSweep (Full AttnRes over separate source tensors, Eq. 4): site t
+    mixes sources o_0..o_{t-1} with query row t-1 (none at site 1); the backward
+    runs t = n..1, the first call writing every gradient and the rest adding,
+    each over the same prefix of sources (and keys); dq starts from zero."""
+    from paper_2607_09694_gb300.sweep import DepthSweep
+
+    n, T, d, r = 6, 3, 16, 4
+    src = [torch.full((T, d), float(i)) for i in range(n)]
+    keys = [torch.zeros(T, r) for _ in range(n)] if variant == "projected" else None
+    dkeys = [torch.zeros(T, r) for _ in range(n)] if variant == "projected" else None
+    q = torch.randn(n, r)
+    dq = torch.ones(n, r)
+    ds = [torch.zeros(T, d) for _ in range(n)]
+    sw = DepthSweep(variant, src, q, [torch.zeros(T, d)] * n, torch.zeros(n, T, d), torch.zeros(n, T), ds, dq,
+                    keys=keys, dkeys=dkeys, r=r)
+    sw.step(STREAM)
+    fw = [cl for cl in fake.calls if cl[0] == "fwd"]
+    assert [len(cl[1]) for cl in fw] == list(range(1, n + 1))
+    for t, cl in enumerate(fw, start=1):
+        assert [float(v[0, 0]) for v in cl[1]] == [float(i) for i in range(t)]
+    bw = [cl for cl in fake.calls if cl[0] == "bwd"]
+    assert [cl[3] for cl in bw] == list(range(n, 0, -1))
+    assert [cl[2] for cl in bw] == [False] + [True] * (n - 1)
+    assert all(cl[1] == [id(g) for g in ds[:cl[3]]] for cl in bw)
+    assert torch.count_nonzero(dq) == 0
